@@ -1,0 +1,384 @@
+/*
+ * cs_oracle.c -- plain, slow, fp64 CPU oracle for the draft-and-verify step.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
+ * cpu_baseline / reference leg of bench.py may load this library.  It shares
+ * no code, header, table or helper with the CUDA path; the two only see the
+ * same seeded inputs.
+ *
+ * What it computes.  In the paper's cache-miss branch (Sec. 3.4) the target
+ * LLM generates while the small model drafts tokens for it, and the target
+ * verifies them with the standard speculative-sampling draft-and-verify step
+ * (also named in Sec. 2 and App. A.4).  The paper gives no formula of its
+ * own and defers the rule to the two speculative-sampling works it cites;
+ * the rule below is that standard one:
+ *
+ *   1. Verify attention: for each request b, query head h and draft row
+ *      i in [0, k], softmax over keys j <= L_b-(k+1)+i of q.K_j*scale, times V.
+ *      Plain definition written out: scores, max, exp, sum, weighted sum.
+ *   2. Speculative acceptance (temperature T > 0): p_i = softmax(z_t,i / T),
+ *      q_i = softmax(z_d,i / T); accept x_i iff u_i < p_i(x_i)/q_i(x_i);
+ *      a = first rejected position (k if none); on rejection draw from
+ *      max(0, p_a - q_a) normalised, else draw the bonus token from p_k;
+ *      the draw is the inverse CDF in ascending token id with uniform u_k.
+ *   3. Greedy (T == 0): g_i = argmax z_t,i (lowest id on ties); accept x_i
+ *      iff x_i == g_i; emit g_a.
+ *
+ * Every floating-point step is fp64; inputs (bf16 bit patterns or fp32) are
+ * widened exactly.  Loops run in the order the definition states (ascending
+ * key index, ascending token id); OpenMP only splits independent requests /
+ * heads across threads and never changes any sum's order.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define ORC_OK 0
+#define ORC_BAD_ARG 1
+#define ORC_NO_MEM 2
+
+/* bf16 is the upper 16 bits of an IEEE binary32; widening is exact. */
+static double bf16_bits_to_double(uint16_t bits) {
+    uint32_t u = ((uint32_t)bits) << 16;
+    float f;
+    memcpy(&f, &u, sizeof f);
+    return (double)f;
+}
+
+/* Element `idx` of a logit row stored as fp32 (dtype 0) or bf16 (dtype 1). */
+static double logit_at(const void* row, int32_t dtype, int64_t idx) {
+    if (dtype == 0) return (double)((const float*)row)[idx];
+    return bf16_bits_to_double(((const uint16_t*)row)[idx]);
+}
+
+int oracle_max_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+void oracle_set_threads(int n) {
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
+/* ------------------------------------------------------------------------
+ * 1. Verify attention over a paged KV cache.
+ *
+ * q        [B, k+1, Hq, D]   bf16 bits
+ * k_pages  [P, Hkv, ps, D]   bf16 bits
+ * v_pages  [P, Hkv, ps, D]   bf16 bits
+ * page_table [B, max_pages]  int32; key j of request b lives in page
+ *                            page_table[b][j / ps] at slot j % ps
+ * ctx_lens [B]               int32; L_b counts the k+1 verify positions and
+ *                            is clamped to [0, max_pages*ps]
+ * out      [B, k+1, Hq, D]   fp64
+ *
+ * Query head h reads KV head h / G with G = Hq / Hkv (consecutive query
+ * heads share one KV head).  A page id outside [0, P) reads as zeros.
+ * A row with no admissible key (L_b - (k+1) + i < 0) outputs zeros.
+ * scale <= 0 selects 1/sqrt(D).
+ * ---------------------------------------------------------------------- */
+int oracle_verify_attention(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,
+                            int32_t head_dim, int32_t page_size,
+                            int32_t max_pages_per_seq, int32_t num_pages,
+                            double scale, const uint16_t* q,
+                            const uint16_t* k_pages, const uint16_t* v_pages,
+                            const int32_t* page_table, const int32_t* ctx_lens,
+                            int32_t n_draft, double* out) {
+    if (batch < 0 || n_q_heads <= 0 || n_kv_heads <= 0 || head_dim <= 0 ||
+        page_size <= 0 || max_pages_per_seq <= 0 || num_pages < 0 || n_draft < 0)
+        return ORC_BAD_ARG;
+    if (n_q_heads % n_kv_heads != 0) return ORC_BAD_ARG;
+    if (batch == 0) return ORC_OK;
+
+    const int64_t n_rows = (int64_t)n_draft + 1;
+    const int64_t group = n_q_heads / n_kv_heads;
+    const int64_t D = head_dim;
+    const int64_t ps = page_size;
+    const int64_t l_cap = (int64_t)max_pages_per_seq * ps;
+    if (scale <= 0.0) scale = 1.0 / sqrt((double)head_dim);
+
+    int status = ORC_OK;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
+    for (int64_t b = 0; b < batch; ++b) {
+        for (int64_t h = 0; h < n_q_heads; ++h) {
+            int64_t L = ctx_lens[b];
+            if (L < 0) L = 0;
+            if (L > l_cap) L = l_cap;
+            const int64_t kvh = h / group;
+            double* s = (double*)malloc((size_t)(L > 0 ? L : 1) * sizeof(double));
+            double* o = (double*)malloc((size_t)D * sizeof(double));
+            if (!s || !o) {
+#pragma omp atomic write
+                status = ORC_NO_MEM;
+                free(s);
+                free(o);
+                continue;
+            }
+            for (int64_t i = 0; i < n_rows; ++i) {
+                const uint16_t* qv = q + ((b * n_rows + i) * n_q_heads + h) * D;
+                double* dst = out + ((b * n_rows + i) * n_q_heads + h) * D;
+                const int64_t last = L - n_rows + i; /* highest admissible key */
+                if (last < 0) {
+                    for (int64_t d = 0; d < D; ++d) dst[d] = 0.0;
+                    continue;
+                }
+                /* scores s_j = scale * q . K_j, j = 0..last */
+                for (int64_t j = 0; j <= last; ++j) {
+                    const int64_t page = page_table[b * max_pages_per_seq + j / ps];
+                    double dot = 0.0;
+                    if (page >= 0 && page < num_pages) {
+                        const uint16_t* kr =
+                            k_pages + ((page * n_kv_heads + kvh) * ps + j % ps) * D;
+                        for (int64_t d = 0; d < D; ++d)
+                            dot += bf16_bits_to_double(qv[d]) * bf16_bits_to_double(kr[d]);
+                    }
+                    s[j] = scale * dot;
+                }
+                /* stable softmax: max, then exp and sum */
+                double m = s[0];
+                for (int64_t j = 1; j <= last; ++j)
+                    if (s[j] > m) m = s[j];
+                double l = 0.0;
+                for (int64_t j = 0; j <= last; ++j) {
+                    s[j] = exp(s[j] - m);
+                    l += s[j];
+                }
+                for (int64_t d = 0; d < D; ++d) o[d] = 0.0;
+                for (int64_t j = 0; j <= last; ++j) {
+                    const int64_t page = page_table[b * max_pages_per_seq + j / ps];
+                    if (page < 0 || page >= num_pages) continue; /* zero row */
+                    const uint16_t* vr =
+                        v_pages + ((page * n_kv_heads + kvh) * ps + j % ps) * D;
+                    for (int64_t d = 0; d < D; ++d) o[d] += s[j] * bf16_bits_to_double(vr[d]);
+                }
+                for (int64_t d = 0; d < D; ++d) dst[d] = o[d] / l;
+            }
+            free(s);
+            free(o);
+        }
+    }
+    return status;
+}
+
+/* ------------------------------------------------------------------------
+ * 2. Speculative acceptance.
+ * ---------------------------------------------------------------------- */
+
+/* p = softmax(z / T) for one row, T > 0: max, then exp((z-m)/T), then sum,
+ * then divide.  Returns the sum of exponentials (the normaliser). */
+double oracle_row_probs(const void* row, int32_t dtype, int32_t vocab,
+                        double temperature, double* p) {
+    double m = logit_at(row, dtype, 0);
+    for (int64_t v = 1; v < vocab; ++v) {
+        const double z = logit_at(row, dtype, v);
+        if (z > m) m = z;
+    }
+    double S = 0.0;
+    for (int64_t v = 0; v < vocab; ++v) {
+        p[v] = exp((logit_at(row, dtype, v) - m) / temperature);
+        S += p[v];
+    }
+    for (int64_t v = 0; v < vocab; ++v) p[v] /= S;
+    return S;
+}
+
+/* Residual distribution of a rejection: r(v) = max(0, p(v) - q(v)),
+ * Z = sum_v r(v) in ascending v.  Returns Z. */
+double oracle_residual(const double* p, const double* q, int32_t vocab, double* r) {
+    double Z = 0.0;
+    for (int64_t v = 0; v < vocab; ++v) {
+        const double d = p[v] - q[v];
+        r[v] = d > 0.0 ? d : 0.0;
+        Z += r[v];
+    }
+    return Z;
+}
+
+/* Inverse-CDF draw over unnormalised weights r with total Z: the smallest v
+ * whose running sum (ascending v) exceeds u*Z; if rounding leaves none, the
+ * largest v with r(v) > 0.  *margin receives the distance of u from the two
+ * CDF values that bracket the chosen cell, both divided by Z. */
+int32_t oracle_inverse_cdf(const double* r, double Z, int32_t vocab, double u,
+                           double* margin) {
+    const double t = u * Z;
+    double cum = 0.0, before = 0.0;
+    int32_t pick = -1;
+    for (int32_t v = 0; v < vocab; ++v) {
+        before = cum;
+        cum += r[v];
+        if (cum > t) {
+            pick = v;
+            break;
+        }
+    }
+    if (pick < 0) {
+        for (int32_t v = vocab - 1; v >= 0; --v)
+            if (r[v] > 0.0) {
+                pick = v;
+                break;
+            }
+        if (pick < 0) pick = 0; /* all-zero weights cannot arise from a softmax */
+        before = cum;
+    }
+    if (margin) {
+        const double m1 = fabs(u - cum / Z), m0 = fabs(u - before / Z);
+        *margin = m1 < m0 ? m1 : m0;
+    }
+    return pick;
+}
+
+/* argmax with the lowest id on ties. */
+int32_t oracle_row_argmax(const void* row, int32_t dtype, int32_t vocab) {
+    int32_t best = 0;
+    double bv = logit_at(row, dtype, 0);
+    for (int32_t v = 1; v < vocab; ++v) {
+        const double z = logit_at(row, dtype, v);
+        if (z > bv) {
+            bv = z;
+            best = v;
+        }
+    }
+    return best;
+}
+
+/*
+ * target   [B, k+1, V]  fp32 (dtype 0) or bf16 bits (dtype 1)
+ * draft    [B, k,   V]  same dtype; ignored (may be NULL) when T == 0
+ * tokens   [B, k]       int32 draft tokens x_i
+ * uniforms [B, k+1]     fp64 here (the fp32 entry below widens them);
+ *                       u_0..u_{k-1} for the accept tests, u_k for the single
+ *                       final draw (residual or bonus)
+ * out_tokens [B, k+1]   x_0..x_{a-1}, then the drawn token, then -1
+ * out_n_accepted [B]    a
+ * out_margin [B]        (may be NULL) smallest |u - threshold| over every
+ *                       comparison that decided the output: the accept tests
+ *                       of positions 0..a and the two CDF values bracketing
+ *                       the draw.  +inf for greedy (no threshold compare).
+ *
+ * A draft token outside [0, V) counts as rejected (its ratio is 0).
+ */
+int oracle_spec_accept_f64u(int32_t batch, int32_t vocab, int32_t dtype,
+                            const void* target, const void* draft,
+                            const int32_t* tokens, const double* uniforms,
+                            int32_t n_draft, double temperature, int32_t* out_tokens,
+                            int32_t* out_n_accepted, double* out_margin) {
+    if (batch < 0 || vocab <= 0 || n_draft < 0 || (dtype != 0 && dtype != 1))
+        return ORC_BAD_ARG;
+    if (!(temperature >= 0.0)) return ORC_BAD_ARG;
+    if (temperature > 0.0 && n_draft > 0 && !draft) return ORC_BAD_ARG;
+    const int64_t k = n_draft;
+    const int64_t V = vocab;
+    const size_t esz = dtype == 0 ? 4 : 2;
+    int status = ORC_OK;
+
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t b = 0; b < batch; ++b) {
+        const char* trow0 = (const char*)target + (size_t)(b * (k + 1) * V) * esz;
+        const char* drow0 = draft ? (const char*)draft + (size_t)(b * k * V) * esz : NULL;
+        const int32_t* x = tokens + b * k;
+        const double* u = uniforms + b * (k + 1);
+        int32_t* out = out_tokens + b * (k + 1);
+        int64_t a = k;
+        double margin = INFINITY;
+
+        if (temperature == 0.0) {
+            /* greedy: argmax agreement */
+            int32_t g = 0;
+            for (int64_t i = 0; i <= k; ++i) {
+                g = oracle_row_argmax(trow0 + (size_t)(i * V) * esz, dtype, vocab);
+                if (i == k || x[i] != g) {
+                    a = i;
+                    break;
+                }
+            }
+            for (int64_t i = 0; i < a; ++i) out[i] = x[i];
+            out[a] = g;
+        } else {
+            double* p = (double*)malloc((size_t)V * sizeof(double));
+            double* q = (double*)malloc((size_t)V * sizeof(double));
+            double* r = (double*)malloc((size_t)V * sizeof(double));
+            if (!p || !q || !r) {
+#pragma omp atomic write
+                status = ORC_NO_MEM;
+                free(p);
+                free(q);
+                free(r);
+                continue;
+            }
+            /* accept tests, in order, until the first rejection */
+            for (int64_t i = 0; i < k; ++i) {
+                oracle_row_probs(trow0 + (size_t)(i * V) * esz, dtype, vocab, temperature, p);
+                oracle_row_probs(drow0 + (size_t)(i * V) * esz, dtype, vocab, temperature, q);
+                double ratio = 0.0;
+                if (x[i] >= 0 && x[i] < vocab)
+                    ratio = q[x[i]] > 0.0 ? p[x[i]] / q[x[i]] : INFINITY;
+                const double gap = fabs(u[i] - ratio);
+                if (gap < margin) margin = gap;
+                if (!(u[i] < ratio)) {
+                    a = i;
+                    break;
+                }
+            }
+            double Z;
+            if (a < k) {
+                /* p and q still hold row a */
+                Z = oracle_residual(p, q, vocab, r);
+                if (!(Z > 0.0)) { /* p == q up to rounding: fall back to p */
+                    Z = 0.0;
+                    for (int64_t v = 0; v < V; ++v) {
+                        r[v] = p[v];
+                        Z += r[v];
+                    }
+                }
+            } else {
+                oracle_row_probs(trow0 + (size_t)(k * V) * esz, dtype, vocab, temperature, p);
+                Z = 0.0;
+                for (int64_t v = 0; v < V; ++v) {
+                    r[v] = p[v];
+                    Z += r[v];
+                }
+            }
+            double dm = INFINITY;
+            const int32_t pick = oracle_inverse_cdf(r, Z, vocab, u[k], &dm);
+            if (dm < margin) margin = dm;
+            for (int64_t i = 0; i < a; ++i) out[i] = x[i];
+            out[a] = pick;
+            free(p);
+            free(q);
+            free(r);
+        }
+        for (int64_t i = a + 1; i <= k; ++i) out[i] = -1;
+        out_n_accepted[b] = (int32_t)a;
+        if (out_margin) out_margin[b] = margin;
+    }
+    return status;
+}
+
+/* The library's own uniform type is fp32; widen exactly and run the core. */
+int oracle_spec_accept(int32_t batch, int32_t vocab, int32_t dtype,
+                       const void* target, const void* draft,
+                       const int32_t* tokens, const float* uniforms,
+                       int32_t n_draft, double temperature, int32_t* out_tokens,
+                       int32_t* out_n_accepted, double* out_margin) {
+    if (batch < 0 || n_draft < 0) return ORC_BAD_ARG;
+    const size_t n = (size_t)batch * (size_t)(n_draft + 1);
+    double* u = (double*)malloc((n ? n : 1) * sizeof(double));
+    if (!u) return ORC_NO_MEM;
+    for (size_t i = 0; i < n; ++i) u[i] = (double)uniforms[i];
+    const int rc = oracle_spec_accept_f64u(batch, vocab, dtype, target, draft, tokens, u,
+                                           n_draft, temperature, out_tokens,
+                                           out_n_accepted, out_margin);
+    free(u);
+    return rc;
+}
