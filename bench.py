@@ -1,0 +1,498 @@
+#!/usr/bin/env python3
+"""Benchmark of the draft-and-verify step on GB300.
+
+One step = one pass of the whole hot path over one batch of synthetic input:
+cs_verify_attention (one layer's verify attention over the paged KV cache)
+followed by cs_spec_accept (the acceptance step at the workload's sampling
+temperature).  The metric is verified draft tokens per second (B*k per step)
+with the achieved HBM bandwidth of the dominant kernel against the measured
+copy peak.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 2] [--impl gb300|reference]
+
+Under torchrun (N > 1) every rank runs an independent replica on its own GPU
+with its own requests (the step shards by request; there is no collective on
+the data path): value = requests*k over all ranks / max-over-ranks time.
+``--impl reference`` times the fp64 CPU oracle on the host cores instead (a
+deliberately slow baseline; rank 0 only).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2607_20507_gb300 import workloads as W  # noqa: E402
+
+METRIC = "verified draft tokens/sec and achieved HBM GB/s (fraction of ~8 TB/s) at 1 GB300"
+UNIT = "verified draft tokens/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_FLUSH_BYTES = 512 << 20
+KERNEL_SOURCES = ("paper_2607_20507_gb300/csrc/verify_attention.cu",
+                  "paper_2607_20507_gb300/csrc/spec_accept.cu",
+                  "paper_2607_20507_gb300/csrc/cs_device.cuh")
+
+
+# --------------------------------------------------------------------------
+# helpers that need no GPU (covered by the CPU tests)
+# --------------------------------------------------------------------------
+
+def dist_env() -> tuple[int, int, int]:
+    return (int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def replica_workload(w: W.Workload, rank: int) -> W.Workload:
+    """Rank r's replica: same shapes, its own seeded requests."""
+    return w if rank == 0 else w.with_(cell=w.cell + 7919 * rank)
+
+
+def reduce_max(x: float, device) -> float:
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_throughput(units_per_rank: float, seconds: float, world: int, device) -> tuple[float, float]:
+    """(whole-job units/s, max-over-ranks seconds): every rank did `units_per_rank`."""
+    t = reduce_max(seconds, device)
+    return units_per_rank * world / t, t
+
+
+def attention_bytes(ctx_lens: np.ndarray, w: W.Workload) -> int:
+    """Algorithmic HBM bytes of one verify-attention call: every admissible K and
+    V row once, Q read and out written once, the used page-table entries and
+    the context lengths."""
+    kv = int(ctx_lens.astype(np.int64).sum()) * 2 * w.n_kv_heads * w.head_dim * 2
+    qo = 2 * w.batch * (w.n_draft + 1) * w.n_q_heads * w.head_dim * 2
+    pages = int(np.ceil(ctx_lens / w.page_size).sum()) * 4
+    return kv + qo + pages + 4 * w.batch
+
+
+def attention_flops(ctx_lens: np.ndarray, w: W.Workload) -> int:
+    k = w.n_draft
+    keys = sum(int(L) * (k + 1) - k * (k + 1) // 2 for L in ctx_lens.tolist())
+    return 4 * w.n_q_heads * w.head_dim * keys
+
+
+def accept_bytes(n_accepted: np.ndarray, w: W.Workload, T: float) -> tuple[int, int]:
+    """(bytes the method must read, bytes of every row) for one acceptance call.
+
+    Sampling: target and draft rows 0..a, plus target row k when a == k.
+    Greedy: target rows 0..a.  Rows after the first rejection cannot change
+    the result.  Small per-request arrays (tokens, uniforms, outputs) added."""
+    s = 4 if w.logit_dtype == "f32" else 2
+    k, V, B = w.n_draft, w.vocab, w.batch
+    a = n_accepted.astype(np.int64)
+    if T > 0:
+        rows = np.where(a < k, 2 * (a + 1), 2 * k + 1)
+        full = B * (2 * k + 1)
+    else:
+        rows = a + 1
+        full = B * (k + 1)
+    small = B * k * 4 + B * (k + 1) * 4 + B * (k + 1) * 4 + B * 4
+    return int(rows.sum()) * V * s + small, full * V * s + small
+
+
+def measured_peaks() -> tuple[dict, str]:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return json.load(f), "of measured"
+    except Exception:
+        return {"hbm_gbs": FALLBACK_HBM_GBS}, "of fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str, workload: str) -> int | None:
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current kernel sources; otherwise None."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(p) as f:
+            rec = json.load(f)
+    except Exception:
+        return None
+    e = rec.get(kernel, {}).get(workload)
+    if not e or e.get("source_hash") != kernel_source_hash():
+        return None
+    return int(e["dram_bytes_per_launch"])
+
+
+def parse_clocks(lines: list[str]) -> dict:
+    sm, mx, reasons = [], [], set()
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    for ln in lines:
+        f = [x.strip() for x in ln.split(",")]
+        if len(f) < 9 or not f[1].replace(".", "").isdigit():
+            continue
+        sm.append(float(f[1]))
+        mx.append(float(f[2]))
+        for name, val in zip(names, f[5:9]):
+            if val.lower() == "active":
+                reasons.add(name)
+    if not sm:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+    return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+            "samples": len(sm)}
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons while the GPU works."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        self.lines: list[str] = []
+        sel = []
+        try:
+            uuid = str(torch.cuda.get_device_properties(device_index).uuid)
+            sel = ["-i", uuid if uuid.startswith("GPU-") else "GPU-" + uuid]
+        except Exception:
+            sel = []
+        self.cmd = ["nvidia-smi", *sel, f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                    "-lms", "100"]
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+                self.lines = out.splitlines()
+            except Exception:
+                self.proc.kill()
+        return False
+
+    def summary(self) -> dict:
+        return parse_clocks(self.lines)
+
+
+# --------------------------------------------------------------------------
+# the GB300 arm
+# --------------------------------------------------------------------------
+
+def run_gb300(args) -> dict | None:
+    import torch.distributed as dist
+    from paper_2607_20507_gb300 import binding
+
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    binding.load_library()
+
+    w = replica_workload(W.WORKLOADS[args.workload], rank)
+    T = args.temperature if args.temperature is not None else max(w.temperatures)
+    att = W.attention_inputs(w, dev)
+    acc = W.accept_inputs(w, T, dev)
+    acc_greedy = W.accept_inputs(w, 0.0, dev) if 0.0 in w.temperatures else None
+    k, B = w.n_draft, w.batch
+    ws = binding.verify_attention_workspace(binding.attn_dims(att["q"], att["k_pages"], att["page_table"]),
+                                            k, dev)
+    out = torch.empty_like(att["q"])
+    out_tok = torch.empty((B, k + 1), dtype=torch.int32, device=dev)
+    out_n = torch.empty((B,), dtype=torch.int32, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def attention():
+        binding.cs_verify_attention(att["q"], att["k_pages"], att["v_pages"], att["page_table"],
+                                    att["ctx_lens"], k, out=out, workspace=ws)
+
+    def accept(inp, temp):
+        binding.cs_spec_accept(inp["target"], inp["draft"] if temp > 0 else None,
+                               inp["draft_tokens"], inp["uniforms"], temp, out_tok, out_n)
+
+    def step():
+        attention()
+        accept(acc, T)
+
+    # warm-up: at least W steps and about a second of work, with clocks sampled
+    sampler = ClockSampler(local)
+    with sampler:
+        t0 = time.time()
+        n = 0
+        while n < args.warmup or time.time() - t0 < 1.0:
+            flush.zero_()
+            step()
+            n += 1
+            if n % 64 == 0:
+                torch.cuda.synchronize()
+        torch.cuda.synchronize()
+
+        # timed region: exactly K steps, L2 flushed between steps (outside the events)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+               torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        for e0, e1, e2 in ev:
+            flush.zero_()
+            e0.record(stream)
+            attention()
+            e1.record(stream)
+            accept(acc, T)
+            e2.record(stream)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+    t_attn = [e0.elapsed_time(e1) * 1e-3 for e0, e1, _ in ev]
+    t_acc = [e1.elapsed_time(e2) * 1e-3 for _, e1, e2 in ev]
+    t_step = [a + b for a, b in zip(t_attn, t_acc)]
+    value, t_max = aggregate_throughput(float(B * k * args.steps), sum(t_step), world, dev)
+    n_acc = out_n.cpu().numpy()
+
+    # greedy mode of the same workload (its temperature list names it)
+    greedy = None
+    if acc_greedy is not None:
+        evg = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        for _ in range(3):
+            accept(acc_greedy, 0.0)
+        for e0, e1 in evg:
+            flush.zero_()
+            e0.record(stream)
+            accept(acc_greedy, 0.0)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        tg = [e0.elapsed_time(e1) * 1e-3 for e0, e1 in evg]
+        ng = out_n.cpu().numpy()
+        gb, gfull = accept_bytes(ng, w, 0.0)
+        greedy = {"accept_us": 1e6 * statistics.mean(tg), "mean_accepted": float(ng.mean()),
+                  "needed_gbs": gb / statistics.mean(tg) / 1e9, "all_rows_gbs": gfull / statistics.mean(tg) / 1e9}
+
+    # end to end through the public API: inputs start in pinned host memory
+    host = {name: t.cpu().pin_memory() for name, t in
+            list(att.items()) + list(acc.items()) if isinstance(t, torch.Tensor)}
+    dev_bufs = {name: (att.get(name) if name in att else acc[name]) for name in host}
+    h2d = sum(t.numel() * t.element_size() for t in host.values())
+    res_host = (torch.empty((B, k + 1), dtype=torch.int32).pin_memory(),
+                torch.empty((B,), dtype=torch.int32).pin_memory())
+    d2h = sum(t.numel() * t.element_size() for t in res_host)
+
+    def e2e_step():
+        for name, t in host.items():
+            dev_bufs[name].copy_(t, non_blocking=True)
+        step()
+        res_host[0].copy_(out_tok, non_blocking=True)
+        res_host[1].copy_(out_n, non_blocking=True)
+
+    for _ in range(max(3, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e_start, e_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e_start.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e_end.record(stream)
+    torch.cuda.synchronize()
+    e2e_value, _ = aggregate_throughput(float(B * k * args.steps), e_start.elapsed_time(e_end) * 1e-3,
+                                        world, dev)
+
+    # roofline of the dominant kernel (the one with the larger share of the step)
+    lens = att["ctx_lens"].cpu().numpy()
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    ab = attention_bytes(lens, w)
+    acc_need, acc_full = accept_bytes(n_acc, w, T)
+    m_attn, m_acc = statistics.mean(t_attn), statistics.mean(t_acc)
+    kernels = {
+        "verify_attention": {"us": 1e6 * m_attn, "bytes": ab, "gbs": ab / m_attn / 1e9,
+                             "tflops": attention_flops(lens, w) / m_attn / 1e12},
+        "spec_accept": {"us": 1e6 * m_acc, "needed_bytes": acc_need, "all_rows_bytes": acc_full,
+                        "gbs": acc_need / m_acc / 1e9, "all_rows_gbs": acc_full / m_acc / 1e9,
+                        "mean_accepted": float(n_acc.mean())},
+    }
+    dom = "verify_attention" if m_attn >= m_acc else "spec_accept"
+    dom_bytes = ab if dom == "verify_attention" else acc_need
+    dom_t = m_attn if dom == "verify_attention" else m_acc
+    achieved = dom_bytes / dom_t / 1e9
+    roofline = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
+                "unit": "GB/s", "frac": round(achieved / hbm_peak, 4), "peak_source": peak_src,
+                "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
+                "traffic": recorded_traffic(dom, w.name)}
+
+    result = None
+    if rank == 0:
+        cpu = None if args.no_cpu_baseline else oracle_baseline(w, T, att, acc, seconds_budget=20.0)
+        result = {
+            "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * t_max / args.steps, 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "dtype_detail": "bf16 tensor-core attention with fp32 softmax and accumulation; fp32 acceptance arithmetic",
+            "data": "synthetic (seeded; shapes of the serving workload, no dataset or weights)",
+            "config": {"workload": w.name, "batch_per_gpu": B, "n_draft": k, "vocab": w.vocab,
+                       "logit_dtype": w.logit_dtype, "temperature": T, "draft_sigma": w.draft_sigma,
+                       "n_q_heads": w.n_q_heads, "n_kv_heads": w.n_kv_heads, "head_dim": w.head_dim,
+                       "page_size": w.page_size, "ctx": list(w.ctx), "mean_ctx": float(lens.mean()),
+                       "l2": "flushed between steps (512 MiB memset outside the timed events)",
+                       "parallelism": f"replicas x{world} (requests shard; no collective)"},
+            "kernels": kernels,
+            "greedy": greedy,
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h,
+                    "note": "host->device copy of every input from pinned memory and device->host "
+                            "read of the emitted tokens inside the timed region"},
+            "gpu_launches": 2 * args.steps * math.ceil(B / 65535),
+            "clocks": sampler.summary() | {"window": "warm-up (>= 1 s) and the timed steps"},
+        }
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+    return result
+
+
+def oracle_baseline(w, T, att, acc, seconds_budget=20.0) -> dict:
+    """The fp64 oracle on the host cores over a bounded sample of the workload."""
+    import oracle
+    cores = os.cpu_count() or 1
+    oracle.set_threads(cores)
+    B = w.batch
+    # grow the request sample until the budget is used (at least one request)
+    n = 1
+    spent = 0.0
+    done = 0
+    rng = np.random.default_rng(0)
+    order = rng.permutation(B)
+    while done < B and spent < seconds_budget:
+        take = order[done:done + n].tolist()
+        sa = W.attention_subset(att, take)
+        sc = W.accept_subset(acc, take)
+        a_host = (W.host_bits(sa["q"]), W.host_bits(sa["k_pages"]), W.host_bits(sa["v_pages"]),
+                  sa["page_table"].cpu().numpy(), sa["ctx_lens"].cpu().numpy())
+        c_host = (W.host_bits(sc["target"]), W.host_bits(sc["draft"]) if T > 0 else None,
+                  sc["draft_tokens"].cpu().numpy(), sc["uniforms"].cpu().numpy())
+        t0 = time.perf_counter()
+        oracle.verify_attention(*a_host, w.n_draft)
+        oracle.spec_accept(*c_host, T)
+        spent += time.perf_counter() - t0
+        done += len(take)
+        n = min(2 * n, B - done) if done < B else n
+    value = done * w.n_draft / spent
+    return {"value": round(value, 2), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{done} of {B} requests of {w.name} (attention + acceptance, fp64, "
+                      f"OpenMP over requests/heads), {spent:.2f} s"}
+
+
+# --------------------------------------------------------------------------
+# the reference arm: the oracle as it stands, on the host cores
+# --------------------------------------------------------------------------
+
+def run_reference(args) -> dict | None:
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return None
+    import oracle
+    w = W.WORKLOADS[args.workload]
+    T = args.temperature if args.temperature is not None else max(w.temperatures)
+    cores = os.cpu_count() or 1
+    oracle.set_threads(cores)
+    att = W.attention_inputs(w, "cpu")
+    acc = W.accept_inputs(w, T, "cpu")
+    # each step is a bounded sample: as many requests as fit about 2 s of oracle work
+    take = list(range(w.batch))
+    probe = W.attention_subset(att, take[:1])
+    ph = (W.host_bits(probe["q"]), W.host_bits(probe["k_pages"]), W.host_bits(probe["v_pages"]),
+          probe["page_table"].numpy(), probe["ctx_lens"].numpy())
+    t0 = time.perf_counter()
+    oracle.verify_attention(*ph, w.n_draft)
+    per_req = max(time.perf_counter() - t0, 1e-4)
+    n_req = max(1, min(w.batch, int(2.0 / per_req)))
+    sa = W.attention_subset(att, take[:n_req])
+    sc = W.accept_subset(acc, take[:n_req])
+    a_host = (W.host_bits(sa["q"]), W.host_bits(sa["k_pages"]), W.host_bits(sa["v_pages"]),
+              sa["page_table"].numpy(), sa["ctx_lens"].numpy())
+    c_host = (W.host_bits(sc["target"]), W.host_bits(sc["draft"]) if T > 0 else None,
+              sc["draft_tokens"].numpy(), sc["uniforms"].numpy())
+
+    def step():
+        oracle.verify_attention(*a_host, w.n_draft)
+        oracle.spec_accept(*c_host, T)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        step()
+        times.append(time.perf_counter() - t0)
+    total = sum(times)
+    value = n_req * w.n_draft * args.steps / total
+    sample = (f"{n_req} of {w.batch} requests of {w.name} per step (attention + acceptance, fp64, "
+              f"OpenMP on {cores} host threads)")
+    return {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded; shapes of the serving workload)",
+            "config": {"workload": w.name, "batch_per_gpu": w.batch, "n_draft": w.n_draft,
+                       "vocab": w.vocab, "temperature": T},
+            "cpu_baseline": {"value": round(value, 3), "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": round(value, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+def main(argv=None) -> int:
+    ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", type=int, default=2, choices=sorted(W.WORKLOADS))
+    ap.add_argument("--temperature", type=float, default=None)
+    ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    args.warmup = max(3, args.warmup)
+    args.steps = max(1, args.steps)
+    res = run_reference(args) if args.impl == "reference" else run_gb300(args)
+    if res is not None:
+        print(json.dumps(res), flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,179 @@
+/*
+ * cachespec.h -- C ABI of libcachespec.so: the draft-and-verify step of
+ * speculative sampling on one GB300 (sm_103a).
+ *
+ * The paper's cache-miss branch (Sec. 3.4) runs the target LLM with the small
+ * model as speculative drafter: the drafter proposes k tokens, the target
+ * scores the k+1 positions in one pass, and the standard speculative-sampling
+ * rule of the works the paper cites (Sec. 2, Sec. 3.4, App. A.4) accepts,
+ * corrects or extends the draft.  This library implements the two
+ * data-parallel operations of that step:
+ *
+ *   cs_verify_attention -- the KV-bound core of the target's verify pass:
+ *                          multi-query GQA attention of the k+1 positions
+ *                          over each request's paged KV cache, causal among
+ *                          the drafted tokens;
+ *   cs_spec_accept      -- the acceptance step: temperature softmax of target
+ *                          and draft logits, accept test, residual / bonus
+ *                          draw by inverse CDF, and its greedy variant.
+ *
+ * Conventions for every entry point
+ *   - All tensor arguments are DEVICE pointers owned by the caller, dense
+ *     row-major in the layouts stated below.  The library never allocates,
+ *     frees or synchronises (except cs_read_device_status, which says so).
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL is the legacy
+ *     default stream) and return once the work is enqueued.
+ *   - Arguments are checked on the host before anything is enqueued; a bad
+ *     argument returns an error code and enqueues nothing.  Values that live
+ *     in device memory (context lengths, page ids, token ids) cannot be
+ *     checked on the host; their out-of-range behaviour is defined per call.
+ *   - On any status other than CS_OK, cs_last_error() returns a message for
+ *     the calling thread.
+ */
+#ifndef CACHESPEC_H
+#define CACHESPEC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st* cs_stream_t;
+
+typedef enum {
+    CS_OK = 0,
+    CS_ERR_INVALID_ARG = 1,   /* a dimension, pointer, alignment or scalar is invalid */
+    CS_ERR_UNSUPPORTED = 2,   /* valid, but outside what these kernels implement */
+    CS_ERR_CUDA = 3,          /* the CUDA runtime or driver reported an error */
+    CS_ERR_WORKSPACE = 4      /* workspace missing or smaller than the query says */
+} cs_status;
+
+typedef enum { CS_F32 = 0, CS_BF16 = 1 } cs_dtype;
+
+/* Geometry of one verify-attention call. */
+typedef struct {
+    int32_t batch;              /* B >= 0 requests (0: nothing to do) */
+    int32_t n_q_heads;          /* Hq > 0 query heads */
+    int32_t n_kv_heads;         /* Hkv > 0 KV heads, Hq % Hkv == 0; G = Hq / Hkv */
+    int32_t head_dim;           /* D; this build implements D == 128 */
+    int32_t page_size;          /* ps tokens per page: 8, 16, 32, 64, 128 or 256 */
+    int32_t max_pages_per_seq;  /* columns of page_table (> 0) */
+    int32_t num_pages;          /* P pages in the pool (> 0) */
+    float sm_scale;             /* softmax scale; <= 0 selects 1/sqrt(D) */
+} cs_attn_dims;
+
+/* Geometry of one acceptance call. */
+typedef struct {
+    int32_t batch;              /* B >= 0 requests (0: nothing to do) */
+    int32_t vocab;              /* V > 0 */
+    int32_t logit_dtype;        /* cs_dtype of target and draft logits */
+} cs_accept_dims;
+
+/* ABI version of this header (bumped on any incompatible change). */
+#define CS_ABI_VERSION 1
+int32_t cs_abi_version(void);
+
+/* Message describing the last non-OK status returned on this thread. */
+const char* cs_last_error(void);
+
+/*
+ * Verify attention (the target's attention over the k+1 verify positions,
+ * Sec. 3.4's verify pass).
+ *
+ * For every request b, query head h and draft row i in [0, k]:
+ *     out[b,i,h,:] = softmax_j( sm_scale * q[b,i,h,:] . K_j ) V_j
+ * over the keys j = 0 .. L_b-(k+1)+i of KV head h / G: each drafted
+ * position sees the whole prefix and the drafts before it.  Key j of
+ * request b is slot j % ps of page page_table[b][j / ps].
+ *
+ *   q          bf16 [B, k+1, Hq, D]
+ *   k_pages    bf16 [P, Hkv, ps, D]   16-byte aligned
+ *   v_pages    bf16 [P, Hkv, ps, D]   16-byte aligned
+ *   page_table int32 [B, max_pages_per_seq]; entries past the last page of a
+ *              request are never read
+ *   ctx_lens   int32 [B]; L_b counts the k+1 verify positions
+ *   n_draft    k in [1, 16]; (k+1)*G must not exceed 144
+ *   out        bf16 [B, k+1, Hq, D] (must not alias the inputs)
+ *   workspace  device scratch of at least
+ *              cs_verify_attention_workspace_bytes(dims, k) bytes, 256-byte
+ *              aligned, ZERO-FILLED before its first use; every call that
+ *              completes leaves it ready for the next call.  Calls that share
+ *              a workspace must be ordered (same stream or events).  May be
+ *              NULL when the query returns 0.
+ *
+ * Defined behaviour for device-resident values: L_b is clamped to
+ * [0, max_pages_per_seq*ps]; a row with no admissible key
+ * (L_b-(k+1)+i < 0) outputs zeros; a page id outside [0, P) reads as zeros.
+ * Pool slots past L_b may hold any bits (including NaN); they never reach
+ * the output.
+ *
+ * Returns CS_ERR_INVALID_ARG (null pointer, misalignment, bad dimension, NaN
+ * scale, n_draft out of range), CS_ERR_UNSUPPORTED (D != 128, page size,
+ * (k+1)*G > 144), CS_ERR_WORKSPACE, or CS_ERR_CUDA (launch failure).
+ */
+size_t cs_verify_attention_workspace_bytes(const cs_attn_dims* dims, int32_t n_draft);
+cs_status cs_verify_attention(const cs_attn_dims* dims, const void* q, const void* k_pages,
+                              const void* v_pages, const int32_t* page_table,
+                              const int32_t* ctx_lens, int32_t n_draft, void* out,
+                              void* workspace, size_t workspace_bytes, cs_stream_t stream);
+
+/*
+ * Speculative acceptance (the accept / correct / extend rule of the
+ * speculative sampling the paper's drafter follows, Sec. 3.4; temperature 0
+ * is the greedy mode of the paper's App. B runs).
+ *
+ * Temperature T > 0, for each request b:
+ *   p_i = softmax(target[b,i,:] / T) for i in [0, k];
+ *   q_i = softmax(draft[b,i,:] / T)  for i in [0, k);
+ *   position i accepts x_i = draft_tokens[b,i] iff u_i < p_i(x_i) / q_i(x_i);
+ *   a = the first rejected position, or k if none is rejected;
+ *   if a < k the emitted token is drawn from max(0, p_a - q_a) normalised,
+ *   else (the bonus token) from p_k, in both cases as the smallest token id
+ *   whose running mass (ascending ids) exceeds u_k times the total.
+ * Temperature 0 (greedy): g_i = argmax target[b,i,:] (lowest id on ties);
+ *   position i accepts iff x_i == g_i; the emitted token is g_a.
+ *
+ *   target_logits  [B, k+1, V] fp32 or bf16 (dims->logit_dtype), element-aligned
+ *   draft_logits   [B, k,   V] same dtype; may be NULL when temperature == 0
+ *   draft_tokens   int32 [B, k]; an id outside [0, V) is rejected at its position
+ *   uniforms       fp32 [B, k+1] in [0, 1): u_0..u_{k-1} for the accept tests,
+ *                  u_k for the single final draw
+ *   n_draft        k in [1, 16]
+ *   temperature    T >= 0 and finite
+ *   out_tokens     int32 [B, k+1]: x_0..x_{a-1}, the emitted token, then -1
+ *   out_n_accepted int32 [B]: a
+ *   workspace      device scratch of cs_spec_accept_workspace_bytes(dims, k)
+ *                  bytes (this build needs none; NULL is accepted)
+ *
+ * Logits must be finite.  Rows after the first rejection are not read: they
+ * cannot change the result.  The result is a deterministic function of the
+ * inputs.
+ *
+ * Returns CS_ERR_INVALID_ARG (null pointer, misalignment, bad dimension,
+ * bad temperature, n_draft out of range), CS_ERR_WORKSPACE or CS_ERR_CUDA.
+ */
+size_t cs_spec_accept_workspace_bytes(const cs_accept_dims* dims, int32_t n_draft);
+cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
+                         const void* draft_logits, const int32_t* draft_tokens,
+                         const float* uniforms, int32_t n_draft, float temperature,
+                         int32_t* out_tokens, int32_t* out_n_accepted, void* workspace,
+                         size_t workspace_bytes, cs_stream_t stream);
+
+/*
+ * Device status word of a verify-attention workspace: 0 when every call that
+ * used it finished normally; otherwise a bit set of CS_DEVICE_* flags (a
+ * bounded wait inside a kernel gave up, so that call's output is invalid).
+ * Copies 4 bytes to the host and SYNCHRONISES `stream`.  The word is sticky
+ * until the caller zero-fills the workspace again.
+ */
+#define CS_DEVICE_WAIT_TIMEOUT 1
+cs_status cs_read_device_status(const void* workspace, int32_t* status_out, cs_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CACHESPEC_H */

@@ -1,0 +1,208 @@
+"""Python binding of libcachespec.so: the same entry points, argument marshalling only.
+
+Every step of the draft-and-verify path runs in the library's CUDA kernels;
+this module checks tensor dtypes, shapes and devices, passes raw device
+pointers and the current CUDA stream through ctypes, and turns a non-OK
+status into an exception.  It never computes any part of the method and has
+no CPU fallback: if the library is missing, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import build as _build
+
+CS_OK, CS_ERR_INVALID_ARG, CS_ERR_UNSUPPORTED, CS_ERR_CUDA, CS_ERR_WORKSPACE = range(5)
+CS_F32, CS_BF16 = 0, 1
+STATUS_NAMES = {0: "CS_OK", 1: "CS_ERR_INVALID_ARG", 2: "CS_ERR_UNSUPPORTED", 3: "CS_ERR_CUDA",
+                4: "CS_ERR_WORKSPACE"}
+EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_workspace_bytes",
+                    "cs_verify_attention", "cs_spec_accept_workspace_bytes", "cs_spec_accept",
+                    "cs_read_device_status")
+
+
+class AttnDims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("page_size", ctypes.c_int32), ("max_pages_per_seq", ctypes.c_int32),
+                ("num_pages", ctypes.c_int32), ("sm_scale", ctypes.c_float)]
+
+
+class AcceptDims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("logit_dtype", ctypes.c_int32)]
+
+
+class CacheSpecError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load_library(path: str | None = None):
+    """Load libcachespec.so (built in-tree by ``__graft_entry__.build()``).  Raises if absent."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or _build.LIB
+        if not os.path.exists(p):
+            raise RuntimeError(f"libcachespec.so not found at {p}; build it with "
+                               "`python -c 'import __graft_entry__ as g; g.build()'`")
+        lib = ctypes.CDLL(p)
+        vp, i32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+        lib.cs_abi_version.restype = i32
+        lib.cs_last_error.restype = ctypes.c_char_p
+        lib.cs_verify_attention_workspace_bytes.restype = sz
+        lib.cs_verify_attention_workspace_bytes.argtypes = [ctypes.POINTER(AttnDims), i32]
+        lib.cs_verify_attention.restype = ctypes.c_int
+        lib.cs_verify_attention.argtypes = [ctypes.POINTER(AttnDims), vp, vp, vp, vp, vp, i32, vp,
+                                            vp, sz, vp]
+        lib.cs_spec_accept_workspace_bytes.restype = sz
+        lib.cs_spec_accept_workspace_bytes.argtypes = [ctypes.POINTER(AcceptDims), i32]
+        lib.cs_spec_accept.restype = ctypes.c_int
+        lib.cs_spec_accept.argtypes = [ctypes.POINTER(AcceptDims), vp, vp, vp, vp, i32,
+                                       ctypes.c_float, vp, vp, vp, sz, vp]
+        lib.cs_read_device_status.restype = ctypes.c_int
+        lib.cs_read_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_int32), vp]
+        if path is None:
+            _lib = lib
+        return lib
+
+
+def _check(lib, status: int) -> None:
+    if status != CS_OK:
+        raise CacheSpecError(status, lib.cs_last_error().decode(errors="replace"))
+
+
+def _ptr(t: torch.Tensor | None) -> int | None:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(device: torch.device) -> int:
+    return torch.cuda.current_stream(device).cuda_stream
+
+
+def _need(t: torch.Tensor, name: str, dtype: torch.dtype, ndim: int, device) -> None:
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if t.dim() != ndim:
+        raise ValueError(f"{name} must have {ndim} dims, got shape {tuple(t.shape)}")
+    if not t.is_cuda or (device is not None and t.device != device):
+        raise ValueError(f"{name} must live on {device or 'a CUDA device'}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def attn_dims(q: torch.Tensor, k_pages: torch.Tensor, page_table: torch.Tensor,
+              sm_scale: float = 0.0) -> AttnDims:
+    B, _, Hq, D = q.shape
+    P, Hkv, ps, _ = k_pages.shape
+    return AttnDims(B, Hq, Hkv, D, ps, page_table.shape[1], P, float(sm_scale))
+
+
+# Workspaces handed out by this module, one per (device, size).  The kernels
+# leave a workspace ready for the next call, so calls ordered on one stream
+# may share it.
+_workspaces: dict = {}
+
+
+def verify_attention_workspace(dims: AttnDims, n_draft: int, device) -> torch.Tensor:
+    lib = load_library()
+    n = lib.cs_verify_attention_workspace_bytes(ctypes.byref(dims), int(n_draft))
+    key = (str(device), n)
+    ws = _workspaces.get(key)
+    if ws is None:
+        ws = torch.zeros(max(n, 256), dtype=torch.uint8, device=device)
+        _workspaces[key] = ws
+    return ws
+
+
+def cs_verify_attention_workspace_bytes(q, k_pages, page_table, n_draft, sm_scale=0.0) -> int:
+    lib = load_library()
+    d = attn_dims(q, k_pages, page_table, sm_scale)
+    return int(lib.cs_verify_attention_workspace_bytes(ctypes.byref(d), int(n_draft)))
+
+
+def cs_verify_attention(q, k_pages, v_pages, page_table, ctx_lens, n_draft, out=None,
+                        workspace=None, sm_scale: float = 0.0, stream: int | None = None):
+    """Verify attention; returns ``out`` (bf16 [B, k+1, Hq, D]).  See include/cachespec.h."""
+    lib = load_library()
+    dev = q.device
+    _need(q, "q", torch.bfloat16, 4, dev)
+    _need(k_pages, "k_pages", torch.bfloat16, 4, dev)
+    _need(v_pages, "v_pages", torch.bfloat16, 4, dev)
+    _need(page_table, "page_table", torch.int32, 2, dev)
+    _need(ctx_lens, "ctx_lens", torch.int32, 1, dev)
+    if v_pages.shape != k_pages.shape:
+        raise ValueError("k_pages and v_pages must have the same shape")
+    if q.shape[1] != n_draft + 1:
+        raise ValueError(f"q has {q.shape[1]} rows per request, n_draft+1 = {n_draft + 1}")
+    d = attn_dims(q, k_pages, page_table, sm_scale)
+    if out is None:
+        out = torch.empty_like(q)
+    else:
+        _need(out, "out", torch.bfloat16, 4, dev)
+    if workspace is None:
+        workspace = verify_attention_workspace(d, n_draft, dev)
+    st = lib.cs_verify_attention(ctypes.byref(d), _ptr(q), _ptr(k_pages), _ptr(v_pages),
+                                 _ptr(page_table), _ptr(ctx_lens), int(n_draft), _ptr(out),
+                                 _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                 _stream(dev) if stream is None else stream)
+    _check(lib, st)
+    return out
+
+
+def cs_spec_accept(target_logits, draft_logits, draft_tokens, uniforms, temperature,
+                   out_tokens=None, out_n_accepted=None, stream: int | None = None):
+    """Speculative acceptance; returns (out_tokens [B, k+1], n_accepted [B]).  See include/cachespec.h."""
+    lib = load_library()
+    dev = target_logits.device
+    if target_logits.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("logits must be float32 or bfloat16")
+    dtype = target_logits.dtype
+    _need(target_logits, "target_logits", dtype, 3, dev)
+    B, rows, V = target_logits.shape
+    k = rows - 1
+    if draft_logits is not None:
+        _need(draft_logits, "draft_logits", dtype, 3, dev)
+        if tuple(draft_logits.shape) != (B, k, V):
+            raise ValueError(f"draft_logits must be [{B}, {k}, {V}]")
+    _need(draft_tokens, "draft_tokens", torch.int32, 2, dev)
+    _need(uniforms, "uniforms", torch.float32, 2, dev)
+    if out_tokens is None:
+        out_tokens = torch.empty((B, k + 1), dtype=torch.int32, device=dev)
+    if out_n_accepted is None:
+        out_n_accepted = torch.empty((B,), dtype=torch.int32, device=dev)
+    _need(out_tokens, "out_tokens", torch.int32, 2, dev)
+    _need(out_n_accepted, "out_n_accepted", torch.int32, 1, dev)
+    d = AcceptDims(B, V, CS_F32 if dtype == torch.float32 else CS_BF16)
+    st = lib.cs_spec_accept(ctypes.byref(d), _ptr(target_logits), _ptr(draft_logits),
+                            _ptr(draft_tokens), _ptr(uniforms), int(k), float(temperature),
+                            _ptr(out_tokens), _ptr(out_n_accepted), None, 0,
+                            _stream(dev) if stream is None else stream)
+    _check(lib, st)
+    return out_tokens, out_n_accepted
+
+
+def cs_read_device_status(workspace: torch.Tensor, stream: int | None = None) -> int:
+    """Status word of a verify-attention workspace (synchronises the stream)."""
+    lib = load_library()
+    v = ctypes.c_int32(0)
+    _check(lib, lib.cs_read_device_status(_ptr(workspace), ctypes.byref(v),
+                                          _stream(workspace.device) if stream is None else stream))
+    return int(v.value)

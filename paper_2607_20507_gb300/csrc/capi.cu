@@ -1,0 +1,170 @@
+// capi.cu -- the extern "C" surface of libcachespec.so (see include/cachespec.h):
+// host-side argument checks, the workspace queries and dispatch to the
+// kernel launchers.  Nothing here allocates, frees or synchronises device
+// memory except cs_read_device_status, which is documented to synchronise.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "cs_internal.h"
+
+namespace cs {
+
+namespace {
+thread_local char g_err[512] = "";
+int g_sms[64] = {0};
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+bool pow2_page(int ps) {
+    return ps == 8 || ps == 16 || ps == 32 || ps == 64 || ps == 128 || ps == 256;
+}
+
+cs_status check_attn(const cs_attn_dims* d, int32_t n_draft) {
+    if (!d) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
+    if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
+    if (d->n_q_heads <= 0 || d->n_kv_heads <= 0)
+        return fail(CS_ERR_INVALID_ARG, "head counts must be positive (Hq=%d, Hkv=%d)", d->n_q_heads,
+                    d->n_kv_heads);
+    if (d->n_q_heads % d->n_kv_heads != 0)
+        return fail(CS_ERR_INVALID_ARG, "Hq=%d is not a multiple of Hkv=%d", d->n_q_heads,
+                    d->n_kv_heads);
+    if (d->head_dim <= 0) return fail(CS_ERR_INVALID_ARG, "head_dim %d <= 0", d->head_dim);
+    if (d->page_size <= 0) return fail(CS_ERR_INVALID_ARG, "page_size %d <= 0", d->page_size);
+    if (d->max_pages_per_seq <= 0)
+        return fail(CS_ERR_INVALID_ARG, "max_pages_per_seq %d <= 0", d->max_pages_per_seq);
+    if (d->num_pages <= 0) return fail(CS_ERR_INVALID_ARG, "num_pages %d <= 0", d->num_pages);
+    if (isnan(d->sm_scale) || isinf(d->sm_scale))
+        return fail(CS_ERR_INVALID_ARG, "sm_scale is not finite");
+    if (n_draft < 1 || n_draft > 16) return fail(CS_ERR_INVALID_ARG, "n_draft %d not in [1, 16]", n_draft);
+    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this build implements 128)", d->head_dim);
+    if (!pow2_page(d->page_size))
+        return fail(CS_ERR_UNSUPPORTED, "page_size %d (supported: 8..256, powers of two)", d->page_size);
+    const long long rows = (long long)(n_draft + 1) * (d->n_q_heads / d->n_kv_heads);
+    if (rows > 144) return fail(CS_ERR_UNSUPPORTED, "(k+1)*G = %lld query rows per KV head (max 144)", rows);
+    if ((long long)d->max_pages_per_seq * d->page_size > (1LL << 30))
+        return fail(CS_ERR_INVALID_ARG, "max_pages_per_seq * page_size exceeds 2^30 keys");
+    return CS_OK;
+}
+
+cs_status check_accept(const cs_accept_dims* d, int32_t n_draft, float temperature) {
+    if (!d) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
+    if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
+    if (d->vocab <= 0) return fail(CS_ERR_INVALID_ARG, "vocab %d <= 0", d->vocab);
+    if (d->logit_dtype != CS_F32 && d->logit_dtype != CS_BF16)
+        return fail(CS_ERR_INVALID_ARG, "logit_dtype %d is neither CS_F32 nor CS_BF16", d->logit_dtype);
+    if (n_draft < 1 || n_draft > 16) return fail(CS_ERR_INVALID_ARG, "n_draft %d not in [1, 16]", n_draft);
+    if (!(temperature >= 0.f) || isinf(temperature))
+        return fail(CS_ERR_INVALID_ARG, "temperature must be finite and >= 0");
+    if ((long long)d->batch * (n_draft + 1) * (long long)d->vocab > (1LL << 46))
+        return fail(CS_ERR_INVALID_ARG, "logit tensor too large");
+    return CS_OK;
+}
+}  // namespace
+
+cs_status fail(cs_status st, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+    return st;
+}
+
+cs_status cuda_fail(cudaError_t e, const char* what) {
+    return fail(CS_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorString(e), cudaGetErrorName(e));
+}
+
+int current_sm_count() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (!g_sms[dev]) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 148;
+        g_sms[dev] = n;
+    }
+    return g_sms[dev];
+}
+
+}  // namespace cs
+
+using namespace cs;
+
+extern "C" {
+
+int32_t cs_abi_version(void) { return CS_ABI_VERSION; }
+
+const char* cs_last_error(void) { return g_err; }
+
+size_t cs_verify_attention_workspace_bytes(const cs_attn_dims* dims, int32_t n_draft) {
+    if (check_attn(dims, n_draft) != CS_OK) return 0;
+    return plan_verify_attention(*dims, n_draft, current_sm_count()).bytes;
+}
+
+cs_status cs_verify_attention(const cs_attn_dims* dims, const void* q, const void* k_pages,
+                              const void* v_pages, const int32_t* page_table,
+                              const int32_t* ctx_lens, int32_t n_draft, void* out,
+                              void* workspace, size_t workspace_bytes, cs_stream_t stream) {
+    cs_status st = check_attn(dims, n_draft);
+    if (st != CS_OK) return st;
+    if (dims->batch == 0) return CS_OK;
+    if (!q || !k_pages || !v_pages || !page_table || !ctx_lens || !out)
+        return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (!aligned(k_pages, 16) || !aligned(v_pages, 16))
+        return fail(CS_ERR_INVALID_ARG, "k_pages and v_pages must be 16-byte aligned");
+    if (!aligned(q, 4) || !aligned(out, 8))
+        return fail(CS_ERR_INVALID_ARG, "q must be 4-byte and out 8-byte aligned");
+    if (!aligned(page_table, 4) || !aligned(ctx_lens, 4))
+        return fail(CS_ERR_INVALID_ARG, "page_table and ctx_lens must be 4-byte aligned");
+    const AttnPlan plan = plan_verify_attention(*dims, n_draft, current_sm_count());
+    if (!workspace || workspace_bytes < plan.bytes)
+        return fail(CS_ERR_WORKSPACE, "workspace of %zu bytes given, %zu needed", workspace_bytes,
+                    plan.bytes);
+    if (!aligned(workspace, 256)) return fail(CS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    return launch_verify_attention(*dims, plan, q, k_pages, v_pages, page_table, ctx_lens, out,
+                                   workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t cs_spec_accept_workspace_bytes(const cs_accept_dims* dims, int32_t n_draft) {
+    (void)dims;
+    (void)n_draft;
+    return 0;
+}
+
+cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
+                         const void* draft_logits, const int32_t* draft_tokens,
+                         const float* uniforms, int32_t n_draft, float temperature,
+                         int32_t* out_tokens, int32_t* out_n_accepted, void* workspace,
+                         size_t workspace_bytes, cs_stream_t stream) {
+    (void)workspace;
+    (void)workspace_bytes;
+    cs_status st = check_accept(dims, n_draft, temperature);
+    if (st != CS_OK) return st;
+    if (dims->batch == 0) return CS_OK;
+    if (!target_logits || !draft_tokens || !uniforms || !out_tokens || !out_n_accepted)
+        return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (temperature > 0.f && !draft_logits)
+        return fail(CS_ERR_INVALID_ARG, "draft_logits is NULL with temperature > 0");
+    const size_t esz = dims->logit_dtype == CS_F32 ? 4 : 2;
+    if (!aligned(target_logits, esz) || (draft_logits && !aligned(draft_logits, esz)))
+        return fail(CS_ERR_INVALID_ARG, "logit pointers must be aligned to their element size");
+    if (!aligned(draft_tokens, 4) || !aligned(uniforms, 4) || !aligned(out_tokens, 4) ||
+        !aligned(out_n_accepted, 4))
+        return fail(CS_ERR_INVALID_ARG, "int32/fp32 pointers must be 4-byte aligned");
+    return launch_spec_accept(*dims, target_logits, temperature > 0.f ? draft_logits : nullptr,
+                              draft_tokens, uniforms, n_draft, temperature, out_tokens,
+                              out_n_accepted, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cs_status cs_read_device_status(const void* workspace, int32_t* status_out, cs_stream_t stream) {
+    if (!workspace || !status_out) return fail(CS_ERR_INVALID_ARG, "NULL argument");
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(status_out, workspace, sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(status)");
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    return CS_OK;
+}
+
+}  // extern "C"

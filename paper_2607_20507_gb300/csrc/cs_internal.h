@@ -1,0 +1,43 @@
+// cs_internal.h -- host-side interface between the C ABI (capi.cu) and the
+// kernel launchers.  Not installed; the public surface is include/cachespec.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "cachespec.h"
+
+namespace cs {
+
+// Records a printf-style message for cs_last_error() and returns `st`.
+cs_status fail(cs_status st, const char* fmt, ...);
+cs_status cuda_fail(cudaError_t e, const char* what);
+
+// Streaming multiprocessors of the current device (cached per device).
+int current_sm_count();
+
+// ------------------------------------------------------------- attention
+struct AttnPlan {
+    int group;        // G = Hq / Hkv
+    int rows;         // k + 1
+    int n_rows;       // (k+1) * G query rows per KV head
+    int row_warps;    // ceil(n_rows / 16) consumer warps
+    int chunk;        // tokens per split (multiple of the 64-token tile)
+    int ns_max;       // splits of the longest admissible context
+    size_t off_tickets, off_part_o, off_part_ml, bytes;   // workspace layout
+};
+AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count);
+
+cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& plan, const void* q,
+                                  const void* k_pages, const void* v_pages,
+                                  const int32_t* page_table, const int32_t* ctx_lens, void* out,
+                                  void* workspace, cudaStream_t stream);
+
+// ------------------------------------------------------------ acceptance
+cs_status launch_spec_accept(const cs_accept_dims& d, const void* target, const void* draft,
+                             const int32_t* tokens, const float* uniforms, int n_draft,
+                             float temperature, int32_t* out_tokens, int32_t* out_n,
+                             cudaStream_t stream);
+
+}  // namespace cs

@@ -1,0 +1,149 @@
+"""The C-ABI library on the host: it builds, loads, exports every symbol the
+header declares, and rejects bad arguments before enqueuing anything.  No
+call here reaches a kernel, so the file runs without a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2607_20507_gb300 import binding, build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "cachespec.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return binding.load_library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(cs_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for must in ("cs_verify_attention", "cs_spec_accept", "cs_verify_attention_workspace_bytes",
+                 "cs_spec_accept_workspace_bytes", "cs_last_error"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert set(binding.EXPORTED_SYMBOLS) == set(declared_functions())
+    assert lib.cs_abi_version() == 1
+
+
+def test_library_is_built_for_sm_103a_only():
+    # the build passes exactly one -gencode, for sm_103a
+    assert build.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+FAKE = 0x10000  # a non-null, 256-byte aligned address that is never dereferenced
+
+
+def attn(lib, dims, n_draft=4, q=FAKE, kp=FAKE, vp=FAKE, pt=FAKE, cl=FAKE, out=FAKE, ws=FAKE,
+         ws_bytes=1 << 40):
+    return lib.cs_verify_attention(ctypes.byref(dims), q, kp, vp, pt, cl, n_draft, out, ws,
+                                   ws_bytes, None)
+
+
+def good_attn_dims():
+    return binding.AttnDims(4, 32, 8, 128, 16, 64, 256, 0.0)
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("batch", -1, binding.CS_ERR_INVALID_ARG),
+    ("n_q_heads", 0, binding.CS_ERR_INVALID_ARG),
+    ("n_kv_heads", 0, binding.CS_ERR_INVALID_ARG),
+    ("n_q_heads", 30, binding.CS_ERR_INVALID_ARG),       # not a multiple of Hkv = 8
+    ("head_dim", 64, binding.CS_ERR_UNSUPPORTED),
+    ("page_size", 12, binding.CS_ERR_UNSUPPORTED),
+    ("page_size", 0, binding.CS_ERR_INVALID_ARG),
+    ("max_pages_per_seq", 0, binding.CS_ERR_INVALID_ARG),
+    ("num_pages", 0, binding.CS_ERR_INVALID_ARG),
+    ("sm_scale", float("nan"), binding.CS_ERR_INVALID_ARG),
+])
+def test_verify_attention_rejects_bad_dims(lib, field, value, code):
+    d = good_attn_dims()
+    setattr(d, field, value)
+    assert attn(lib, d) == code
+    assert lib.cs_last_error()
+
+
+@pytest.mark.parametrize("n_draft", [0, -1, 17])
+def test_verify_attention_rejects_bad_n_draft(lib, n_draft):
+    assert attn(lib, good_attn_dims(), n_draft=n_draft) == binding.CS_ERR_INVALID_ARG
+
+
+def test_verify_attention_rejects_too_many_rows(lib):
+    d = binding.AttnDims(1, 128, 8, 128, 16, 8, 8, 0.0)     # G = 16, (k+1)*G = 272
+    assert attn(lib, d, n_draft=16) == binding.CS_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("arg", ["q", "kp", "vp", "pt", "cl", "out"])
+def test_verify_attention_rejects_null_pointers(lib, arg):
+    assert attn(lib, good_attn_dims(), **{arg: None}) == binding.CS_ERR_INVALID_ARG
+
+
+def test_verify_attention_rejects_misaligned_pool(lib):
+    assert attn(lib, good_attn_dims(), kp=FAKE + 8) == binding.CS_ERR_INVALID_ARG
+    assert attn(lib, good_attn_dims(), ws=FAKE + 64) == binding.CS_ERR_INVALID_ARG
+
+
+def test_verify_attention_workspace_is_checked(lib):
+    d = good_attn_dims()
+    need = lib.cs_verify_attention_workspace_bytes(ctypes.byref(d), 4)
+    assert need >= 256
+    assert attn(lib, d, ws=None) == binding.CS_ERR_WORKSPACE
+    assert attn(lib, d, ws_bytes=need - 1) == binding.CS_ERR_WORKSPACE
+    assert "needed" in lib.cs_last_error().decode()
+
+
+def test_empty_batch_is_a_no_op(lib):
+    d = good_attn_dims()
+    d.batch = 0
+    assert attn(lib, d, q=None, kp=None, vp=None, pt=None, cl=None, out=None, ws=None) == binding.CS_OK
+    a = binding.AcceptDims(0, 32000, binding.CS_BF16)
+    assert lib.cs_spec_accept(ctypes.byref(a), None, None, None, None, 4, 1.0, None, None, None, 0,
+                              None) == binding.CS_OK
+
+
+def accept(lib, dims, n_draft=4, T=1.0, t=FAKE, d=FAKE, x=FAKE, u=FAKE, out=FAKE, n=FAKE):
+    return lib.cs_spec_accept(ctypes.byref(dims), t, d, x, u, n_draft, T, out, n, None, 0, None)
+
+
+@pytest.mark.parametrize("field,value", [("batch", -2), ("vocab", 0), ("logit_dtype", 7)])
+def test_spec_accept_rejects_bad_dims(lib, field, value):
+    dims = binding.AcceptDims(4, 32000, binding.CS_BF16)
+    setattr(dims, field, value)
+    assert accept(lib, dims) == binding.CS_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("T", [-0.5, float("nan"), float("inf")])
+def test_spec_accept_rejects_bad_temperature(lib, T):
+    assert accept(lib, binding.AcceptDims(4, 32000, binding.CS_BF16), T=T) == binding.CS_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("n_draft", [0, 17])
+def test_spec_accept_rejects_bad_n_draft(lib, n_draft):
+    assert accept(lib, binding.AcceptDims(4, 32000, binding.CS_BF16), n_draft=n_draft) == binding.CS_ERR_INVALID_ARG
+
+
+def test_spec_accept_null_and_alignment(lib):
+    dims = binding.AcceptDims(4, 32000, binding.CS_F32)
+    for arg in ("t", "x", "u", "out", "n"):
+        assert accept(lib, dims, **{arg: None}) == binding.CS_ERR_INVALID_ARG
+    assert accept(lib, dims, d=None) == binding.CS_ERR_INVALID_ARG            # T > 0 needs the draft
+    assert accept(lib, dims, t=FAKE + 2) == binding.CS_ERR_INVALID_ARG        # fp32 logits, 2-byte offset
+    assert lib.cs_spec_accept_workspace_bytes(ctypes.byref(dims), 4) == 0
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    with pytest.raises(RuntimeError, match="not found"):
+        binding.load_library(str(tmp_path / "missing.so"))
