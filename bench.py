@@ -249,7 +249,7 @@ def run_gb300(args) -> dict | None:
     with sampler:
         t0 = time.time()
         n = 0
-        while n < args.warmup or time.time() - t0 < 1.0:
+        while n < args.warmup or time.time() - t0 < args.warmup_seconds:
             flush.zero_()
             step()
             n += 1
@@ -377,7 +377,7 @@ def run_gb300(args) -> dict | None:
                     "note": "host->device copy of every input from pinned memory and device->host "
                             "read of the emitted tokens inside the timed region"},
             "gpu_launches": 2 * args.steps * math.ceil(B / 65535),
-            "clocks": sampler.summary() | {"window": "warm-up (>= 1 s) and the timed steps"},
+            "clocks": sampler.summary() | {"window": f"warm-up (>= {args.warmup_seconds:g} s) and the timed steps"},
         }
     if world > 1:
         dist.barrier()
@@ -485,6 +485,8 @@ def main(argv=None) -> int:
     ap.add_argument("--temperature", type=float, default=None)
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--warmup-seconds", type=float, default=1.0,
+                    help="keep warming up (and sampling clocks) for at least this long")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)
     args.steps = max(1, args.steps)

@@ -48,9 +48,9 @@ def _load():
         lib.oracle_verify_attention.restype = ctypes.c_int
         lib.oracle_verify_attention.argtypes = [i32] * 7 + [f64] + [vp] * 5 + [i32, vp]
         lib.oracle_spec_accept.restype = ctypes.c_int
-        lib.oracle_spec_accept.argtypes = [i32, i32, i32, vp, vp, vp, vp, i32, f64, vp, vp, vp]
+        lib.oracle_spec_accept.argtypes = [i32, i32, i32, vp, vp, vp, vp, i32, f64, vp, vp, vp, vp]
         lib.oracle_spec_accept_f64u.restype = ctypes.c_int
-        lib.oracle_spec_accept_f64u.argtypes = [i32, i32, i32, vp, vp, vp, vp, i32, f64, vp, vp, vp]
+        lib.oracle_spec_accept_f64u.argtypes = [i32, i32, i32, vp, vp, vp, vp, i32, f64, vp, vp, vp, vp]
         lib.oracle_row_probs.restype = f64
         lib.oracle_row_probs.argtypes = [vp, i32, i32, f64, vp]
         lib.oracle_residual.restype = f64
@@ -113,14 +113,17 @@ def verify_attention(q_bits, k_bits, v_bits, page_table, ctx_lens, n_draft, scal
     return out
 
 
-def spec_accept(target, draft, draft_tokens, uniforms, temperature):
+def spec_accept(target, draft, draft_tokens, uniforms, temperature, with_draw_margin=False):
     """fp64 speculative acceptance.
 
     target [B, k+1, V] (float32 or uint16 bf16 bits); draft [B, k, V] same dtype
     (None allowed when temperature == 0); draft_tokens [B, k] int32;
     uniforms [B, k+1] float32 (or float64, which the pins use to place u
     exactly on either side of a threshold).  Returns (out_tokens [B, k+1] int32,
-    n_accepted [B] int32, margin [B] float64).
+    n_accepted [B] int32, margin [B] float64): margin is the smallest
+    |u_i - p_i(x_i)/q_i(x_i)| over the deciding accept tests.  With
+    ``with_draw_margin`` a fourth array gives |u_k - CDF| at the two edges of
+    the drawn cell.
     """
     lib = _load()
     t, code = _logit_array(target)
@@ -141,10 +144,13 @@ def spec_accept(target, draft, draft_tokens, uniforms, temperature):
     out = np.zeros((B, k + 1), dtype=np.int32)
     acc = np.zeros((B,), dtype=np.int32)
     margin = np.zeros((B,), dtype=np.float64)
+    draw_margin = np.zeros((B,), dtype=np.float64)
     rc = fn(B, V, code, _ptr(t), _ptr(d), _ptr(x), _ptr(u), k,
-            float(temperature), _ptr(out), _ptr(acc), _ptr(margin))
+            float(temperature), _ptr(out), _ptr(acc), _ptr(margin), _ptr(draw_margin))
     if rc != 0:
         raise RuntimeError(f"oracle_spec_accept failed with status {rc}")
+    if with_draw_margin:
+        return out, acc, margin, draw_margin
     return out, acc, margin
 
 

@@ -261,10 +261,13 @@ int32_t oracle_row_argmax(const void* row, int32_t dtype, int32_t vocab) {
  *                       final draw (residual or bonus)
  * out_tokens [B, k+1]   x_0..x_{a-1}, then the drawn token, then -1
  * out_n_accepted [B]    a
- * out_margin [B]        (may be NULL) smallest |u - threshold| over every
- *                       comparison that decided the output: the accept tests
- *                       of positions 0..a and the two CDF values bracketing
- *                       the draw.  +inf for greedy (no threshold compare).
+ * out_margin [B]        (may be NULL) smallest |u_i - p_i(x_i)/q_i(x_i)| over
+ *                       the accept tests that decided the output (positions
+ *                       0..a); +inf when there is none (greedy, or a = 0
+ *                       through an invalid token)
+ * out_draw_margin [B]   (may be NULL) distance of u_k from the two CDF values
+ *                       C(v-1)/Z and C(v)/Z that bracket the drawn token v;
+ *                       +inf for greedy
  *
  * A draft token outside [0, V) counts as rejected (its ratio is 0).
  */
@@ -272,7 +275,8 @@ int oracle_spec_accept_f64u(int32_t batch, int32_t vocab, int32_t dtype,
                             const void* target, const void* draft,
                             const int32_t* tokens, const double* uniforms,
                             int32_t n_draft, double temperature, int32_t* out_tokens,
-                            int32_t* out_n_accepted, double* out_margin) {
+                            int32_t* out_n_accepted, double* out_margin,
+                            double* out_draw_margin) {
     if (batch < 0 || vocab <= 0 || n_draft < 0 || (dtype != 0 && dtype != 1))
         return ORC_BAD_ARG;
     if (!(temperature >= 0.0)) return ORC_BAD_ARG;
@@ -290,7 +294,7 @@ int oracle_spec_accept_f64u(int32_t batch, int32_t vocab, int32_t dtype,
         const double* u = uniforms + b * (k + 1);
         int32_t* out = out_tokens + b * (k + 1);
         int64_t a = k;
-        double margin = INFINITY;
+        double margin = INFINITY, draw_margin = INFINITY;
 
         if (temperature == 0.0) {
             /* greedy: argmax agreement */
@@ -349,9 +353,7 @@ int oracle_spec_accept_f64u(int32_t batch, int32_t vocab, int32_t dtype,
                     Z += r[v];
                 }
             }
-            double dm = INFINITY;
-            const int32_t pick = oracle_inverse_cdf(r, Z, vocab, u[k], &dm);
-            if (dm < margin) margin = dm;
+            const int32_t pick = oracle_inverse_cdf(r, Z, vocab, u[k], &draw_margin);
             for (int64_t i = 0; i < a; ++i) out[i] = x[i];
             out[a] = pick;
             free(p);
@@ -361,6 +363,7 @@ int oracle_spec_accept_f64u(int32_t batch, int32_t vocab, int32_t dtype,
         for (int64_t i = a + 1; i <= k; ++i) out[i] = -1;
         out_n_accepted[b] = (int32_t)a;
         if (out_margin) out_margin[b] = margin;
+        if (out_draw_margin) out_draw_margin[b] = draw_margin;
     }
     return status;
 }
@@ -370,7 +373,8 @@ int oracle_spec_accept(int32_t batch, int32_t vocab, int32_t dtype,
                        const void* target, const void* draft,
                        const int32_t* tokens, const float* uniforms,
                        int32_t n_draft, double temperature, int32_t* out_tokens,
-                       int32_t* out_n_accepted, double* out_margin) {
+                       int32_t* out_n_accepted, double* out_margin,
+                       double* out_draw_margin) {
     if (batch < 0 || n_draft < 0) return ORC_BAD_ARG;
     const size_t n = (size_t)batch * (size_t)(n_draft + 1);
     double* u = (double*)malloc((n ? n : 1) * sizeof(double));
@@ -378,7 +382,7 @@ int oracle_spec_accept(int32_t batch, int32_t vocab, int32_t dtype,
     for (size_t i = 0; i < n; ++i) u[i] = (double)uniforms[i];
     const int rc = oracle_spec_accept_f64u(batch, vocab, dtype, target, draft, tokens, u,
                                            n_draft, temperature, out_tokens,
-                                           out_n_accepted, out_margin);
+                                           out_n_accepted, out_margin, out_draw_margin);
     free(u);
     return rc;
 }

@@ -273,6 +273,8 @@ def test_margin_reports_threshold_distance():
     rows = {k: np.log(np.asarray(v, np.float64)).astype(np.float32) for k, v in g["rows"].items()}
     zt = np.stack([rows["H"], rows["R"]])[None]
     zd = rows["U"][None, None]
-    _, _, m = oracle.spec_accept(zt, zd, np.array([[2]], np.int32), np.array([[0.49, 0.05]], np.float32), 1.0)
-    # closest decisive comparison: u_0 = 0.49 against the ratio 0.5; the draw cell [0, 0.1) is farther
+    _, _, m, dm = oracle.spec_accept(zt, zd, np.array([[2]], np.int32),
+                                     np.array([[0.49, 0.05]], np.float32), 1.0, with_draw_margin=True)
+    # accept test: u_0 = 0.49 against the ratio 0.5; draw: u_1 = 0.05 inside the cell [0, 0.1)
     assert m[0] == pytest.approx(0.01, abs=1e-6)
+    assert dm[0] == pytest.approx(0.05, abs=1e-6)
