@@ -163,6 +163,38 @@ cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
                          size_t workspace_bytes, cs_stream_t stream);
 
 /*
+ * Allocation-free verify attention.  The paper has no counterpart: this entry
+ * point serves callers of this library that cannot allocate device memory
+ * themselves -- code running inside a host framework that owns every device
+ * allocation, serving loops that allow no allocation after start-up
+ * (cudaMalloc can stall the whole device), or bindings without a device
+ * allocator.
+ *
+ * Same arguments, layouts, results and error codes as cs_verify_attention,
+ * without the workspace: the scratch is a fixed array of
+ * CS_NOALLOC_SCRATCH_BYTES compiled into this library, which every GPU that
+ * loads the library holds until the process exits.  The call never runs
+ * cudaMalloc, cudaFree or any other allocating routine.
+ *   - A problem that needs more scratch than that (see
+ *     cs_verify_attention_workspace_bytes) returns CS_ERR_UNSUPPORTED with a
+ *     message giving both sizes; use cs_verify_attention then.
+ *   - The first call on each device looks up the array's device address with
+ *     cudaGetSymbolAddress (with that device current) and caches it; make
+ *     that first call before any stream capture begins.
+ *   - Each call clears the part of the scratch that must start at zero (an
+ *     asynchronous memset on `stream`), so a failed call does not affect the
+ *     next one.
+ *   - Every call on a device shares the one array: calls whose kernels may
+ *     overlap on the GPU (different streams, or host threads using different
+ *     streams) race on it.  Order them on one stream or with events.
+ */
+#define CS_NOALLOC_SCRATCH_BYTES (32u << 20)
+cs_status cs_verify_attention_noalloc(const cs_attn_dims* dims, const void* q, const void* k_pages,
+                                      const void* v_pages, const int32_t* page_table,
+                                      const int32_t* ctx_lens, int32_t n_draft, void* out,
+                                      cs_stream_t stream);
+
+/*
  * Device status word of a verify-attention workspace: 0 when every call that
  * used it finished normally; otherwise a bit set of CS_DEVICE_* flags (a
  * bounded wait inside a kernel gave up, so that call's output is invalid).

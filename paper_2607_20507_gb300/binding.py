@@ -22,7 +22,7 @@ STATUS_NAMES = {0: "CS_OK", 1: "CS_ERR_INVALID_ARG", 2: "CS_ERR_UNSUPPORTED", 3:
                 4: "CS_ERR_WORKSPACE"}
 EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_workspace_bytes",
                     "cs_verify_attention", "cs_spec_accept_workspace_bytes", "cs_spec_accept",
-                    "cs_read_device_status")
+                    "cs_read_device_status", "cs_verify_attention_noalloc")
 
 
 class AttnDims(ctypes.Structure):
@@ -75,6 +75,9 @@ def load_library(path: str | None = None):
         lib.cs_spec_accept.restype = ctypes.c_int
         lib.cs_spec_accept.argtypes = [ctypes.POINTER(AcceptDims), vp, vp, vp, vp, i32,
                                        ctypes.c_float, vp, vp, vp, sz, vp]
+        lib.cs_verify_attention_noalloc.restype = ctypes.c_int
+        lib.cs_verify_attention_noalloc.argtypes = [ctypes.POINTER(AttnDims), vp, vp, vp, vp, vp,
+                                                    i32, vp, vp]
         lib.cs_read_device_status.restype = ctypes.c_int
         lib.cs_read_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_int32), vp]
         if path is None:
@@ -197,6 +200,28 @@ def cs_spec_accept(target_logits, draft_logits, draft_tokens, uniforms, temperat
                             _stream(dev) if stream is None else stream)
     _check(lib, st)
     return out_tokens, out_n_accepted
+
+
+def cs_verify_attention_noalloc(q, k_pages, v_pages, page_table, ctx_lens, n_draft, out=None,
+                                sm_scale: float = 0.0, stream: int | None = None):
+    """Verify attention without a workspace, for callers that cannot allocate device
+    memory (the library's own fixed scratch is used; see include/cachespec.h)."""
+    lib = load_library()
+    dev = q.device
+    _need(q, "q", torch.bfloat16, 4, dev)
+    _need(k_pages, "k_pages", torch.bfloat16, 4, dev)
+    _need(v_pages, "v_pages", torch.bfloat16, 4, dev)
+    _need(page_table, "page_table", torch.int32, 2, dev)
+    _need(ctx_lens, "ctx_lens", torch.int32, 1, dev)
+    d = attn_dims(q, k_pages, page_table, sm_scale)
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16, 4, dev)
+    st = lib.cs_verify_attention_noalloc(ctypes.byref(d), _ptr(q), _ptr(k_pages), _ptr(v_pages),
+                                         _ptr(page_table), _ptr(ctx_lens), int(n_draft), _ptr(out),
+                                         _stream(dev) if stream is None else stream)
+    _check(lib, st)
+    return out
 
 
 def cs_read_device_status(workspace: torch.Tensor, stream: int | None = None) -> int:
