@@ -219,6 +219,8 @@ def run_gb300(args) -> dict | None:
     binding.load_library()
 
     w = replica_workload(W.WORKLOADS[args.workload], rank)
+    if args.batch:
+        w = w.with_(batch=args.batch)
     T = args.temperature if args.temperature is not None else max(w.temperatures)
     att = W.attention_inputs(w, dev)
     acc = W.accept_inputs(w, T, dev)
@@ -244,6 +246,19 @@ def run_gb300(args) -> dict | None:
         attention()
         accept(acc, T)
 
+    # Each call is also captured once into a CUDA graph: the device-timed
+    # steps replay them, so that host-side enqueue time (Python, ctypes,
+    # tensor-map encoding) cannot open gaps inside the timed events.
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize()
+    g_attn, g_acc = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_attn):
+        attention()
+    with torch.cuda.graph(g_acc):
+        accept(acc, T)
+    torch.cuda.synchronize()
+
     # warm-up: at least W steps and about a second of work, with clocks sampled
     sampler = ClockSampler(local)
     with sampler:
@@ -251,7 +266,8 @@ def run_gb300(args) -> dict | None:
         n = 0
         while n < args.warmup or time.time() - t0 < args.warmup_seconds:
             flush.zero_()
-            step()
+            g_attn.replay()
+            g_acc.replay()
             n += 1
             if n % 64 == 0:
                 torch.cuda.synchronize()
@@ -266,14 +282,24 @@ def run_gb300(args) -> dict | None:
         for e0, e1, e2 in ev:
             flush.zero_()
             e0.record(stream)
-            attention()
+            g_attn.replay()
             e1.record(stream)
-            accept(acc, T)
+            g_acc.replay()
             e2.record(stream)
         torch.cuda.synchronize()
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
+    # the same K steps through the direct API calls (host enqueue on the path)
+    evd = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    for e0, e1 in evd:
+        flush.zero_()
+        e0.record(stream)
+        step()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    direct_us = 1e6 * statistics.mean(e0.elapsed_time(e1) * 1e-3 for e0, e1 in evd)
     t_attn = [e0.elapsed_time(e1) * 1e-3 for e0, e1, _ in ev]
     t_acc = [e1.elapsed_time(e2) * 1e-3 for _, e1, e2 in ev]
     t_step = [a + b for a, b in zip(t_attn, t_acc)]
@@ -287,10 +313,14 @@ def run_gb300(args) -> dict | None:
                for _ in range(args.steps)]
         for _ in range(3):
             accept(acc_greedy, 0.0)
+        torch.cuda.synchronize()
+        g_gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_gr):
+            accept(acc_greedy, 0.0)
         for e0, e1 in evg:
             flush.zero_()
             e0.record(stream)
-            accept(acc_greedy, 0.0)
+            g_gr.replay()
             e1.record(stream)
         torch.cuda.synchronize()
         tg = [e0.elapsed_time(e1) * 1e-3 for e0, e1 in evg]
@@ -369,6 +399,8 @@ def run_gb300(args) -> dict | None:
                        "l2": "flushed between steps (512 MiB memset outside the timed events)",
                        "parallelism": f"replicas x{world} (requests shard; no collective)"},
             "kernels": kernels,
+            "launch": {"timed_steps": "CUDA-graph replay of each C-ABI call (one graph per call)",
+                       "direct_call_step_us": round(direct_us, 2)},
             "greedy": greedy,
             "roofline": roofline,
             "cpu_baseline": cpu,
@@ -376,7 +408,9 @@ def run_gb300(args) -> dict | None:
                     "d2h_bytes_per_step": d2h,
                     "note": "host->device copy of every input from pinned memory and device->host "
                             "read of the emitted tokens inside the timed region"},
-            "gpu_launches": 2 * args.steps * math.ceil(B / 65535),
+            # per step: the verify-attention kernel and its split merge (one pair per
+            # 1024-request slice) and the acceptance kernel (one per 65535 requests)
+            "gpu_launches": args.steps * (2 * math.ceil(B / 1024) + math.ceil(B / 65535)),
             "clocks": sampler.summary() | {"window": f"warm-up (>= {args.warmup_seconds:g} s) and the timed steps"},
         }
     if world > 1:
@@ -483,6 +517,8 @@ def main(argv=None) -> int:
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--workload", type=int, default=2, choices=sorted(W.WORKLOADS))
     ap.add_argument("--temperature", type=float, default=None)
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the workload's batch (smaller cases for profiling)")
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--warmup-seconds", type=float, default=1.0,

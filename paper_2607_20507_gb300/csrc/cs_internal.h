@@ -23,9 +23,8 @@ struct AttnPlan {
     int rows;         // k + 1
     int n_rows;       // (k+1) * G query rows per KV head
     int row_warps;    // ceil(n_rows / 16) consumer warps
-    int chunk;        // tokens per split (multiple of the 64-token tile)
-    int ns_max;       // splits of the longest admissible context
-    size_t off_tickets, off_part_o, off_part_ml, bytes;   // workspace layout
+    int grid;         // persistent CTAs (resident capacity of the device)
+    size_t off_part_o, off_part_ml, bytes;   // workspace layout (status word at 0)
 };
 AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count);
 

@@ -69,12 +69,9 @@ extern "C" cs_status cs_verify_attention_noalloc(const cs_attn_dims* dims, const
     void* scratch = nullptr;
     cs_status st = scratch_address(&scratch);
     if (st != CS_OK) return st;
-    // The status word and the split tickets must start at zero; the previous
-    // call leaves them at zero when it completes, but clear them anyway so
-    // that a failed or interrupted call cannot leak into this one.
-    const cs::AttnPlan plan = cs::plan_verify_attention(*dims, n_draft, cs::current_sm_count());
-    const size_t zero_bytes = plan.ns_max > 1 ? plan.off_part_ml : 256;
-    cudaError_t e = cudaMemsetAsync(scratch, 0, zero_bytes, reinterpret_cast<cudaStream_t>(stream));
+    // The status word must start at zero: clear it, so that a failed or
+    // interrupted call cannot leak into this one.
+    cudaError_t e = cudaMemsetAsync(scratch, 0, 256, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cs::cuda_fail(e, "cudaMemsetAsync(noalloc scratch)");
     return cs_verify_attention(dims, q, k_pages, v_pages, page_table, ctx_lens, n_draft, out,
                                scratch, CS_NOALLOC_SCRATCH_BYTES, stream);

@@ -153,7 +153,9 @@ __device__ __forceinline__ void slice_stats(const T* rt, const T* rd, bool two, 
     }
 }
 
-// Block reduction of per-thread (m, s) pairs for two rows, in a fixed order.
+// Block reduction of per-thread (m, s) pairs for two rows, in a fixed order
+// (xor butterflies within each warp, then across the warp results in warp 0).
+// Thread 0 ends with the CTA's pairs.
 __device__ __forceinline__ void block_fold2(float (&m)[2], float (&s)[2], float c_hi, float c_lo,
                                             float (*red)[4]) {
 #pragma unroll
@@ -173,18 +175,49 @@ __device__ __forceinline__ void block_fold2(float (&m)[2], float (&s)[2], float 
         red[warp][3] = s[1];
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        float M[2] = {kNegInf, kNegInf}, S[2] = {0.f, 0.f};
-        for (int w = 0; w < kWarps; ++w) {
-            fold(M[0], S[0], red[w][0], red[w][1], c_hi, c_lo);
-            fold(M[1], S[1], red[w][2], red[w][3], c_hi, c_lo);
+    if (warp == 0) {
+        const bool have = lane < kWarps;
+        m[0] = have ? red[lane][0] : kNegInf;
+        s[0] = have ? red[lane][1] : 0.f;
+        m[1] = have ? red[lane][2] : kNegInf;
+        s[1] = have ? red[lane][3] : 0.f;
+#pragma unroll
+        for (int off = kWarps / 2; off > 0; off >>= 1) {
+#pragma unroll
+            for (int r = 0; r < 2; ++r) {
+                const float m2 = __shfl_xor_sync(0xffffffffu, m[r], off);
+                const float s2 = __shfl_xor_sync(0xffffffffu, s[r], off);
+                fold(m[r], s[r], m2, s2, c_hi, c_lo);
+            }
         }
-        m[0] = M[0];
-        s[0] = S[0];
-        m[1] = M[1];
-        s[1] = S[1];
     }
-    __syncthreads();
+}
+
+// Cluster fold of the CTAs' (m, s) pairs for two rows: lane r of warp 0
+// reads rank r's pairs from distributed shared memory, then an xor butterfly
+// in a fixed order.  Every CTA folds the same values in the same order, so
+// lane 0 of every CTA holds bit-identical results.  Warp 0 only.
+__device__ __forceinline__ void cluster_fold2(cg::cluster_group& cl, const float* mine, int n_ranks,
+                                              float c_hi, float c_lo, float (&M)[2], float (&S)[2]) {
+    const int lane = threadIdx.x & 31;
+    M[0] = M[1] = kNegInf;
+    S[0] = S[1] = 0.f;
+    if (lane < n_ranks) {
+        const float4 v = *reinterpret_cast<const float4*>(cl.map_shared_rank(mine, lane));
+        M[0] = v.x;
+        S[0] = v.y;
+        M[1] = v.z;
+        S[1] = v.w;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+            const float m2 = __shfl_xor_sync(0xffffffffu, M[r], off);
+            const float s2 = __shfl_xor_sync(0xffffffffu, S[r], off);
+            fold(M[r], S[r], m2, s2, c_hi, c_lo);
+        }
+    }
 }
 
 // Block-wide inclusive scan of one float per thread (fixed order).  Returns
@@ -322,7 +355,7 @@ __global__ void __launch_bounds__(kThreads) spec_accept_kernel(const AcceptParam
     const float* u = p.uniforms + (size_t)b * (k + 1);
     const float c_hi = p.c_hi, c_lo = p.c_lo;
 
-    __shared__ float xch[2][4];          // this CTA's contribution to the current exchange
+    __shared__ __align__(16) float xch[2][4];   // this CTA's contribution to the current exchange
     __shared__ float red[kWarps][4];
     __shared__ float wsum[2 * kWarps + 1];
     __shared__ float bc[8];              // values broadcast by thread 0
@@ -335,6 +368,7 @@ __global__ void __launch_bounds__(kThreads) spec_accept_kernel(const AcceptParam
         for (int i = 0; i <= k; ++i) {
             const T* row = tgt + (size_t)i * V;
             const bool vec = aligned16(row);
+            const int x_i = (threadIdx.x == 0 && i < k) ? __ldg(x + i) : -1;
             float best = kNegInf;
             int bi = INT_MAX;
             const int ng = c1 > c0 ? (c1 - c0 + kGroup - 1) / kGroup : 0;
@@ -372,34 +406,48 @@ __global__ void __launch_bounds__(kThreads) spec_accept_kernel(const AcceptParam
                 red[threadIdx.x >> 5][1] = __int_as_float(bi);
             }
             __syncthreads();
-            if (threadIdx.x == 0) {
-                for (int w = 1; w < kWarps; ++w) {
-                    const float b2 = red[w][0];
-                    const int i2 = __float_as_int(red[w][1]);
+            if (threadIdx.x < 32) {
+                const int lane = threadIdx.x;
+                best = lane < kWarps ? red[lane][0] : kNegInf;
+                bi = lane < kWarps ? __float_as_int(red[lane][1]) : INT_MAX;
+#pragma unroll
+                for (int off = kWarps / 2; off > 0; off >>= 1) {
+                    const float b2 = __shfl_xor_sync(0xffffffffu, best, off);
+                    const int i2 = __shfl_xor_sync(0xffffffffu, bi, off);
                     if (b2 > best || (b2 == best && i2 < bi)) {
                         best = b2;
                         bi = i2;
                     }
                 }
-                xch[epoch & 1][0] = best;
-                xch[epoch & 1][1] = __int_as_float(bi);
+                if (lane == 0) {
+                    xch[epoch & 1][0] = best;
+                    xch[epoch & 1][1] = __int_as_float(bi);
+                }
             }
             cl.sync();
-            if (threadIdx.x == 0) {
+            if (threadIdx.x < 32) {
+                const int lane = threadIdx.x;
                 float gb = kNegInf;
                 int gidx = INT_MAX;
-                for (int r = 0; r < n_ranks; ++r) {
-                    const float* rx = cl.map_shared_rank(&xch[epoch & 1][0], r);
-                    const float b2 = rx[0];
-                    const int i2 = __float_as_int(rx[1]);
+                if (lane < n_ranks) {
+                    const float* rx = cl.map_shared_rank(&xch[epoch & 1][0], lane);
+                    gb = rx[0];
+                    gidx = __float_as_int(rx[1]);
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1) {
+                    const float b2 = __shfl_xor_sync(0xffffffffu, gb, off);
+                    const int i2 = __shfl_xor_sync(0xffffffffu, gidx, off);
                     if (b2 > gb || (b2 == gb && i2 < gidx)) {
                         gb = b2;
                         gidx = i2;
                     }
                 }
-                if (gidx == INT_MAX) gidx = 0;   // a row with no finite entry
-                bci[0] = gidx;
-                bci[1] = (i == k || __ldg(x + i) != gidx) ? 1 : 0;
+                if (lane == 0) {
+                    if (gidx == INT_MAX) gidx = 0;   // a row with no finite entry
+                    bci[0] = gidx;
+                    bci[1] = (i == k || x_i != gidx) ? 1 : 0;
+                }
             }
             __syncthreads();
             ++epoch;
@@ -426,6 +474,17 @@ __global__ void __launch_bounds__(kThreads) spec_accept_kernel(const AcceptParam
     int a = k;
     for (int i = 0; i <= k; ++i) {
         const bool two = i < k;
+        // thread 0 fetches what the accept test needs while the slice streams
+        int xi = -1;
+        float zt_x = 0.f, zd_x = 0.f, ui = 0.f;
+        if (threadIdx.x == 0 && two) {
+            xi = __ldg(x + i);
+            ui = __ldg(u + i);
+            if (xi >= 0 && xi < V) {
+                zt_x = to_f(tgt[(size_t)i * V + xi]);
+                zd_x = to_f(drf[(size_t)i * V + xi]);
+            }
+        }
         float m[2], s[2];
         slice_stats(tgt + (size_t)i * V, two ? drf + (size_t)i * V : tgt, two, c0, c1, c_hi, m, s);
         block_fold2(m, s, c_hi, c_lo, red);
@@ -436,44 +495,34 @@ __global__ void __launch_bounds__(kThreads) spec_accept_kernel(const AcceptParam
             xch[epoch & 1][3] = s[1];
         }
         cl.sync();
-        if (threadIdx.x == 0) {
-            float M[2] = {kNegInf, kNegInf}, S[2] = {0.f, 0.f};
-            for (int r = 0; r < n_ranks; ++r) {
-                const float* rx = cl.map_shared_rank(&xch[epoch & 1][0], r);
-                fold(M[0], S[0], rx[0], rx[1], c_hi, c_lo);
-                fold(M[1], S[1], rx[2], rx[3], c_hi, c_lo);
-            }
-            bc[0] = M[0];
-            bc[1] = S[0];
-            bc[2] = M[1];
-            bc[3] = S[1];
-            int reject = 0;
-            if (two) {
-                const int xi = __ldg(x + i);
-                if (xi < 0 || xi >= V) {
-                    reject = 1;
-                } else {
-                    // log2 p(x)/q(x) = ((zt - mt) - (zd - md)) c + log2 Sd - log2 St,
-                    // carried as an unevaluated float pair
-                    const float zt = to_f(tgt[(size_t)i * V + xi]);
-                    const float zd = to_f(drf[(size_t)i * V + xi]);
-                    float ratio;
-                    if (zt == kNegInf) {
-                        ratio = 0.f;
+        if (threadIdx.x < 32) {
+            float M[2], S[2];
+            cluster_fold2(cl, &xch[epoch & 1][0], n_ranks, c_hi, c_lo, M, S);
+            if (threadIdx.x == 0) {
+                bc[0] = M[0];
+                bc[1] = S[0];
+                bc[2] = M[1];
+                bc[3] = S[1];
+                int reject = 0;
+                if (two) {
+                    if (xi < 0 || xi >= V || zt_x == kNegInf) {
+                        reject = 1;
                     } else {
-                        const float dz = (zt - M[0]) - (zd - M[1]);
+                        // log2 p(x)/q(x) = ((zt - mt) - (zd - md)) c + log2 Sd - log2 St,
+                        // carried as an unevaluated float pair
+                        const float dz = (zt_x - M[0]) - (zd_x - M[1]);
                         const float A = dz * c_hi;
                         float E = fmaf(dz, c_lo, fmaf(dz, c_hi, -A));
                         const float Bl = lg2(S[1]) - lg2(S[0]);
                         const float H = A + Bl;
                         const float bb = H - A;
                         E += (A - (H - bb)) + (Bl - bb);
-                        ratio = ex2(H) * fmaf(E, kLn2, 1.f);
+                        const float ratio = ex2(H) * fmaf(E, kLn2, 1.f);
+                        reject = !(ui < ratio);
                     }
-                    reject = !(__ldg(u + i) < ratio);
                 }
+                bci[0] = reject;
             }
-            bci[0] = reject;
         }
         __syncthreads();
         ++epoch;
@@ -499,37 +548,45 @@ __global__ void __launch_bounds__(kThreads) spec_accept_kernel(const AcceptParam
         const float mass = draw_scan(rt, rd, c0, c1, w, c_hi, c_lo, false, 0.f, 0.f, &s_found, wsum);
         if (threadIdx.x == 0) xch[epoch & 1][0] = mass;
         cl.sync();
-        if (threadIdx.x == 0) {
-            float Z = 0.f;
-            for (int r = 0; r < n_ranks; ++r) Z += *cl.map_shared_rank(&xch[epoch & 1][0], r);
-            int retry = 0, own = -1, lastp = -1;
+        if (threadIdx.x < 32) {
+            // lane r holds rank r's mass; an inclusive scan in a fixed order
+            // gives every CTA the same cumulative masses
+            const int lane = threadIdx.x;
+            const float Mr = lane < n_ranks ? *cl.map_shared_rank(&xch[epoch & 1][0], lane) : 0.f;
+            float incl = Mr;
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const float y = __shfl_up_sync(0xffffffffu, incl, off);
+                if (lane >= off) incl += y;
+            }
+            const float Z = __shfl_sync(0xffffffffu, incl, 31);
+            const float excl = incl - Mr;   // only used as the owner's base (see below)
+            const float up = __shfl_up_sync(0xffffffffu, incl, 1);
+            const float base_l = lane == 0 ? 0.f : up;
+            (void)excl;
+            int retry = 0, own = -1;
             float base = 0.f, t = 0.f;
             if (!(Z > 0.f)) {
                 retry = 1;   // p == q up to rounding: fall back to p of the same row
             } else {
                 t = __ldg(u + k) * Z;
-                float P = 0.f;
-                for (int r = 0; r < n_ranks; ++r) {
-                    const float Mr = *cl.map_shared_rank(&xch[epoch & 1][0], r);
-                    if (Mr > 0.f) {
-                        if (own < 0 && P + Mr > t) {
-                            own = r;
-                            base = P;
-                        }
-                        lastp = r;
-                    }
-                    P = P + Mr;
-                }
-                if (own < 0) {   // u*Z at or past the total through rounding
-                    own = lastp;
+                const unsigned cross = __ballot_sync(0xffffffffu, lane < n_ranks && Mr > 0.f && incl > t);
+                const unsigned pos = __ballot_sync(0xffffffffu, lane < n_ranks && Mr > 0.f);
+                if (cross) {
+                    own = __ffs(cross) - 1;
+                    base = __shfl_sync(0xffffffffu, base_l, own);
+                } else {   // u*Z at or past the total through rounding
+                    own = 31 - __clz(pos);
                     base = 0.f;
                     t = __int_as_float(0x7f800000);
                 }
             }
-            bci[0] = retry;
-            bci[1] = own;
-            bc[4] = base;
-            bc[5] = t;
+            if (lane == 0) {
+                bci[0] = retry;
+                bci[1] = own;
+                bc[4] = base;
+                bc[5] = t;
+            }
         }
         __syncthreads();
         ++epoch;
@@ -589,8 +646,15 @@ template <typename T, bool G>
 cs_status launch_typed(AcceptParams p, int cluster, int batch, cudaStream_t stream) {
     auto kern = spec_accept_kernel<T, G>;
     if (cluster > 8) {
-        const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-        if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(non-portable cluster)");
+        static bool done[64] = {};
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (dev < 0 || dev >= 64 || !done[dev]) {
+            const cudaError_t e =
+                cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+            if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(non-portable cluster)");
+            if (dev >= 0 && dev < 64) done[dev] = true;
+        }
     }
     for (int b0 = 0; b0 < batch; b0 += 65535) {
         p.b_base = b0;

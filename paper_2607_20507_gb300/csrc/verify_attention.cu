@@ -2,20 +2,26 @@
 // cache (the KV-bound core of the target's verify pass in the paper's
 // draft-and-verify step, Sec. 3.4).
 //
-// Work decomposition (flash-decoding style split-KV):
-//   one CTA = (request b, KV head h, split s) over keys [s*C, min((s+1)*C, L_b)).
-//   The (k+1)*G query rows that read KV head h (draft row i = r / G, query
-//   head h*G + r % G) are packed into one tile, 16 rows per consumer warp, so
-//   every K/V byte staged in shared memory serves all of them.
-// Pipeline: one producer warp streams 64-token K and V tiles of the pages
-//   through TMA (128-byte swizzle) into a 3-stage shared-memory ring guarded
-//   by mbarriers; consumer warps run S = Q K^T and O += P V on bf16 tensor
-//   cores (mma.sync m16n8k16, fp32 accumulate) with an fp32 online softmax in
-//   the log2 domain.
-// Splits: a request whose context needs one split writes bf16 output
-//   directly; otherwise every split writes (O, m, l) partials to the
-//   workspace and the last CTA to finish (an atomic ticket that wraps back
-//   to zero, no spin-wait) merges them with log-sum-exp weights.
+// Schedule (persistent, balanced).  The work is the flattened sequence of
+// 64-key tiles of every (request b, KV head h) span, requests in order, heads
+// in order, tiles in key order; span (b, h) has T_b = ceil(L_b / 64) tiles.
+// The grid holds exactly as many CTAs as are resident at once, and CTA c
+// takes the contiguous tile range [c*W/G, (c+1)*W/G) of the W tiles, so every
+// CTA streams the same number of tiles whatever the context lengths.  A span
+// that lies inside one CTA's range is finished there and written in bf16;
+// a span cut by range boundaries leaves one (O, m, l) partial per piece (each
+// CTA writes at most two: its first and its last piece), and a second small
+// kernel merges the pieces of every cut span with log-sum-exp weights, all
+// spans in parallel.
+//
+// Per CTA: one producer warp streams the K and V tiles of its range through
+// TMA (one 4-D tensor map over the page pool, 128-byte swizzle, one box per
+// page piece) into a 3-stage shared-memory ring guarded by mbarriers, without
+// draining between spans.  Consumer warps own 16 of the (k+1)*G query rows of
+// the current span each (draft row i = r / G, query head h*G + r % G), so
+// every K/V byte staged in shared memory serves all rows; they run S = Q K^T
+// and O += P V on bf16 tensor cores (mma.sync m16n8k16, fp32 accumulate) with
+// an fp32 online softmax in the log2 domain.
 #include <math.h>
 #include <stdio.h>
 
@@ -34,24 +40,66 @@ constexpr int kTensorTileBytes = 2 * kHalfBytes;
 constexpr int kStageBytes = 2 * kTensorTileBytes;   // K + V
 constexpr int kStages = 3;
 constexpr int kMaxRowWarps = 9;               // 144 query rows
-constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 128 /*barriers*/;
+constexpr int kMaxBatchPerLaunch = 1024;      // requests whose schedule one launch holds
+constexpr int kMaxGrid = 512;                 // persistent CTAs at most (slot list size)
+constexpr int kMinTilesPerCta = 8;            // 256 KB of K/V per CTA before a span is cut
+constexpr int kBarrierBytes = 128;
+constexpr int kSmemBytes = kStages * kStageBytes + kBarrierBytes +
+                           (kMaxBatchPerLaunch + 1) * 8 /*prefix*/ + kMaxBatchPerLaunch * 4 /*L*/ +
+                           1024 /*alignment slack*/;
 
 struct AttnParams {
     const __nv_bfloat16* q;      // [B, R, Hq, D]
     __nv_bfloat16* out;          // [B, R, Hq, D]
     const int32_t* page_table;   // [B, max_pages]
     const int32_t* ctx_lens;     // [B]
-    float* part_o;               // [B, Hkv, ns_max, n_rows, D]
-    float2* part_ml;             // [B, Hkv, ns_max, n_rows]  (m in log2 units, l)
-    unsigned int* tickets;       // [B, Hkv]
+    float* part_o;               // [2 * grid, n_rows, D]
+    float2* part_ml;             // [2 * grid, n_rows]  (m in log2 units, l)
     int* status;
-    int Hq, Hkv, G, R, n_rows, ps, box_t, max_pages, chunk, ns_max, row_warps;
-    int b_base;                  // first request of this launch (grids hold <= 65535 requests)
+    int Hq, Hkv, G, R, n_rows, ps, box_t, max_pages, row_warps;
+    int b_base, n_batch;         // requests [b_base, b_base + n_batch) in this launch
     float scale_log2;            // sm_scale * log2(e)
 };
 
 __device__ __forceinline__ void flag_timeout(int* status) {
     atomicOr(status, CS_DEVICE_WAIT_TIMEOUT);
+}
+
+__device__ __forceinline__ int tiles_of(int L) { return max(1, (L + kTileT - 1) / kTileT); }
+
+// The CTA whose tile range holds flat tile f (ranges start at floor(c*W/G)).
+__device__ __forceinline__ int owner_of(long long f, long long W, int G) {
+    return (int)(((f + 1) * G + W - 1) / W) - 1;
+}
+
+// Position of flat tile f in the schedule: request (launch-local), head, tile.
+struct Cursor {
+    int b, h, t, T;
+};
+
+__device__ __forceinline__ Cursor locate(long long f, const long long* prefix, const int* lens,
+                                         int n_batch, int Hkv) {
+    int lo = 0, hi = n_batch - 1;   // largest b with prefix[b] <= f
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (prefix[mid] <= f) lo = mid;
+        else hi = mid - 1;
+    }
+    Cursor c;
+    c.b = lo;
+    c.T = tiles_of(lens[lo]);
+    const long long local = f - prefix[lo];
+    c.h = (int)(local / c.T);
+    c.t = (int)(local % c.T);
+    return c;
+}
+
+__device__ __forceinline__ void advance(Cursor& c, const int* lens, int n_batch, int Hkv) {
+    if (++c.t < c.T) return;
+    c.t = 0;
+    if (++c.h < Hkv) return;
+    c.h = 0;
+    if (++c.b < n_batch) c.T = tiles_of(lens[c.b]);
 }
 
 __global__ void __launch_bounds__((kMaxRowWarps + 1) * 32, 1)
@@ -62,294 +110,429 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
     uint64_t* empty = full + kStages;
-    __shared__ int s_last;
-    __shared__ int s_abort;
-
-    const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z + p.b_base;
-    int L = __ldg(p.ctx_lens + b);
-    L = max(0, min(L, p.max_pages * p.ps));
-    const int ns = max(1, (L + p.chunk - 1) / p.chunk);
-    if (split >= ns) return;
-    const int t_begin = split * p.chunk;
-    const int t_end = min(L, t_begin + p.chunk);
-    const int n_tiles = t_end > t_begin ? (t_end - t_begin + kTileT - 1) / kTileT : 0;
+    long long* s_prefix = reinterpret_cast<long long*>(smem + kStages * kStageBytes + kBarrierBytes);
+    int* s_len = reinterpret_cast<int*>(s_prefix + kMaxBatchPerLaunch + 1);
+    __shared__ long long s_wtot[kMaxRowWarps + 1];
+    __shared__ long long s_carry;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nw = p.row_warps;
+    const int nb = p.n_batch;
 
+    // ---- schedule: exclusive prefix of tiles per request (x heads), clamped L
     if (threadIdx.x == 0) {
+        s_carry = 0;
         for (int i = 0; i < kStages; ++i) {
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], nw);
         }
-        s_abort = 0;
         fence_barrier_init();
     }
     __syncthreads();
+    const int l_cap = p.max_pages * p.ps;
+    for (int base = 0; base < nb; base += blockDim.x) {
+        const int bl = base + threadIdx.x;
+        long long v = 0;
+        if (bl < nb) {
+            int L = __ldg(p.ctx_lens + p.b_base + bl);
+            L = max(0, min(L, l_cap));
+            s_len[bl] = L;
+            v = (long long)tiles_of(L) * p.Hkv;
+        }
+        long long inc = v;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const long long y = __shfl_up_sync(0xffffffffu, inc, off);
+            if (lane >= off) inc += y;
+        }
+        if (lane == 31) s_wtot[warp] = inc;
+        __syncthreads();
+        long long before = s_carry;
+        for (int w = 0; w < warp; ++w) before += s_wtot[w];
+        if (bl < nb) s_prefix[bl] = before + inc - v;
+        __syncthreads();
+        if (threadIdx.x == blockDim.x - 1) s_carry = before + inc;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) s_prefix[nb] = s_carry;
+    __syncthreads();
 
+    const long long W = s_prefix[nb];
+    // at least kMinTilesPerCta tiles per CTA: small problems use fewer CTAs
+    // rather than cutting every span into one-tile pieces
+    const long long g_need = (W + kMinTilesPerCta - 1) / kMinTilesPerCta;
+    const int Gc = (int)(g_need < (long long)gridDim.x ? (g_need > 0 ? g_need : 1) : gridDim.x);
+    const int cta = blockIdx.x;
+    if (cta >= Gc) return;
+    const long long f0 = (long long)cta * W / Gc, f1 = (long long)(cta + 1) * W / Gc;
+    if (f0 >= f1) return;
+    const int n_tiles = (int)(f1 - f0);
     const uint32_t smem_base = smem_u32(smem);
 
     if (warp == nw) {
         // ------------------------------------------------------ producer
-        if (lane == 0 && n_tiles > 0) {
+        // The whole warp produces: lane pc owns page piece pc of a tile (its
+        // page id is loaded one tile ahead, so the table lookups of all pieces
+        // overlap each other and the previous tile), lane 0 arms the stage's
+        // barrier, and every lane issues the TMA copies of its own piece.
+        if (lane == 0) {
             tma_prefetch_desc(&tmap_k);
             tma_prefetch_desc(&tmap_v);
-            const int pieces = kTileT / p.box_t;
-            const uint32_t piece_bytes = (uint32_t)p.box_t * 128u;
-            const int32_t* table = p.page_table + (size_t)b * p.max_pages;
-            for (int t = 0; t < n_tiles; ++t) {
-                const int st = t % kStages;
-                const uint32_t use = (uint32_t)(t / kStages);
-                if (t >= kStages && !mbar_wait_bounded(&empty[st], (use - 1) & 1)) {
-                    flag_timeout(p.status);
-                    s_abort = 1;
-                    break;
-                }
-                const int ts = t_begin + t * kTileT;
-                int valid = 0;
-                for (int pc = 0; pc < pieces; ++pc)
-                    if (ts + pc * p.box_t < t_end) ++valid;
-                mbar_arrive_expect_tx(&full[st], (uint32_t)valid * piece_bytes * 4u);
-                const uint32_t kdst = smem_base + st * kStageBytes;
+        }
+        const int pieces = kTileT / p.box_t;
+        const uint32_t piece_bytes = (uint32_t)p.box_t * 128u;
+        Cursor cur = locate(f0, s_prefix, s_len, nb, p.Hkv);
+        auto piece_page = [&](const Cursor& cc) -> int {
+            const int tok = cc.t * kTileT + lane * p.box_t;
+            if (lane >= pieces || tok >= s_len[cc.b]) return -1;
+            return __ldg(p.page_table + (size_t)(p.b_base + cc.b) * p.max_pages + tok / p.ps);
+        };
+        int page_next = piece_page(cur);
+        for (int j = 0; j < n_tiles; ++j) {
+            const int st = j % kStages;
+            const uint32_t use = (uint32_t)(j / kStages);
+            const int page = page_next;
+            const int L = s_len[cur.b];
+            const int ts = cur.t * kTileT;
+            const int h_cur = cur.h;
+            advance(cur, s_len, nb, p.Hkv);
+            if (j + 1 < n_tiles) page_next = piece_page(cur);
+            int ok = 1;
+            if (lane == 0 && j >= kStages && !mbar_wait_bounded(&empty[st], (use - 1) & 1)) {
+                flag_timeout(p.status);
+                ok = 0;
+            }
+            if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+            int valid = 0;
+            for (int pc = 0; pc < pieces; ++pc)
+                if (ts + pc * p.box_t < L) ++valid;
+            if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)valid * piece_bytes * 4u);
+            __syncwarp();
+            if (lane < valid) {
+                const uint32_t kdst = smem_base + st * kStageBytes + (uint32_t)lane * piece_bytes;
                 const uint32_t vdst = kdst + kTensorTileBytes;
-                for (int pc = 0; pc < valid; ++pc) {
-                    const int tok = ts + pc * p.box_t;
-                    const int page = __ldg(table + tok / p.ps);
-                    const int slot = tok % p.ps;
-                    const uint32_t off = (uint32_t)pc * piece_bytes;
+                const int slot = (ts + lane * p.box_t) % p.ps;
 #pragma unroll
-                    for (int hh = 0; hh < 2; ++hh) {
-                        tma_load_4d(kdst + hh * kHalfBytes + off, &tmap_k, &full[st], hh * 64, slot,
-                                    h, page);
-                        tma_load_4d(vdst + hh * kHalfBytes + off, &tmap_v, &full[st], hh * 64, slot,
-                                    h, page);
-                    }
+                for (int hh = 0; hh < 2; ++hh) {
+                    tma_load_4d(kdst + hh * kHalfBytes, &tmap_k, &full[st], hh * 64, slot, h_cur, page);
+                    tma_load_4d(vdst + hh * kHalfBytes, &tmap_v, &full[st], hh * 64, slot, h_cur, page);
                 }
             }
         }
-    } else {
-        // ------------------------------------------------------ consumers
-        const int g = lane >> 2, tq = lane & 3;
-        const int row0 = warp * 16 + g, row1 = row0 + 8;
-        // Q fragments (A operand, 16 rows x 128 dims) straight from global memory.
-        uint32_t qa[8][4];
-        {
-            const __nv_bfloat16* qr[2] = {nullptr, nullptr};
-            const int rr[2] = {row0, row1};
+        return;
+    }
+
+    // ---------------------------------------------------------- consumers
+    const int g = lane >> 2, tq = lane & 3;
+    const int row0 = warp * 16 + g, row1 = row0 + 8;
+    const int lm = lane >> 3, lr = lane & 7;   // ldmatrix: matrix index, row within it
+    const float c = p.scale_log2;
+
+    Cursor cur = locate(f0, s_prefix, s_len, nb, p.Hkv);
+    int seg_t0 = cur.t;
+    bool first_seg = true;
+
+    uint32_t qa[8][4];
+    float o[16][4];
+    float m_raw[2], l[2];
+    int lim0 = 0, lim1 = 0;
+
+    auto begin_span = [&](const Cursor& cc) {
+        const int bg = p.b_base + cc.b;
 #pragma unroll
-            for (int k = 0; k < 2; ++k) {
-                if (rr[k] < p.n_rows) {
-                    const int i = rr[k] / p.G, gi = rr[k] % p.G;
-                    qr[k] = p.q + (((size_t)b * p.R + i) * p.Hq + (size_t)h * p.G + gi) * kD;
-                }
+        for (int k = 0; k < 2; ++k) {
+            const int r = k ? row1 : row0;
+            const __nv_bfloat16* qr = nullptr;
+            if (r < p.n_rows) {
+                const int i = r / p.G, gi = r % p.G;
+                qr = p.q + (((size_t)bg * p.R + i) * p.Hq + (size_t)cc.h * p.G + gi) * kD;
             }
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk) {
-                const int c = kk * 16 + tq * 2;
-                qa[kk][0] = qr[0] ? __ldg(reinterpret_cast<const uint32_t*>(qr[0] + c)) : 0u;
-                qa[kk][1] = qr[1] ? __ldg(reinterpret_cast<const uint32_t*>(qr[1] + c)) : 0u;
-                qa[kk][2] = qr[0] ? __ldg(reinterpret_cast<const uint32_t*>(qr[0] + c + 8)) : 0u;
-                qa[kk][3] = qr[1] ? __ldg(reinterpret_cast<const uint32_t*>(qr[1] + c + 8)) : 0u;
+                const int col = kk * 16 + tq * 2;
+                qa[kk][k] = qr ? __ldg(reinterpret_cast<const uint32_t*>(qr + col)) : 0u;
+                qa[kk][2 + k] = qr ? __ldg(reinterpret_cast<const uint32_t*>(qr + col + 8)) : 0u;
             }
         }
-        // exclusive key limit of each of this thread's two rows
-        const int lim0 = row0 < p.n_rows ? min(t_end, L - p.R + 1 + row0 / p.G) : t_end;
-        const int lim1 = row1 < p.n_rows ? min(t_end, L - p.R + 1 + row1 / p.G) : t_end;
-        const int lim_min = min(lim0, lim1);
-        const float c = p.scale_log2;
-
-        float o[16][4];
 #pragma unroll
         for (int i = 0; i < 16; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-        float m_raw[2] = {kNegInf, kNegInf};
-        float l[2] = {0.f, 0.f};
+        m_raw[0] = m_raw[1] = kNegInf;
+        l[0] = l[1] = 0.f;
+        const int L = s_len[cc.b];
+        // exclusive key limit of each of this thread's two rows
+        lim0 = row0 < p.n_rows ? L - p.R + 1 + row0 / p.G : L;
+        lim1 = row1 < p.n_rows ? L - p.R + 1 + row1 / p.G : L;
+    };
+    begin_span(cur);
 
-        // per-lane ldmatrix address pieces: matrix index and row within it
-        const int lm = lane >> 3, lr = lane & 7;
-
-        for (int t = 0; t < n_tiles; ++t) {
-            const int st = t % kStages;
-            const uint32_t use = (uint32_t)(t / kStages);
-            if (!mbar_wait_bounded(&full[st], use & 1)) {
-                flag_timeout(p.status);
-                s_abort = 1;
-                break;
+    for (int j = 0; j < n_tiles; ++j) {
+        const int st = j % kStages;
+        const uint32_t use = (uint32_t)(j / kStages);
+        if (!mbar_wait_bounded(&full[st], use & 1)) {
+            flag_timeout(p.status);
+            break;
+        }
+        const int L = s_len[cur.b];
+        const int ts = cur.t * kTileT;
+        const uint32_t kb = smem_base + st * kStageBytes;
+        const uint32_t vb = kb + kTensorTileBytes;
+        if (ts + kTileT > L) {
+            // keys past L_b (pages not loaded, or slots past the context) may
+            // hold any bits: zero their V rows so that P = 0 cannot meet NaN
+            const int first = max(0, L - ts);
+            uint8_t* vrow = smem + st * kStageBytes + kTensorTileBytes;
+            for (int idx = lane; idx < (kTileT - first) * 16; idx += 32) {
+                const int r = first + (idx >> 4), ch = idx & 15;
+                *reinterpret_cast<uint4*>(vrow + (ch >> 3) * kHalfBytes + r * 128 + (ch & 7) * 16) =
+                    make_uint4(0, 0, 0, 0);
             }
-            const int ts = t_begin + t * kTileT;
-            const uint32_t kb = smem_base + st * kStageBytes;
-            const uint32_t vb = kb + kTensorTileBytes;
-            if (ts + kTileT > t_end) {
-                // keys past the split (pages not loaded, or slots past L_b) may
-                // hold any bits: zero their V rows so that P = 0 cannot meet NaN
-                const int first = t_end - ts;
-                uint8_t* vrow = smem + st * kStageBytes + kTensorTileBytes;
-                for (int idx = lane; idx < (kTileT - first) * 16; idx += 32) {
-                    const int r = first + (idx >> 4), ch = idx & 15;
-                    *reinterpret_cast<uint4*>(vrow + (ch >> 3) * kHalfBytes + r * 128 +
-                                              (ch & 7) * 16) = make_uint4(0, 0, 0, 0);
-                }
-                __syncwarp();
-            }
-
-            // ---- S = Q K^T over 64 keys: 8 n-tiles of 8 keys
-            float sc[8][4];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-                const uint32_t half = kb + (kk >> 2) * kHalfBytes;
-#pragma unroll
-                for (int np = 0; np < 4; ++np) {
-                    const int key = (2 * np + (lm >> 1)) * 8 + lr;
-                    const int ch = (kk & 3) * 2 + (lm & 1);
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4(half + key * 128 + ((ch ^ (key & 7)) << 4), b0, b1, b2, b3);
-                    mma_bf16_16816(sc[2 * np], qa[kk], b0, b1);
-                    mma_bf16_16816(sc[2 * np + 1], qa[kk], b2, b3);
-                }
-            }
-            // ---- causal-verify mask and split end
-            if (ts + kTileT > lim_min) {
-#pragma unroll
-                for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int key = ts + nt * 8 + tq * 2 + e;
-                        if (key >= lim0) sc[nt][e] = kNegInf;
-                        if (key >= lim1) sc[nt][2 + e] = kNegInf;
-                    }
-                }
-            }
-            // ---- online softmax (log2 domain)
-#pragma unroll
-            for (int rh = 0; rh < 2; ++rh) {
-                float mx = kNegInf;
-#pragma unroll
-                for (int nt = 0; nt < 8; ++nt) mx = fmaxf(mx, fmaxf(sc[nt][2 * rh], sc[nt][2 * rh + 1]));
-                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-                mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-                const float m_new = fmaxf(m_raw[rh], mx);
-                const float m_use = m_new == kNegInf ? 0.f : m_new;
-                const float alpha = ex2((m_raw[rh] - m_use) * c);
-                m_raw[rh] = m_new;
-                const float neg = -m_use * c;
-                float rs = 0.f;
-#pragma unroll
-                for (int nt = 0; nt < 8; ++nt) {
-                    const float p0 = ex2(fmaf(sc[nt][2 * rh], c, neg));
-                    const float p1 = ex2(fmaf(sc[nt][2 * rh + 1], c, neg));
-                    sc[nt][2 * rh] = p0;
-                    sc[nt][2 * rh + 1] = p1;
-                    rs += p0 + p1;
-                }
-                l[rh] = l[rh] * alpha + rs;
-#pragma unroll
-                for (int dn = 0; dn < 16; ++dn) {
-                    o[dn][2 * rh] *= alpha;
-                    o[dn][2 * rh + 1] *= alpha;
-                }
-            }
-            // ---- O += P V over the 64 keys: 4 k-steps of 16 keys
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk) {
-                uint32_t a[4];
-                a[0] = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
-                a[1] = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
-                a[2] = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-                a[3] = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
-                const int key = kk * 16 + (lm & 1) * 8 + lr;
-#pragma unroll
-                for (int dp = 0; dp < 8; ++dp) {
-                    const int dblk = 2 * dp + (lm >> 1);
-                    const int ch = dblk & 7;
-                    uint32_t b0, b1, b2, b3;
-                    ldsm_x4_trans(vb + (dblk >> 3) * kHalfBytes + key * 128 + ((ch ^ (key & 7)) << 4),
-                                  b0, b1, b2, b3);
-                    mma_bf16_16816(o[2 * dp], a, b0, b1);
-                    mma_bf16_16816(o[2 * dp + 1], a, b2, b3);
-                }
-            }
-            // generic-proxy writes (the zeroed rows) must be ordered before the
-            // next TMA write into this stage
-            if (ts + kTileT > t_end) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[st]);
         }
 
-        // ---- epilogue of this warp's 16 rows
-        if (!s_abort) {
+        // ---- S = Q K^T over 64 keys: 8 n-tiles of 8 keys
+        float sc[8][4];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t half = kb + (kk >> 2) * kHalfBytes;
+#pragma unroll
+            for (int np = 0; np < 4; ++np) {
+                const int key = (2 * np + (lm >> 1)) * 8 + lr;
+                const int ch = (kk & 3) * 2 + (lm & 1);
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4(half + key * 128 + ((ch ^ (key & 7)) << 4), b0, b1, b2, b3);
+                mma_bf16_16816(sc[2 * np], qa[kk], b0, b1);
+                mma_bf16_16816(sc[2 * np + 1], qa[kk], b2, b3);
+            }
+        }
+        // ---- causal-verify mask (and the context end)
+        if (ts + kTileT > min(lim0, lim1)) {
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int key = ts + nt * 8 + tq * 2 + e;
+                    if (key >= lim0) sc[nt][e] = kNegInf;
+                    if (key >= lim1) sc[nt][2 + e] = kNegInf;
+                }
+            }
+        }
+        // ---- online softmax (log2 domain)
+#pragma unroll
+        for (int rh = 0; rh < 2; ++rh) {
+            float mx = kNegInf;
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) mx = fmaxf(mx, fmaxf(sc[nt][2 * rh], sc[nt][2 * rh + 1]));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+            const float m_new = fmaxf(m_raw[rh], mx);
+            const float m_use = m_new == kNegInf ? 0.f : m_new;
+            const float alpha = ex2((m_raw[rh] - m_use) * c);
+            m_raw[rh] = m_new;
+            const float neg = -m_use * c;
+            float rs = 0.f;
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                const float p0 = ex2(fmaf(sc[nt][2 * rh], c, neg));
+                const float p1 = ex2(fmaf(sc[nt][2 * rh + 1], c, neg));
+                sc[nt][2 * rh] = p0;
+                sc[nt][2 * rh + 1] = p1;
+                rs += p0 + p1;
+            }
+            l[rh] = l[rh] * alpha + rs;
+#pragma unroll
+            for (int dn = 0; dn < 16; ++dn) {
+                o[dn][2 * rh] *= alpha;
+                o[dn][2 * rh + 1] *= alpha;
+            }
+        }
+        // ---- O += P V over the 64 keys: 4 k-steps of 16 keys
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+            uint32_t a[4];
+            a[0] = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
+            a[1] = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
+            a[2] = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+            a[3] = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+            const int key = kk * 16 + (lm & 1) * 8 + lr;
+#pragma unroll
+            for (int dp = 0; dp < 8; ++dp) {
+                const int dblk = 2 * dp + (lm >> 1);
+                const int ch = dblk & 7;
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4_trans(vb + (dblk >> 3) * kHalfBytes + key * 128 + ((ch ^ (key & 7)) << 4), b0,
+                              b1, b2, b3);
+                mma_bf16_16816(o[2 * dp], a, b0, b1);
+                mma_bf16_16816(o[2 * dp + 1], a, b2, b3);
+            }
+        }
+        // generic-proxy writes (the zeroed rows) must be ordered before the
+        // next TMA write into this stage
+        if (ts + kTileT > L) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[st]);
+
+        if (j + 1 < n_tiles && cur.t + 1 < cur.T) {
+            advance(cur, s_len, nb, p.Hkv);
+            continue;
+        }
+
+        // ---------------------------------------------- end of a piece of span
+        const int bg = p.b_base + cur.b;
+        const bool complete = seg_t0 == 0 && cur.t + 1 == cur.T;
+        float lt[2];
+#pragma unroll
+        for (int rh = 0; rh < 2; ++rh) {
+            lt[rh] = l[rh];
+            lt[rh] += __shfl_xor_sync(0xffffffffu, lt[rh], 1);
+            lt[rh] += __shfl_xor_sync(0xffffffffu, lt[rh], 2);
+        }
+        if (complete) {
 #pragma unroll
             for (int rh = 0; rh < 2; ++rh) {
-                float lt = l[rh];
-                lt += __shfl_xor_sync(0xffffffffu, lt, 1);
-                lt += __shfl_xor_sync(0xffffffffu, lt, 2);
                 const int row = rh ? row1 : row0;
                 if (row >= p.n_rows) continue;
-                if (ns == 1) {
-                    const float inv = lt > 0.f ? 1.f / lt : 0.f;
-                    const int i = row / p.G, gi = row % p.G;
-                    __nv_bfloat16* dst =
-                        p.out + (((size_t)b * p.R + i) * p.Hq + (size_t)h * p.G + gi) * kD + tq * 2;
+                const float inv = lt[rh] > 0.f ? 1.f / lt[rh] : 0.f;
+                const int i = row / p.G, gi = row % p.G;
+                __nv_bfloat16* dst =
+                    p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)cur.h * p.G + gi) * kD + tq * 2;
 #pragma unroll
-                    for (int dn = 0; dn < 16; ++dn)
-                        *reinterpret_cast<uint32_t*>(dst + dn * 8) =
-                            pack_bf16x2(o[dn][2 * rh] * inv, o[dn][2 * rh + 1] * inv);
-                } else {
-                    const size_t slot = ((size_t)b * p.Hkv + h) * p.ns_max + split;
-                    float* dst = p.part_o + (slot * p.n_rows + row) * kD + tq * 2;
+                for (int dn = 0; dn < 16; ++dn)
+                    *reinterpret_cast<uint32_t*>(dst + dn * 8) =
+                        pack_bf16x2(o[dn][2 * rh] * inv, o[dn][2 * rh + 1] * inv);
+            }
+        } else {
+            const size_t slot = 2 * (size_t)cta + (first_seg ? 0 : 1);
 #pragma unroll
-                    for (int dn = 0; dn < 16; ++dn)
-                        *reinterpret_cast<float2*>(dst + dn * 8) =
-                            make_float2(o[dn][2 * rh], o[dn][2 * rh + 1]);
-                    if (tq == 0)
-                        p.part_ml[slot * p.n_rows + row] =
-                            make_float2(m_raw[rh] == kNegInf ? kNegInf : m_raw[rh] * c, lt);
-                }
+            for (int rh = 0; rh < 2; ++rh) {
+                const int row = rh ? row1 : row0;
+                if (row >= p.n_rows) continue;
+                float* dst = p.part_o + (slot * p.n_rows + row) * kD + tq * 2;
+#pragma unroll
+                for (int dn = 0; dn < 16; ++dn)
+                    *reinterpret_cast<float2*>(dst + dn * 8) = make_float2(o[dn][2 * rh], o[dn][2 * rh + 1]);
+                if (tq == 0)
+                    p.part_ml[slot * p.n_rows + row] =
+                        make_float2(m_raw[rh] == kNegInf ? kNegInf : m_raw[rh] * c, lt[rh]);
             }
         }
+        if (j + 1 < n_tiles) {
+            advance(cur, s_len, nb, p.Hkv);
+            seg_t0 = cur.t;
+            first_seg = false;
+            begin_span(cur);
+        }
     }
+}
 
-    if (ns == 1) return;
+// ---------------------------------------------------------------------------
+// Merge of split spans.  Every CTA recomputes the schedule of the main kernel
+// from the context lengths, so it knows which CTAs cut its span (b, h) and in
+// which slots their pieces are; a span with a single piece was written by the
+// main kernel and is skipped.  The pieces are folded with log-sum-exp weights:
+// one warp per query row, lanes across the 128 dims (one coalesced 512-byte
+// read per piece), every piece's loads issued before any is used.
+// ---------------------------------------------------------------------------
+constexpr int kMergeThreads = 256;
+constexpr int kMergePieces = 8;   // pieces in flight per row
 
-    // ---------------------------------------------- last split merges
-    __threadfence();
+__global__ void __launch_bounds__(kMergeThreads)
+verify_attention_merge_kernel(const AttnParams p, int grid_main) {
+    __shared__ long long s_red[2][kMergeThreads / 32];
+    __shared__ int s_slots[kMaxGrid];
+    __shared__ int s_np;
+    const int h = blockIdx.x, bl = blockIdx.y;
+    const int nb = p.n_batch;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int l_cap = p.max_pages * p.ps;
+
+    // tiles before request bl, and in total (x heads)
+    long long before = 0, total = 0;
+    for (int b = threadIdx.x; b < nb; b += kMergeThreads) {
+        int L = __ldg(p.ctx_lens + p.b_base + b);
+        L = max(0, min(L, l_cap));
+        const long long v = (long long)tiles_of(L) * p.Hkv;
+        total += v;
+        if (b < bl) before += v;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        before += __shfl_xor_sync(0xffffffffu, before, off);
+        total += __shfl_xor_sync(0xffffffffu, total, off);
+    }
+    if (lane == 0) {
+        s_red[0][warp] = before;
+        s_red[1][warp] = total;
+    }
     __syncthreads();
     if (threadIdx.x == 0) {
-        int last = 0;
-        if (!s_abort) {
-            const unsigned int prev = atomicInc(p.tickets + (size_t)b * p.Hkv + h, (unsigned)(ns - 1));
-            last = prev == (unsigned)(ns - 1);
+        long long bf = 0, W = 0;
+        for (int w = 0; w < kMergeThreads / 32; ++w) {
+            bf += s_red[0][w];
+            W += s_red[1][w];
         }
-        s_last = last;
+        int L = __ldg(p.ctx_lens + p.b_base + bl);
+        L = max(0, min(L, l_cap));
+        const int T = tiles_of(L);
+        const long long g_need = (W + kMinTilesPerCta - 1) / kMinTilesPerCta;
+        const int Gc = (int)(g_need < (long long)grid_main ? (g_need > 0 ? g_need : 1) : grid_main);
+        const long long span0 = bf + (long long)h * T;
+        const int c_first = owner_of(span0, W, Gc);
+        const int c_last = owner_of(span0 + T - 1, W, Gc);
+        int n_p = 0;
+        long long start_c = (long long)c_first * W / Gc;
+        for (int cc = c_first; cc <= c_last && n_p < kMaxGrid; ++cc) {
+            const long long start_n = (long long)(cc + 1) * W / Gc;
+            if (start_n > start_c) s_slots[n_p++] = 2 * cc + ((cc == c_first && span0 > start_c) ? 1 : 0);
+            start_c = start_n;
+        }
+        s_np = n_p;
     }
     __syncthreads();
-    if (!s_last) return;
-    __threadfence();
+    const int n_p = s_np;
+    if (n_p <= 1) return;   // written whole by the main kernel
 
-    const size_t slot0 = ((size_t)b * p.Hkv + h) * p.ns_max;
-    for (int e = threadIdx.x; e < p.n_rows * (kD / 4); e += blockDim.x) {
-        const int row = e / (kD / 4), d4 = (e % (kD / 4)) * 4;
-        float M = kNegInf;
-        for (int s = 0; s < ns; ++s) M = fmaxf(M, __ldcg(&p.part_ml[(slot0 + s) * p.n_rows + row]).x);
+    const int bg = p.b_base + bl;
+    for (int row = warp; row < p.n_rows; row += kMergeThreads / 32) {
+        float M = kNegInf, lsum = 0.f;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        float lsum = 0.f;
-        if (M != kNegInf) {
-            for (int s = 0; s < ns; ++s) {
-                const float2 ml = __ldcg(&p.part_ml[(slot0 + s) * p.n_rows + row]);
-                const float w = ex2(ml.x - M);
-                if (w == 0.f) continue;
-                const float4 v = __ldcg(reinterpret_cast<const float4*>(
-                    p.part_o + ((slot0 + s) * p.n_rows + row) * kD + d4));
-                lsum = fmaf(w, ml.y, lsum);
-                acc.x = fmaf(w, v.x, acc.x);
-                acc.y = fmaf(w, v.y, acc.y);
-                acc.z = fmaf(w, v.z, acc.z);
-                acc.w = fmaf(w, v.w, acc.w);
+        for (int q0 = 0; q0 < n_p; q0 += kMergePieces) {
+            float2 ml[kMergePieces];
+            float4 v[kMergePieces];
+#pragma unroll
+            for (int qq = 0; qq < kMergePieces; ++qq) {
+                const bool ok = q0 + qq < n_p;
+                const size_t sl = (size_t)s_slots[ok ? q0 + qq : 0];
+                ml[qq] = ok ? __ldcg(&p.part_ml[sl * p.n_rows + row]) : make_float2(kNegInf, 0.f);
+                v[qq] = ok ? __ldcg(reinterpret_cast<const float4*>(p.part_o + (sl * p.n_rows + row) * kD +
+                                                                    lane * 4))
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
             }
+            float Mn = M;
+#pragma unroll
+            for (int qq = 0; qq < kMergePieces; ++qq) Mn = fmaxf(Mn, ml[qq].x);
+            if (Mn == kNegInf) continue;
+            const float sc_old = M == kNegInf ? 0.f : ex2(M - Mn);
+            lsum *= sc_old;
+            acc.x *= sc_old;
+            acc.y *= sc_old;
+            acc.z *= sc_old;
+            acc.w *= sc_old;
+#pragma unroll
+            for (int qq = 0; qq < kMergePieces; ++qq) {
+                const float wgt = ml[qq].x == kNegInf ? 0.f : ex2(ml[qq].x - Mn);
+                lsum = fmaf(wgt, ml[qq].y, lsum);
+                acc.x = fmaf(wgt, v[qq].x, acc.x);
+                acc.y = fmaf(wgt, v[qq].y, acc.y);
+                acc.z = fmaf(wgt, v[qq].z, acc.z);
+                acc.w = fmaf(wgt, v[qq].w, acc.w);
+            }
+            M = Mn;
         }
         const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
         const int i = row / p.G, gi = row % p.G;
-        __nv_bfloat16* dst = p.out + (((size_t)b * p.R + i) * p.Hq + (size_t)h * p.G + gi) * kD + d4;
+        __nv_bfloat16* dst = p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)h * p.G + gi) * kD + lane * 4;
         uint2 pk;
         pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
         pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
@@ -389,6 +572,31 @@ cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
+// Resident CTAs per SM of the kernel at a given block size (cached per device).
+int resident_per_sm(int threads) {
+    static int cache[64][kMaxRowWarps + 2] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+        cudaGetLastError();
+        return 1;
+    }
+    const int key = threads / 32;
+    if (key <= 0 || key > kMaxRowWarps + 1) return 1;
+    if (!cache[dev][key]) {
+        int n = 0;
+        if (cudaFuncSetAttribute(verify_attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kSmemBytes) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, verify_attention_kernel, threads,
+                                                          kSmemBytes) != cudaSuccess ||
+            n <= 0) {
+            cudaGetLastError();
+            n = 1;
+        }
+        cache[dev][key] = n;
+    }
+    return cache[dev][key];
+}
+
 }  // namespace
 
 AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count) {
@@ -397,27 +605,14 @@ AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count)
     pl.rows = n_draft + 1;
     pl.n_rows = pl.rows * pl.group;
     pl.row_warps = (pl.n_rows + 15) / 16;
-    const long long l_cap = (long long)d.max_pages_per_seq * d.page_size;
-    // Aim for about four CTAs per SM slot (two resident per SM) over the
-    // expected half-full contexts; one split never exceeds 4096 keys so that
-    // a long request cannot leave a long tail, and is at least one tile.
-    const long long target_units = 8LL * (sm_count > 0 ? sm_count : 148);
-    long long want = ((long long)d.batch * d.n_kv_heads * (l_cap / 2) + target_units - 1) / target_units;
-    want = (want + kTileT - 1) / kTileT * kTileT;
-    if (want < kTileT) want = kTileT;
-    if (want > 4096) want = 4096;
-    pl.chunk = (int)want;
-    pl.ns_max = (int)((l_cap + pl.chunk - 1) / pl.chunk);
-    if (pl.ns_max < 1) pl.ns_max = 1;
+    // persistent grid: exactly the CTAs that are resident at once
+    pl.grid = (sm_count > 0 ? sm_count : 148) * resident_per_sm((pl.row_warps + 1) * 32);
+    if (pl.grid > kMaxGrid) pl.grid = kMaxGrid;
     size_t off = 256;   // status word lives at offset 0
-    if (pl.ns_max > 1) {
-        pl.off_tickets = off;
-        off = align_up(off + sizeof(unsigned int) * (size_t)d.batch * d.n_kv_heads, 256);
-        pl.off_part_ml = off;
-        off = align_up(off + sizeof(float) * 2 * (size_t)d.batch * d.n_kv_heads * pl.ns_max * pl.n_rows, 256);
-        pl.off_part_o = off;
-        off = align_up(off + sizeof(float) * kD * (size_t)d.batch * d.n_kv_heads * pl.ns_max * pl.n_rows, 256);
-    }
+    pl.off_part_ml = off;
+    off = align_up(off + sizeof(float) * 2 * (size_t)2 * pl.grid * pl.n_rows, 256);
+    pl.off_part_o = off;
+    off = align_up(off + sizeof(float) * kD * (size_t)2 * pl.grid * pl.n_rows, 256);
     pl.bytes = off;
     return pl;
 }
@@ -440,9 +635,8 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     p.page_table = page_table;
     p.ctx_lens = ctx_lens;
     p.status = reinterpret_cast<int*>(ws);
-    p.tickets = pl.ns_max > 1 ? reinterpret_cast<unsigned int*>(ws + pl.off_tickets) : nullptr;
-    p.part_ml = pl.ns_max > 1 ? reinterpret_cast<float2*>(ws + pl.off_part_ml) : nullptr;
-    p.part_o = pl.ns_max > 1 ? reinterpret_cast<float*>(ws + pl.off_part_o) : nullptr;
+    p.part_ml = reinterpret_cast<float2*>(ws + pl.off_part_ml);
+    p.part_o = reinterpret_cast<float*>(ws + pl.off_part_o);
     p.Hq = d.n_q_heads;
     p.Hkv = d.n_kv_heads;
     p.G = pl.group;
@@ -451,26 +645,33 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     p.ps = d.page_size;
     p.box_t = box_t;
     p.max_pages = d.max_pages_per_seq;
-    p.chunk = pl.chunk;
-    p.ns_max = pl.ns_max;
     p.row_warps = pl.row_warps;
     const float scale = d.sm_scale > 0.f ? d.sm_scale : 1.0f / sqrtf((float)d.head_dim);
     p.scale_log2 = scale * 1.4426950408889634f;
 
-    static bool attr_set = false;
-    if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(verify_attention_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-        if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_attention_kernel)");
-        attr_set = true;
+    cudaError_t e = cudaSuccess;
+    {
+        static bool attr_done[64] = {};
+        int dev = 0;
+        e = cudaGetDevice(&dev);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+        if (dev < 0 || dev >= 64 || !attr_done[dev]) {
+            e = cudaFuncSetAttribute(verify_attention_kernel,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+            if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_attention_kernel)");
+            if (dev >= 0 && dev < 64) attr_done[dev] = true;
+        }
     }
     const dim3 block((pl.row_warps + 1) * 32);
-    for (int b0 = 0; b0 < d.batch; b0 += 65535) {
+    for (int b0 = 0; b0 < d.batch; b0 += kMaxBatchPerLaunch) {
         p.b_base = b0;
-        const dim3 grid(pl.ns_max, d.n_kv_heads, d.batch - b0 < 65535 ? d.batch - b0 : 65535);
-        verify_attention_kernel<<<grid, block, kSmemBytes, stream>>>(tk, tv, p);
-        const cudaError_t e = cudaGetLastError();
+        p.n_batch = d.batch - b0 < kMaxBatchPerLaunch ? d.batch - b0 : kMaxBatchPerLaunch;
+        verify_attention_kernel<<<pl.grid, block, kSmemBytes, stream>>>(tk, tv, p);
+        e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_fail(e, "verify_attention_kernel launch");
+        verify_attention_merge_kernel<<<dim3(d.n_kv_heads, p.n_batch), kMergeThreads, 0, stream>>>(p, pl.grid);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return cuda_fail(e, "verify_attention_merge_kernel launch");
     }
     return CS_OK;
 }

@@ -63,12 +63,18 @@ def test_noalloc_matches_the_workspace_entry_point_twice(w):
         assert (err <= tol).all(), f"call {call}: {int((err > tol).sum())} elements outside tolerance"
 
 
-def test_noalloc_rejects_problems_beyond_its_scratch():
+def test_noalloc_covers_the_largest_supported_geometry():
+    # (k+1)*G = 144 query rows per KV head is the largest geometry the kernel
+    # takes; its scratch need must fit the fixed array, and the results must
+    # match the workspace entry point
     lib = binding.load_library()
-    d = binding.AttnDims(512, 64, 8, 128, 16, 1024, 1 << 20, 0.0)
-    need = lib.cs_verify_attention_workspace_bytes(ctypes.byref(d), 8)
-    assert need > (32 << 20)
-    fake = 1 << 16
-    st = lib.cs_verify_attention_noalloc(ctypes.byref(d), fake, fake, fake, fake, fake, 8, fake, None)
-    assert st == binding.CS_ERR_UNSUPPORTED
-    assert "scratch" in lib.cs_last_error().decode()
+    w = W.Workload(94, "noalloc-144rows", batch=2, n_draft=8, vocab=64, logit_dtype="bf16",
+                   draft_sigma=1.0, temperatures=(1.0,), n_q_heads=128, n_kv_heads=8,
+                   head_dim=128, ctx=("uniform", 200, 3000), page_size=32)
+    inp = W.attention_inputs(w, DEV)
+    d = binding.attn_dims(inp["q"], inp["k_pages"], inp["page_table"])
+    assert lib.cs_verify_attention_workspace_bytes(ctypes.byref(d), 8) <= (32 << 20)
+    expect = with_workspace(inp).float()
+    for call in range(2):
+        got = noalloc(lib, inp, torch.empty_like(inp["q"])).float()
+        assert ((got - expect).abs() <= ATOL + RTOL * expect.abs()).all(), f"call {call}"
