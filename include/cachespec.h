@@ -145,16 +145,21 @@ cs_status cs_verify_attention(const cs_attn_dims* dims, const void* q, const voi
  *   temperature    T >= 0 and finite
  *   out_tokens     int32 [B, k+1]: x_0..x_{a-1}, the emitted token, then -1
  *   out_n_accepted int32 [B]: a
- *   workspace      device scratch of cs_spec_accept_workspace_bytes(dims, k)
- *                  bytes (this build needs none; NULL is accepted)
+ *   workspace      device scratch of at least cs_spec_accept_workspace_bytes(dims, k)
+ *                  bytes, 256-byte aligned, any initial contents: every call
+ *                  writes each scratch word it later reads (one pair per row
+ *                  segment of the statistics pass).  Calls that share a
+ *                  workspace must be ordered (same stream or events).
  *
- * Logits must be finite.  Rows after the first rejection are not read: they
- * cannot change the result.  The result is a deterministic function of the
- * inputs.
+ * A logit of -inf marks a masked token (probability zero); NaN and +inf are
+ * not allowed, and every row needs a finite entry.  The result is a
+ * deterministic function of the inputs.
  *
  * Returns CS_ERR_INVALID_ARG (null pointer, misalignment, bad dimension,
- * bad temperature, n_draft out of range), CS_ERR_WORKSPACE or CS_ERR_CUDA.
+ * bad temperature, n_draft out of range), CS_ERR_UNSUPPORTED (vocab above
+ * CS_MAX_VOCAB), CS_ERR_WORKSPACE (missing or too small) or CS_ERR_CUDA.
  */
+#define CS_MAX_VOCAB (1 << 22)
 size_t cs_spec_accept_workspace_bytes(const cs_accept_dims* dims, int32_t n_draft);
 cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
                          const void* draft_logits, const int32_t* draft_tokens,

@@ -170,8 +170,20 @@ def cs_verify_attention(q, k_pages, v_pages, page_table, ctx_lens, n_draft, out=
     return out
 
 
+def spec_accept_workspace(dims: AcceptDims, n_draft: int, device) -> torch.Tensor:
+    lib = load_library()
+    n = lib.cs_spec_accept_workspace_bytes(ctypes.byref(dims), int(n_draft))
+    key = ("accept", str(device), n)
+    ws = _workspaces.get(key)
+    if ws is None:
+        ws = torch.zeros(max(n, 256), dtype=torch.uint8, device=device)
+        _workspaces[key] = ws
+    return ws
+
+
 def cs_spec_accept(target_logits, draft_logits, draft_tokens, uniforms, temperature,
-                   out_tokens=None, out_n_accepted=None, stream: int | None = None):
+                   out_tokens=None, out_n_accepted=None, workspace=None,
+                   stream: int | None = None):
     """Speculative acceptance; returns (out_tokens [B, k+1], n_accepted [B]).  See include/cachespec.h."""
     lib = load_library()
     dev = target_logits.device
@@ -194,9 +206,12 @@ def cs_spec_accept(target_logits, draft_logits, draft_tokens, uniforms, temperat
     _need(out_tokens, "out_tokens", torch.int32, 2, dev)
     _need(out_n_accepted, "out_n_accepted", torch.int32, 1, dev)
     d = AcceptDims(B, V, CS_F32 if dtype == torch.float32 else CS_BF16)
+    if workspace is None:
+        workspace = spec_accept_workspace(d, k, dev)
     st = lib.cs_spec_accept(ctypes.byref(d), _ptr(target_logits), _ptr(draft_logits),
                             _ptr(draft_tokens), _ptr(uniforms), int(k), float(temperature),
-                            _ptr(out_tokens), _ptr(out_n_accepted), None, 0,
+                            _ptr(out_tokens), _ptr(out_n_accepted), _ptr(workspace),
+                            workspace.numel() * workspace.element_size(),
                             _stream(dev) if stream is None else stream)
     _check(lib, st)
     return out_tokens, out_n_accepted

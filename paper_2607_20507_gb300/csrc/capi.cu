@@ -59,6 +59,8 @@ cs_status check_accept(const cs_accept_dims* d, int32_t n_draft, float temperatu
         return fail(CS_ERR_INVALID_ARG, "temperature must be finite and >= 0");
     if ((long long)d->batch * (n_draft + 1) * (long long)d->vocab > (1LL << 46))
         return fail(CS_ERR_INVALID_ARG, "logit tensor too large");
+    if (d->vocab > CS_MAX_VOCAB)
+        return fail(CS_ERR_UNSUPPORTED, "vocab %d (this build implements up to %d)", d->vocab, CS_MAX_VOCAB);
     return CS_OK;
 }
 }  // namespace
@@ -127,9 +129,8 @@ cs_status cs_verify_attention(const cs_attn_dims* dims, const void* q, const voi
 }
 
 size_t cs_spec_accept_workspace_bytes(const cs_accept_dims* dims, int32_t n_draft) {
-    (void)dims;
-    (void)n_draft;
-    return 0;
+    if (check_accept(dims, n_draft, 1.0f) != CS_OK) return 0;
+    return accept_workspace_bytes_any(*dims, n_draft);
 }
 
 cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
@@ -137,8 +138,6 @@ cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
                          const float* uniforms, int32_t n_draft, float temperature,
                          int32_t* out_tokens, int32_t* out_n_accepted, void* workspace,
                          size_t workspace_bytes, cs_stream_t stream) {
-    (void)workspace;
-    (void)workspace_bytes;
     cs_status st = check_accept(dims, n_draft, temperature);
     if (st != CS_OK) return st;
     if (dims->batch == 0) return CS_OK;
@@ -152,9 +151,13 @@ cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
     if (!aligned(draft_tokens, 4) || !aligned(uniforms, 4) || !aligned(out_tokens, 4) ||
         !aligned(out_n_accepted, 4))
         return fail(CS_ERR_INVALID_ARG, "int32/fp32 pointers must be 4-byte aligned");
+    const size_t need = accept_workspace_bytes(*dims, n_draft, temperature);
+    if (!workspace || workspace_bytes < need)
+        return fail(CS_ERR_WORKSPACE, "workspace of %zu bytes given, %zu needed", workspace_bytes, need);
+    if (!aligned(workspace, 256)) return fail(CS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
     return launch_spec_accept(*dims, target_logits, temperature > 0.f ? draft_logits : nullptr,
                               draft_tokens, uniforms, n_draft, temperature, out_tokens,
-                              out_n_accepted, reinterpret_cast<cudaStream_t>(stream));
+                              out_n_accepted, workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
 cs_status cs_read_device_status(const void* workspace, int32_t* status_out, cs_stream_t stream) {

@@ -34,9 +34,12 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& plan, c
                                   void* workspace, cudaStream_t stream);
 
 // ------------------------------------------------------------ acceptance
+size_t accept_workspace_bytes(const cs_accept_dims& d, int n_draft, float temperature);
+// The larger of the sampling and greedy requirements.
+size_t accept_workspace_bytes_any(const cs_accept_dims& d, int n_draft);
 cs_status launch_spec_accept(const cs_accept_dims& d, const void* target, const void* draft,
                              const int32_t* tokens, const float* uniforms, int n_draft,
                              float temperature, int32_t* out_tokens, int32_t* out_n,
-                             cudaStream_t stream);
+                             void* workspace, cudaStream_t stream);
 
 }  // namespace cs

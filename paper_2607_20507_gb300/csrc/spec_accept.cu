@@ -3,37 +3,52 @@
 // target and draft rows, the min(1, p/q) accept test, the residual
 // max(0, p - q) or bonus draw by inverse CDF, and the greedy variant.
 //
-// Design.  One thread-block cluster per request; CTA r of the cluster owns a
-// contiguous slice of the vocabulary.  Positions are handled in order:
-//   1. each CTA streams its slice of target row i (and draft row i) once
-//      with 128-bit loads, keeping a running (max, sum 2^((z-max)c)) per
-//      thread (one exponential per logit), then reduces it with warp
-//      shuffles and shared memory;
-//   2. the CTAs swap their partial statistics through distributed shared
-//      memory and fold them in rank order, so every CTA holds bit-identical
-//      row statistics and takes the same accept decision;
-//   3. the first rejection ends the loop: rows after it cannot change the
-//      result and are never read.
-// The draw re-reads the slice of the deciding row pair (just read, so served
-// by L2): a block prefix scan over the slice gives each CTA its mass, the
-// cluster folds the masses in rank order, and the CTA whose cell contains
-// u*Z scans again to find the token.  No probability is written to memory.
-#include <cooperative_groups.h>
+// Two kernels per call, no atomics, no spin-waits and no scratch that has to
+// start at a known value:
+//   1. accept_stats_kernel streams every row of every request (target rows
+//      0..k, then draft rows 0..k-1; target rows only when greedy) once.  The
+//      rows are cut into 4 KB items and the flattened item sequence is split
+//      into one contiguous, equal range per warp of a grid that fills the
+//      device, so every SM reads the same number of bytes.  A warp keeps the
+//      next item in flight while it reduces the current one and writes one
+//      partial per row segment of its range: (max, sum 2^((z-max)c)) -- one
+//      exponential per logit -- or, greedy, (max, lowest id of the max).
+//      The partials of a row sit side by side in the order of the row, and
+//      the warp that holds a row's last item records how many there are.
+//   2. accept_draw_kernel runs one thread-block cluster per request and is
+//      launched as a programmatic dependent of kernel 1: it loads its inputs
+//      while kernel 1 finishes.  Every CTA folds the partials of the
+//      request's rows in the same fixed order (so all of them hold
+//      bit-identical statistics), runs the accept tests
+//      (one lane per position, the first rejection found by a ballot) and
+//      computes the draw mass of its slice of the vocabulary for the deciding
+//      row pair.  The CTAs swap their masses through distributed shared
+//      memory, fold them in rank order, and the CTA whose cell holds u_k * Z
+//      finds the token within its slice.
+//   Greedy mode replaces kernel 2 by accept_greedy_kernel (one warp per
+//   request: argmax agreement).
+// No probability is written to memory; the scratch holds the row-segment
+// pairs and one count per row.
 #include <limits.h>
 #include <math.h>
 
 #include "cs_device.cuh"
 #include "cs_internal.h"
 
-namespace cg = cooperative_groups;
-
 namespace cs {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 256;                  // kernel 1 and the greedy kernel
 constexpr int kWarps = kThreads / 32;
-constexpr int kGroup = 8;     // consecutive logits a thread takes per step (one 16-byte bf16 vector)
-constexpr int kBatch = 2;     // groups per row in flight per thread
+constexpr int kDrawThreads = 512;              // kernel 2
+constexpr int kDrawWarps = kDrawThreads / 32;
+constexpr int kVecs = 8;                       // kernel 1: 16-byte vectors per lane per item
+constexpr int kItemBytes = 32 * kVecs * 16;    // 4 KB of one row
+constexpr int kRunVecs = 2;                    // kernel 2: 16-byte vectors per thread per row per pass
+constexpr int kMaxRows = 33;                   // 2k+1 rows of a request, k <= 16
+constexpr int kRowsPerDrawWarp = (kMaxRows + kDrawWarps - 1) / kDrawWarps;
+constexpr int kMaxPasses = 128;                // passes of one CTA over its vocabulary slice
+constexpr int kMaxCluster = 16;
 
 struct AcceptParams {
     const void* target;       // [B, k+1, V]
@@ -42,12 +57,20 @@ struct AcceptParams {
     const float* uniforms;    // [B, k+1]
     int32_t* out_tokens;      // [B, k+1]
     int32_t* out_n;           // [B]
-    int V, k, chunk;
-    int b_base;               // first request of this launch (grids hold <= 65535 requests)
+    int B, V, k;
+    int R;                    // rows per request: 2k+1 (sampling) or k+1 (greedy)
+    int I;                    // 4 KB items per row
+    long long N;              // B * R * I items in all
+    int W;                    // busy warps of kernel 1 (warp w owns items [w*N/W, (w+1)*N/W)), W <= N
+    int J;                    // partial slots per row (row segments a row can have)
+    int slice;                // kernel 2: logits of the vocabulary per CTA of a cluster
+    int b_base;               // kernel 2: first request of this launch
     float c_hi, c_lo;         // log2(e) / T as a float pair
+    float2* part;             // [B*R, J] row-segment partials, in row order
+    int* cnt;                 // [B*R] segments of each row
 };
 
-// ------------------------------------------------------------ logit loads
+// ------------------------------------------------------------ small helpers
 __device__ __forceinline__ uint4 ld_stream(const void* p) {
     uint4 v;
     asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
@@ -59,45 +82,30 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
 __device__ __forceinline__ float to_f(float v) { return v; }
 __device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
 
-// Eight consecutive logits row[start .. start+8) as fp32; entries at or past
-// `end` read as -inf.  `vec` says the row base is 16-byte aligned.
-__device__ __forceinline__ void load8(const __nv_bfloat16* row, int start, int end, bool vec,
-                                      float (&v)[kGroup]) {
-    if (vec && start + kGroup <= end) {
-        const uint4 u = ld_stream(row + start);
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            v[2 * e] = bf16_bits_to_float(w[e] & 0xffffu);
-            v[2 * e + 1] = bf16_bits_to_float(w[e] >> 16);
-        }
-    } else {
-#pragma unroll
-        for (int e = 0; e < kGroup; ++e)
-            v[e] = start + e < end ? __bfloat162float(row[start + e]) : kNegInf;
-    }
-}
-
-__device__ __forceinline__ void load8(const float* row, int start, int end, bool vec,
-                                      float (&v)[kGroup]) {
-    if (vec && start + kGroup <= end) {
-        const uint4 a = ld_stream(row + start), b = ld_stream(row + start + 4);
-        v[0] = __uint_as_float(a.x); v[1] = __uint_as_float(a.y);
-        v[2] = __uint_as_float(a.z); v[3] = __uint_as_float(a.w);
-        v[4] = __uint_as_float(b.x); v[5] = __uint_as_float(b.y);
-        v[6] = __uint_as_float(b.z); v[7] = __uint_as_float(b.w);
-    } else {
-#pragma unroll
-        for (int e = 0; e < kGroup; ++e) v[e] = start + e < end ? row[start + e] : kNegInf;
-    }
-}
-
 template <typename T>
 __device__ __forceinline__ bool aligned16(const T* p) {
     return (reinterpret_cast<uintptr_t>(p) & 15u) == 0;
 }
 
-// ------------------------------------------------------- (max, sum) algebra
+template <typename T>
+union Vec16 {
+    uint4 q;
+    T t[16 / sizeof(T)];
+};
+
+// 16 bytes of row[start ..]; entries at or past `end` read as -inf.  `stream`
+// bypasses L1 (kernel 1 touches every byte once).
+template <typename T, bool kStream>
+__device__ __forceinline__ uint4 load16(const T* row, int start, int end, bool vec) {
+    constexpr int kPer = 16 / (int)sizeof(T);
+    if (vec && start + kPer <= end)
+        return kStream ? ld_stream(row + start) : __ldg(reinterpret_cast<const uint4*>(row + start));
+    Vec16<T> v;
+#pragma unroll
+    for (int e = 0; e < kPer; ++e) v.t[e] = start + e < end ? row[start + e] : (T)kNegInf;
+    return v.q;
+}
+
 // A pair (m, s) stands for sum_v 2^((z_v - m) c); empty is (-inf, 0).
 __device__ __forceinline__ void fold(float& m, float& s, float m2, float s2, float c_hi, float c_lo) {
     const float M = fmaxf(m, m2);
@@ -108,595 +116,800 @@ __device__ __forceinline__ void fold(float& m, float& s, float m2, float s2, flo
     m = M;
 }
 
-template <int N>
-__device__ __forceinline__ void running_update(float& m, float& s, const float (&v)[N][kGroup],
-                                               float c) {
-    float bm = kNegInf;
-#pragma unroll
-    for (int u = 0; u < N; ++u)
-#pragma unroll
-        for (int e = 0; e < kGroup; ++e) bm = fmaxf(bm, v[u][e]);
-    if (bm > m) {
-        s = m == kNegInf ? 0.f : s * ex2((m - bm) * c);
-        m = bm;
-    }
-    if (m == kNegInf) return;
-#pragma unroll
-    for (int u = 0; u < N; ++u)
-#pragma unroll
-        for (int e = 0; e < kGroup; ++e) s += ex2((v[u][e] - m) * c);
+// (max, id) with the lowest id on ties; the id travels as int bits.
+__device__ __forceinline__ void argmax_fold(float2& acc, float2 o) {
+    if (o.x > acc.x || (o.x == acc.x && __float_as_int(o.y) < __float_as_int(acc.y))) acc = o;
 }
 
-// Per-thread statistics of this CTA's slice [c0, c1) of one or two rows.
-template <typename T>
-__device__ __forceinline__ void slice_stats(const T* rt, const T* rd, bool two, int c0, int c1,
-                                            float c, float (&m)[2], float (&s)[2]) {
-    m[0] = m[1] = kNegInf;
-    s[0] = s[1] = 0.f;
-    const int ng = c1 > c0 ? (c1 - c0 + kGroup - 1) / kGroup : 0;
-    const bool vt = aligned16(rt), vd = two && aligned16(rd);
-    for (int g0 = threadIdx.x; g0 < ng; g0 += kThreads * kBatch) {
-        float at[kBatch][kGroup], ad[kBatch][kGroup];
-#pragma unroll
-        for (int u = 0; u < kBatch; ++u) {
-            const int gi = g0 + u * kThreads;
-            if (gi < ng) {
-                load8(rt, c0 + gi * kGroup, c1, vt, at[u]);
-                if (two) load8(rd, c0 + gi * kGroup, c1, vd, ad[u]);
-            } else {
-#pragma unroll
-                for (int e = 0; e < kGroup; ++e) at[u][e] = ad[u][e] = kNegInf;
-            }
-        }
-        running_update(m[0], s[0], at, c);
-        if (two) running_update(m[1], s[1], ad, c);
-    }
-}
+// Unnormalised weight of one logit, 2^((z - m) c), with the same single-term
+// exponent the statistics summed (so that the weights of a row add up to its
+// normaliser S).  m is finite, so -inf weighs 2^-inf = 0.
+__device__ __forceinline__ float weight(float z, float m, float c_hi) { return ex2((z - m) * c_hi); }
 
-// Block reduction of per-thread (m, s) pairs for two rows, in a fixed order
-// (xor butterflies within each warp, then across the warp results in warp 0).
-// Thread 0 ends with the CTA's pairs.
-__device__ __forceinline__ void block_fold2(float (&m)[2], float (&s)[2], float c_hi, float c_lo,
-                                            float (*red)[4]) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            const float m2 = __shfl_xor_sync(0xffffffffu, m[r], off);
-            const float s2 = __shfl_xor_sync(0xffffffffu, s[r], off);
-            fold(m[r], s[r], m2, s2, c_hi, c_lo);
-        }
-    }
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) {
-        red[warp][0] = m[0];
-        red[warp][1] = s[0];
-        red[warp][2] = m[1];
-        red[warp][3] = s[1];
-    }
-    __syncthreads();
-    if (warp == 0) {
-        const bool have = lane < kWarps;
-        m[0] = have ? red[lane][0] : kNegInf;
-        s[0] = have ? red[lane][1] : 0.f;
-        m[1] = have ? red[lane][2] : kNegInf;
-        s[1] = have ? red[lane][3] : 0.f;
-#pragma unroll
-        for (int off = kWarps / 2; off > 0; off >>= 1) {
-#pragma unroll
-            for (int r = 0; r < 2; ++r) {
-                const float m2 = __shfl_xor_sync(0xffffffffu, m[r], off);
-                const float s2 = __shfl_xor_sync(0xffffffffu, s[r], off);
-                fold(m[r], s[r], m2, s2, c_hi, c_lo);
-            }
-        }
-    }
-}
-
-// Cluster fold of the CTAs' (m, s) pairs for two rows: lane r of warp 0
-// reads rank r's pairs from distributed shared memory, then an xor butterfly
-// in a fixed order.  Every CTA folds the same values in the same order, so
-// lane 0 of every CTA holds bit-identical results.  Warp 0 only.
-__device__ __forceinline__ void cluster_fold2(cg::cluster_group& cl, const float* mine, int n_ranks,
-                                              float c_hi, float c_lo, float (&M)[2], float (&S)[2]) {
-    const int lane = threadIdx.x & 31;
-    M[0] = M[1] = kNegInf;
-    S[0] = S[1] = 0.f;
-    if (lane < n_ranks) {
-        const float4 v = *reinterpret_cast<const float4*>(cl.map_shared_rank(mine, lane));
-        M[0] = v.x;
-        S[0] = v.y;
-        M[1] = v.z;
-        S[1] = v.w;
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {
-            const float m2 = __shfl_xor_sync(0xffffffffu, M[r], off);
-            const float s2 = __shfl_xor_sync(0xffffffffu, S[r], off);
-            fold(M[r], S[r], m2, s2, c_hi, c_lo);
-        }
-    }
-}
-
-// Block-wide inclusive scan of one float per thread (fixed order).  Returns
-// the inclusive prefix; `excl` gets the exclusive one, `total` the block sum.
-__device__ __forceinline__ float block_scan(float x, float& excl, float& total, float* wsum) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    float inc = x;
+__device__ __forceinline__ float warp_incl_scan(float x, int lane) {
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
-        const float y = __shfl_up_sync(0xffffffffu, inc, off);
-        if (lane >= off) inc += y;
+        const float y = __shfl_up_sync(0xffffffffu, x, off);
+        if (lane >= off) x += y;
     }
-    if (lane == 31) wsum[warp] = inc;
-    __syncthreads();
-    if (warp == 0) {
-        float w = lane < kWarps ? wsum[lane] : 0.f;
-        float wi = w;
+    return x;
+}
+
+__device__ __forceinline__ int warp_max_int(int x) {
 #pragma unroll
-        for (int off = 1; off < kWarps; off <<= 1) {
-            const float y = __shfl_up_sync(0xffffffffu, wi, off);
-            if (lane >= off) wi += y;
-        }
-        if (lane < kWarps) wsum[kWarps + lane] = wi - w;   // exclusive warp prefix
-        if (lane == kWarps - 1) wsum[2 * kWarps] = wi;     // block total
+    for (int off = 16; off > 0; off >>= 1) x = max(x, __shfl_xor_sync(0xffffffffu, x, off));
+    return x;
+}
+
+// Folds the (m, s) pairs of the 32 lanes: the maximum first, then one
+// rescale per lane and a butterfly sum.  Every lane ends with the same pair.
+__device__ __forceinline__ float2 warp_fold_sum(float m, float s, float c_hi, float c_lo) {
+    float M = m;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float t = m == kNegInf ? 0.f : s * ex2_scaled(m - M, c_hi, c_lo);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
+    return make_float2(M, t);
+}
+
+// (max, lowest id of the max) over the 32 lanes, in every lane.
+__device__ __forceinline__ float2 warp_fold_argmax(float2 acc) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        float2 o;
+        o.x = __shfl_xor_sync(0xffffffffu, acc.x, off);
+        o.y = __shfl_xor_sync(0xffffffffu, acc.y, off);
+        argmax_fold(acc, o);
     }
-    __syncthreads();
-    const float wp = wsum[kWarps + warp];
-    const float incl = wp + inc;
-    const float up = __shfl_up_sync(0xffffffffu, incl, 1);
-    excl = lane == 0 ? wp : up;
-    total = wsum[2 * kWarps];
-    __syncthreads();   // wsum is reused by the next call
-    return incl;
+    return acc;
 }
 
-// Probability-scale weight of one logit: 2^((z - m) c) / S, zero for -inf.
-__device__ __forceinline__ float weight(float z, float m, float inv_s, float c_hi, float c_lo) {
-    return z == kNegInf ? 0.f : ex2_scaled(z - m, c_hi, c_lo) * inv_s;
-}
-
-struct DrawRow {
-    float mt, inv_st, md, inv_sd;
-    int residual;   // 1: max(0, p - q); 0: p only
-};
-
-// Scans this CTA's slice of the draw distribution in ascending token order.
-// Without `search` it returns the slice mass.  With `search` it returns the
-// first token whose running mass (starting from `base`) exceeds `t`, or the
-// slice's last token of positive weight when rounding leaves none; -1 if the
-// slice has no positive weight.
 template <typename T>
-__device__ float draw_scan(const T* rt, const T* rd, int c0, int c1, const DrawRow& w, float c_hi,
-                           float c_lo, bool search, float base, float t, int* s_found,
-                           float* wsum) {
-    const int ng = c1 > c0 ? (c1 - c0 + kGroup - 1) / kGroup : 0;
-    const bool vt = aligned16(rt), vd = w.residual && aligned16(rd);
-    float run = base;
-    int last_pos = -1;
-    if (search && threadIdx.x == 0) *s_found = INT_MAX;
-    __syncthreads();
-    for (int g0 = 0; g0 < ng; g0 += kThreads) {
-        const int gi = g0 + threadIdx.x;
-        float r[kGroup];
-        if (gi < ng) {
-            float zt[kGroup], zd[kGroup];
-            load8(rt, c0 + gi * kGroup, c1, vt, zt);
-            if (w.residual) load8(rd, c0 + gi * kGroup, c1, vd, zd);
+__device__ __forceinline__ const T* row_ptr(const AcceptParams& p, int b, int r) {
+    const int V = p.V, k = p.k;
+    return r <= k ? static_cast<const T*>(p.target) + ((size_t)b * (k + 1) + r) * V
+                  : static_cast<const T*>(p.draft) + ((size_t)b * k + (r - k - 1)) * V;
+}
+
+// x / d for x >= 0, d > 0: one 32-bit division whenever both fit (every
+// realistic problem), the 64-bit routine otherwise.
+__device__ __forceinline__ long long div_nn(long long x, long long d) {
+    if ((unsigned long long)x <= 0xffffffffull && (unsigned long long)d <= 0xffffffffull)
+        return (long long)((unsigned)x / (unsigned)d);
+    return x / d;
+}
+
+// First item of warp w's range (kernel 1's balanced split).
+__device__ __forceinline__ long long range_lo(const AcceptParams& p, long long w) {
+    return div_nn(w * p.N, p.W);
+}
+
+// Programmatic dependent launch: the draw kernel may start while the
+// statistics kernel runs; it waits here before reading what that kernel
+// wrote (a no-op when it was launched without the attribute).
+__device__ __forceinline__ void wait_prior_grid() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void allow_dependent_launch() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// ------------------------------------------------------------ kernel 1
+// Largest of the 8 * kVecs logits of one lane's item (bf16: packed maxima,
+// one instruction per pair).
+__device__ __forceinline__ float item_max(const uint4 (&v)[kVecs], __nv_bfloat16) {
+    __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&v[0].x);
+    __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&v[0].y);
+    __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&v[0].z);
+    __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&v[0].w);
 #pragma unroll
-            for (int e = 0; e < kGroup; ++e) {
-                const float pt = weight(zt[e], w.mt, w.inv_st, c_hi, c_lo);
-                const float qd = w.residual ? weight(zd[e], w.md, w.inv_sd, c_hi, c_lo) : 0.f;
-                r[e] = fmaxf(pt - qd, 0.f);
-                if (r[e] > 0.f) last_pos = c0 + gi * kGroup + e;
+    for (int u = 1; u < kVecs; ++u) {
+        a = __hmax2(a, *reinterpret_cast<const __nv_bfloat162*>(&v[u].x));
+        b = __hmax2(b, *reinterpret_cast<const __nv_bfloat162*>(&v[u].y));
+        c = __hmax2(c, *reinterpret_cast<const __nv_bfloat162*>(&v[u].z));
+        d = __hmax2(d, *reinterpret_cast<const __nv_bfloat162*>(&v[u].w));
+    }
+    a = __hmax2(__hmax2(a, b), __hmax2(c, d));
+    return fmaxf(__low2float(a), __high2float(a));
+}
+
+__device__ __forceinline__ float item_max(const uint4 (&v)[kVecs], float) {
+    float a = kNegInf, b = kNegInf;
+#pragma unroll
+    for (int u = 0; u < kVecs; ++u) {
+        a = fmaxf(a, fmaxf(__uint_as_float(v[u].x), __uint_as_float(v[u].y)));
+        b = fmaxf(b, fmaxf(__uint_as_float(v[u].z), __uint_as_float(v[u].w)));
+    }
+    return fmaxf(a, b);
+}
+
+// The logits of a 32-bit word: two bf16 (low half first) or one fp32.
+__device__ __forceinline__ float word_lo(uint32_t x, __nv_bfloat16) { return __uint_as_float(x << 16); }
+__device__ __forceinline__ float word_hi(uint32_t x, __nv_bfloat16) { return __uint_as_float(x & 0xffff0000u); }
+
+// sum over one lane's item of 2^((z - m) c_hi), four independent partial sums.
+template <typename T>
+__device__ __forceinline__ float item_sum(const uint4 (&v)[kVecs], float m, float c_hi) {
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+#pragma unroll
+    for (int u = 0; u < kVecs; ++u) {
+        const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+        if constexpr (sizeof(T) == 2) {
+            s0 += ex2((word_lo(w[0], T()) - m) * c_hi);
+            s1 += ex2((word_hi(w[0], T()) - m) * c_hi);
+            s2 += ex2((word_lo(w[1], T()) - m) * c_hi);
+            s3 += ex2((word_hi(w[1], T()) - m) * c_hi);
+            s0 += ex2((word_lo(w[2], T()) - m) * c_hi);
+            s1 += ex2((word_hi(w[2], T()) - m) * c_hi);
+            s2 += ex2((word_lo(w[3], T()) - m) * c_hi);
+            s3 += ex2((word_hi(w[3], T()) - m) * c_hi);
+        } else {
+            s0 += ex2((__uint_as_float(w[0]) - m) * c_hi);
+            s1 += ex2((__uint_as_float(w[1]) - m) * c_hi);
+            s2 += ex2((__uint_as_float(w[2]) - m) * c_hi);
+            s3 += ex2((__uint_as_float(w[3]) - m) * c_hi);
+        }
+    }
+    return (s0 + s1) + (s2 + s3);
+}
+
+template <typename T, bool kGreedy>
+__global__ void __launch_bounds__(kThreads, 2) accept_stats_kernel(const AcceptParams p) {
+    constexpr int kPer = 16 / (int)sizeof(T);
+    constexpr int kItem = kItemBytes / (int)sizeof(T);
+    const int lane = threadIdx.x & 31;
+    const long long w = (long long)blockIdx.x * kWarps + (threadIdx.x >> 5);
+    allow_dependent_launch();
+    if (w >= p.W) return;
+    const long long lo = range_lo(p, w), hi = range_lo(p, w + 1);
+    const int I = p.I, V = p.V, R = p.R;
+
+    // One item into registers: lane l holds vectors u*32 + l; entries past
+    // the row's end read as -inf.
+    auto load = [&](long long row, int item, uint4 (&v)[kVecs]) {
+        const T* rp = row_ptr<T>(p, (int)(row / R), (int)(row % R));
+        const int e0 = item * kItem, e1 = min(V, e0 + kItem);
+        if (aligned16(rp) && e1 - e0 == kItem) {
+#pragma unroll
+            for (int u = 0; u < kVecs; ++u) v[u] = ld_stream(rp + e0 + (u * 32 + lane) * kPer);
+        } else {
+            const bool vec = aligned16(rp);
+#pragma unroll
+            for (int u = 0; u < kVecs; ++u) v[u] = load16<T, true>(rp, e0 + (u * 32 + lane) * kPer, e1, vec);
+        }
+    };
+
+    long long row = div_nn(lo, I);
+    int item = (int)(lo - row * I);
+    uint4 cur[kVecs], nxt[kVecs];
+    load(row, item, cur);
+    float m = kNegInf, s = 0.f;            // sampling: lane's running (max, sum)
+    int id = INT_MAX;                      // greedy: lane's lowest id of the max (m)
+    for (long long f = lo; f < hi; ++f) {
+        long long nrow = row;
+        int nitem = item + 1;
+        if (nitem == I) {
+            nrow = row + 1;
+            nitem = 0;
+        }
+        if (f + 1 < hi) load(nrow, nitem, nxt);
+        if (kGreedy) {
+            const int base = item * kItem;
+#pragma unroll
+            for (int u = 0; u < kVecs; ++u) {   // ascending ids: strict > keeps the lowest
+                Vec16<T> v;
+                v.q = cur[u];
+#pragma unroll
+                for (int e = 0; e < kPer; ++e) {
+                    const float z = to_f(v.t[e]);
+                    if (z > m) {
+                        m = z;
+                        id = base + (u * 32 + lane) * kPer + e;
+                    }
+                }
             }
         } else {
-#pragma unroll
-            for (int e = 0; e < kGroup; ++e) r[e] = 0.f;
-        }
-        float sj = 0.f;
-#pragma unroll
-        for (int e = 0; e < kGroup; ++e) sj += r[e];
-        float excl, total;
-        const float incl = block_scan(sj, excl, total, wsum);
-        if (search) {
-            const bool cross = run + incl > t;
-            if (cross) atomicMin(s_found, threadIdx.x);
-            __syncthreads();
-            const int owner = *s_found;
-            if (owner != INT_MAX) {
-                // the owner thread walks its eight weights; the result goes back
-                // through s_found as a token id (>= 0) offset below INT_MIN/2
-                __syncthreads();
-                if (threadIdx.x == owner) {
-                    float cum = run + excl;
-                    int pick = -1, lastp = -1;
-#pragma unroll
-                    for (int e = 0; e < kGroup; ++e) {
-                        cum += r[e];
-                        if (r[e] > 0.f) lastp = c0 + gi * kGroup + e;
-                        if (pick < 0 && cum > t) pick = c0 + gi * kGroup + e;
-                    }
-                    *s_found = INT_MIN + 1 + (pick >= 0 ? pick : lastp);
-                }
-                __syncthreads();
-                const int res = *s_found - (INT_MIN + 1);
-                __syncthreads();
-                return (float)res;
+            const float mi = item_max(cur, T());
+            if (mi > m) {
+                s = m == kNegInf ? 0.f : s * ex2_scaled(m - mi, p.c_hi, p.c_lo);
+                m = mi;
             }
+            if (m != kNegInf) s += item_sum<T>(cur, m, p.c_hi);
         }
-        run += total;
+        if (nitem == 0 || f + 1 == hi) {
+            // the row segment ends: fold the lanes and publish the pair in
+            // slot w - (owner of the row's first item) of the row
+            const float2 acc = kGreedy ? warp_fold_argmax(make_float2(m, __int_as_float(id)))
+                                       : warp_fold_sum(m, s, p.c_hi, p.c_lo);
+            if (lane == 0) {
+                const long long first_owner = div_nn((row * I + 1) * p.W - 1, p.N);
+                const int j = (int)(w - first_owner);
+                p.part[row * p.J + j] = acc;
+                if (nitem == 0) p.cnt[row] = j + 1;   // this warp holds the row's last item
+            }
+            m = kNegInf;
+            s = 0.f;
+            id = INT_MAX;
+        }
+        row = nrow;
+        item = nitem;
+#pragma unroll
+        for (int u = 0; u < kVecs; ++u) cur[u] = nxt[u];
     }
-    if (!search) return run;
-    // no crossing inside the slice: its last token of positive weight
-    if (threadIdx.x == 0) *s_found = -1;
-    __syncthreads();
-    if (last_pos >= 0) atomicMax(s_found, last_pos);
-    __syncthreads();
-    const int res = *s_found;
-    __syncthreads();
-    return (float)res;
 }
 
-// ------------------------------------------------------------------ kernel
-template <typename T, bool kGreedy>
-__global__ void __launch_bounds__(kThreads) spec_accept_kernel(const AcceptParams p) {
-    cg::cluster_group cl = cg::this_cluster();
-    const int n_ranks = (int)cl.num_blocks();
-    const int rank = (int)cl.block_rank();
-    const int b = blockIdx.y + p.b_base;
-    const int V = p.V, k = p.k;
-    const int c0 = min(V, rank * p.chunk), c1 = min(V, c0 + p.chunk);
-    const T* tgt = static_cast<const T*>(p.target) + (size_t)b * (k + 1) * V;
-    const T* drf = kGreedy ? nullptr : static_cast<const T*>(p.draft) + (size_t)b * k * V;
-    const int32_t* x = p.tokens + (size_t)b * k;
-    const float* u = p.uniforms + (size_t)b * (k + 1);
-    const float c_hi = p.c_hi, c_lo = p.c_lo;
-
-    __shared__ __align__(16) float xch[2][4];   // this CTA's contribution to the current exchange
-    __shared__ float red[kWarps][4];
-    __shared__ float wsum[2 * kWarps + 1];
-    __shared__ float bc[8];              // values broadcast by thread 0
-    __shared__ int bci[4];
-    __shared__ int s_found;
-    int epoch = 0;
-
-    if (kGreedy) {
-        int a = k, emit = 0;
-        for (int i = 0; i <= k; ++i) {
-            const T* row = tgt + (size_t)i * V;
-            const bool vec = aligned16(row);
-            const int x_i = (threadIdx.x == 0 && i < k) ? __ldg(x + i) : -1;
-            float best = kNegInf;
-            int bi = INT_MAX;
-            const int ng = c1 > c0 ? (c1 - c0 + kGroup - 1) / kGroup : 0;
-            for (int g0 = threadIdx.x; g0 < ng; g0 += kThreads * kBatch) {
-                float v[kBatch][kGroup];
+// ------------------------------------------------- row statistics (kernel 2)
+// Row g's partials are part[g*J .. g*J + cnt[g]), in the order of the row.
+// Lane l folds slots l, l+32, ... in order, then the lanes are folded; the
+// result is the same in every lane and in every CTA that folds row g.
+// The rows of one call are folded kBatch at a time, with the loads of a
+// whole batch in flight together.
+template <bool kGreedy, int kBatch>
+__device__ __forceinline__ void fold_rows(const AcceptParams& p, int b, int first_row, int row_step,
+                                          int n_rows, int lane, float2* s_stat) {
+    const float2 empty = make_float2(kNegInf, kGreedy ? __int_as_float(INT_MAX) : 0.f);
+    for (int r0 = first_row; r0 < n_rows; r0 += kBatch * row_step) {
+        float2 pre[kBatch];
+        int n[kBatch];
 #pragma unroll
-                for (int uu = 0; uu < kBatch; ++uu) {
-                    const int gi = g0 + uu * kThreads;
-                    if (gi < ng) load8(row, c0 + gi * kGroup, c1, vec, v[uu]);
-                }
-#pragma unroll
-                for (int uu = 0; uu < kBatch; ++uu) {
-                    const int gi = g0 + uu * kThreads;
-                    if (gi >= ng) continue;
-#pragma unroll
-                    for (int e = 0; e < kGroup; ++e)
-                        if (v[uu][e] > best) {   // ascending ids: strict > keeps the lowest
-                            best = v[uu][e];
-                            bi = c0 + gi * kGroup + e;
-                        }
-                }
-            }
-            // block argmax, lowest id on ties
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) {
-                const float b2 = __shfl_xor_sync(0xffffffffu, best, off);
-                const int i2 = __shfl_xor_sync(0xffffffffu, bi, off);
-                if (b2 > best || (b2 == best && i2 < bi)) {
-                    best = b2;
-                    bi = i2;
-                }
-            }
-            if ((threadIdx.x & 31) == 0) {
-                red[threadIdx.x >> 5][0] = best;
-                red[threadIdx.x >> 5][1] = __int_as_float(bi);
-            }
-            __syncthreads();
-            if (threadIdx.x < 32) {
-                const int lane = threadIdx.x;
-                best = lane < kWarps ? red[lane][0] : kNegInf;
-                bi = lane < kWarps ? __float_as_int(red[lane][1]) : INT_MAX;
-#pragma unroll
-                for (int off = kWarps / 2; off > 0; off >>= 1) {
-                    const float b2 = __shfl_xor_sync(0xffffffffu, best, off);
-                    const int i2 = __shfl_xor_sync(0xffffffffu, bi, off);
-                    if (b2 > best || (b2 == best && i2 < bi)) {
-                        best = b2;
-                        bi = i2;
-                    }
-                }
-                if (lane == 0) {
-                    xch[epoch & 1][0] = best;
-                    xch[epoch & 1][1] = __int_as_float(bi);
-                }
-            }
-            cl.sync();
-            if (threadIdx.x < 32) {
-                const int lane = threadIdx.x;
-                float gb = kNegInf;
-                int gidx = INT_MAX;
-                if (lane < n_ranks) {
-                    const float* rx = cl.map_shared_rank(&xch[epoch & 1][0], lane);
-                    gb = rx[0];
-                    gidx = __float_as_int(rx[1]);
-                }
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1) {
-                    const float b2 = __shfl_xor_sync(0xffffffffu, gb, off);
-                    const int i2 = __shfl_xor_sync(0xffffffffu, gidx, off);
-                    if (b2 > gb || (b2 == gb && i2 < gidx)) {
-                        gb = b2;
-                        gidx = i2;
-                    }
-                }
-                if (lane == 0) {
-                    if (gidx == INT_MAX) gidx = 0;   // a row with no finite entry
-                    bci[0] = gidx;
-                    bci[1] = (i == k || x_i != gidx) ? 1 : 0;
-                }
-            }
-            __syncthreads();
-            ++epoch;
-            if (bci[1]) {
-                a = i;
-                emit = bci[0];
-                break;
-            }
-            __syncthreads();
-        }
-        if (rank == 0 && threadIdx.x == 0) {
-            int32_t* out = p.out_tokens + (size_t)b * (k + 1);
-            for (int j = 0; j < a; ++j) out[j] = __ldg(x + j);
-            out[a] = emit;
-            for (int j = a + 1; j <= k; ++j) out[j] = -1;
-            p.out_n[b] = a;
-        }
-        cl.sync();
-        return;
-    }
-
-    // ----------------------------------------------------------- T > 0
-    float mt = 0.f, St = 1.f, md = 0.f, Sd = 1.f;
-    int a = k;
-    for (int i = 0; i <= k; ++i) {
-        const bool two = i < k;
-        // thread 0 fetches what the accept test needs while the slice streams
-        int xi = -1;
-        float zt_x = 0.f, zd_x = 0.f, ui = 0.f;
-        if (threadIdx.x == 0 && two) {
-            xi = __ldg(x + i);
-            ui = __ldg(u + i);
-            if (xi >= 0 && xi < V) {
-                zt_x = to_f(tgt[(size_t)i * V + xi]);
-                zd_x = to_f(drf[(size_t)i * V + xi]);
+        for (int j = 0; j < kBatch; ++j) {
+            const int r = r0 + j * row_step;
+            pre[j] = empty;
+            n[j] = 0;
+            if (r < n_rows) {
+                const long long g = (long long)b * p.R + r;
+                n[j] = __ldcg(p.cnt + g);
+                if (lane < p.J) pre[j] = __ldcg(p.part + g * p.J + lane);
             }
         }
-        float m[2], s[2];
-        slice_stats(tgt + (size_t)i * V, two ? drf + (size_t)i * V : tgt, two, c0, c1, c_hi, m, s);
-        block_fold2(m, s, c_hi, c_lo, red);
-        if (threadIdx.x == 0) {
-            xch[epoch & 1][0] = m[0];
-            xch[epoch & 1][1] = s[0];
-            xch[epoch & 1][2] = m[1];
-            xch[epoch & 1][3] = s[1];
-        }
-        cl.sync();
-        if (threadIdx.x < 32) {
-            float M[2], S[2];
-            cluster_fold2(cl, &xch[epoch & 1][0], n_ranks, c_hi, c_lo, M, S);
-            if (threadIdx.x == 0) {
-                bc[0] = M[0];
-                bc[1] = S[0];
-                bc[2] = M[1];
-                bc[3] = S[1];
-                int reject = 0;
-                if (two) {
-                    if (xi < 0 || xi >= V || zt_x == kNegInf) {
-                        reject = 1;
-                    } else {
-                        // log2 p(x)/q(x) = ((zt - mt) - (zd - md)) c + log2 Sd - log2 St,
-                        // carried as an unevaluated float pair
-                        const float dz = (zt_x - M[0]) - (zd_x - M[1]);
-                        const float A = dz * c_hi;
-                        float E = fmaf(dz, c_lo, fmaf(dz, c_hi, -A));
-                        const float Bl = lg2(S[1]) - lg2(S[0]);
-                        const float H = A + Bl;
-                        const float bb = H - A;
-                        E += (A - (H - bb)) + (Bl - bb);
-                        const float ratio = ex2(H) * fmaf(E, kLn2, 1.f);
-                        reject = !(ui < ratio);
-                    }
-                }
-                bci[0] = reject;
+#pragma unroll
+        for (int j = 0; j < kBatch; ++j) {
+            const int r = r0 + j * row_step;
+            if (r >= n_rows) break;
+            const long long g = (long long)b * p.R + r;
+            float2 f = lane < n[j] ? pre[j] : empty;
+            for (int l = lane + 32; l < n[j]; l += 32) {
+                const float2 o = __ldcg(p.part + g * p.J + l);
+                if (kGreedy) argmax_fold(f, o);
+                else fold(f.x, f.y, o.x, o.y, p.c_hi, p.c_lo);
             }
-        }
-        __syncthreads();
-        ++epoch;
-        mt = bc[0];
-        St = bc[1];
-        md = bc[2];
-        Sd = bc[3];
-        const int reject = bci[0];
-        __syncthreads();
-        if (i == k) break;
-        if (reject) {
-            a = i;
-            break;
+            f = kGreedy ? warp_fold_argmax(f) : warp_fold_sum(f.x, f.y, p.c_hi, p.c_lo);
+            if (lane == 0) s_stat[r] = f;
         }
     }
+}
 
-    // ------------------------------------------------------------ the draw
-    const T* rt = tgt + (size_t)a * V;
-    const T* rd = a < k ? drf + (size_t)a * V : tgt;
-    DrawRow w{mt, 1.f / St, md, 1.f / Sd, a < k ? 1 : 0};
-    int token = -1, owner = -1;
-    for (int attempt = 0; attempt < 2; ++attempt) {
-        const float mass = draw_scan(rt, rd, c0, c1, w, c_hi, c_lo, false, 0.f, 0.f, &s_found, wsum);
-        if (threadIdx.x == 0) xch[epoch & 1][0] = mass;
-        cl.sync();
-        if (threadIdx.x < 32) {
-            // lane r holds rank r's mass; an inclusive scan in a fixed order
-            // gives every CTA the same cumulative masses
-            const int lane = threadIdx.x;
-            const float Mr = lane < n_ranks ? *cl.map_shared_rank(&xch[epoch & 1][0], lane) : 0.f;
-            float incl = Mr;
+// ------------------------------------------------------------ accept test
+// Whether position i rejects: u_i < p_i(x_i) / q_i(x_i) fails.  zt, zd are
+// the target and draft logits of x_i, st, sd the rows' statistics.
+__device__ __forceinline__ bool rejects(bool valid, float zt, float zd, float2 st, float2 sd, float u,
+                                        float c_hi, float c_lo) {
+    if (!valid || zt == kNegInf) return true;
+    // log2 p(x)/q(x) = ((zt - mt) - (zd - md)) c + log2 Sd - log2 St, carried
+    // as an unevaluated float pair
+    const float dz = (zt - st.x) - (zd - sd.x);
+    const float A = dz * c_hi;
+    float E = fmaf(dz, c_lo, fmaf(dz, c_hi, -A));
+    const float Bl = lg2(sd.y) - lg2(st.y);
+    const float H = A + Bl;
+    const float bb = H - A;
+    E += (A - (H - bb)) + (Bl - bb);
+    const float ratio = ex2(H) * fmaf(E, kLn2, 1.f);
+    return !(u < ratio);
+}
+
+// ------------------------------------------------------------ cluster PTX
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_size() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ void cluster_arrive() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_wait() {
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Reads a float2 at the same shared-memory offset in CTA `rank` of the cluster.
+__device__ __forceinline__ float2 ld_cluster_f2(const float2* local, uint32_t rank) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+    float2 v;
+    asm volatile("ld.shared::cluster.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(remote) : "memory");
+    return v;
+}
+
+// ------------------------------------------------------------ draw weights
+// Weights of thread-run [start, start + kRun) of the draw row pair (entries at
+// or past `end` weigh zero): max(p - q, 0), or p alone when !residual.
+template <typename T>
+// The draw weights are p and max(p - q, 0) scaled by S_t (the inverse CDF
+// does not depend on a common factor): 2^((zt - mt)c) and
+// max(2^((zt - mt)c) - rho 2^((zd - md)c), 0) with rho = S_t / S_d.
+struct DrawRow {
+    const T* rt;
+    const T* rd;
+    float mt, md, rho, c_hi;
+    bool at, ad;
+};
+
+template <typename T, bool kResidual>
+__device__ __forceinline__ void run_weights(const DrawRow<T>& d, int start, int end,
+                                            float (&w)[kRunVecs * 16 / sizeof(T)]) {
+    constexpr int kPer = 16 / (int)sizeof(T);
+    uint4 vt[kRunVecs], vd[kRunVecs];
+    if (d.at && (!kResidual || d.ad) && start + kRunVecs * kPer <= end) {
 #pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                const float y = __shfl_up_sync(0xffffffffu, incl, off);
-                if (lane >= off) incl += y;
-            }
-            const float Z = __shfl_sync(0xffffffffu, incl, 31);
-            const float excl = incl - Mr;   // only used as the owner's base (see below)
-            const float up = __shfl_up_sync(0xffffffffu, incl, 1);
-            const float base_l = lane == 0 ? 0.f : up;
-            (void)excl;
-            int retry = 0, own = -1;
-            float base = 0.f, t = 0.f;
-            if (!(Z > 0.f)) {
-                retry = 1;   // p == q up to rounding: fall back to p of the same row
-            } else {
-                t = __ldg(u + k) * Z;
-                const unsigned cross = __ballot_sync(0xffffffffu, lane < n_ranks && Mr > 0.f && incl > t);
-                const unsigned pos = __ballot_sync(0xffffffffu, lane < n_ranks && Mr > 0.f);
-                if (cross) {
-                    own = __ffs(cross) - 1;
-                    base = __shfl_sync(0xffffffffu, base_l, own);
-                } else {   // u*Z at or past the total through rounding
-                    own = 31 - __clz(pos);
-                    base = 0.f;
-                    t = __int_as_float(0x7f800000);
-                }
-            }
-            if (lane == 0) {
-                bci[0] = retry;
-                bci[1] = own;
-                bc[4] = base;
-                bc[5] = t;
-            }
+        for (int u = 0; u < kRunVecs; ++u) {
+            vt[u] = __ldg(reinterpret_cast<const uint4*>(d.rt + start + u * kPer));
+            if (kResidual) vd[u] = __ldg(reinterpret_cast<const uint4*>(d.rd + start + u * kPer));
         }
-        __syncthreads();
-        ++epoch;
-        const int retry = bci[0];
-        owner = bci[1];
-        const float base = bc[4], t = bc[5];
-        __syncthreads();
-        if (retry && attempt == 0 && w.residual) {
-            w.residual = 0;
+    } else {
+#pragma unroll
+        for (int u = 0; u < kRunVecs; ++u) {
+            vt[u] = load16<T, false>(d.rt, start + u * kPer, end, d.at);
+            if (kResidual) vd[u] = load16<T, false>(d.rd, start + u * kPer, end, d.ad);
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kRunVecs; ++u) {
+        Vec16<T> a, b;
+        a.q = vt[u];
+        if (kResidual) b.q = vd[u];
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) {
+            const float pt = weight(to_f(a.t[e]), d.mt, d.c_hi);
+            if (kResidual) w[u * kPer + e] = fmaxf(fmaf(-d.rho, weight(to_f(b.t[e]), d.md, d.c_hi), pt), 0.f);
+            else w[u * kPer + e] = pt;
+        }
+    }
+}
+
+// One pass of a CTA over logits [pass_start, pass_start + kDrawThreads*kRun):
+// every thread's weights, its inclusive scan position and the pass total.
+// The warp totals are folded in warp order, so the pass total and every
+// thread's prefix are the same numbers whenever the pass is recomputed.
+struct PassScan {
+    float incl;    // mass of the pass up to and including this thread's run
+    float excl;    // incl less the thread's own run (the start of its walk)
+    float own;     // mass of this thread's run
+    float total;   // mass of the pass
+    int last;      // largest id of the pass with positive weight, -1 if none
+};
+
+template <typename T, bool kResidual>
+__device__ __forceinline__ PassScan pass_scan_t(const DrawRow<T>& d, int pass_start, int end,
+                                              float (&w)[kRunVecs * 16 / sizeof(T)], float (&s_wsum)[kDrawWarps],
+                                              int (&s_wlast)[kDrawWarps]) {
+    constexpr int kRun = kRunVecs * 16 / (int)sizeof(T);
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int start = pass_start + tid * kRun;
+    run_weights<T, kResidual>(d, start, end, w);
+    float ls = 0.f;
+    int lp = -1;
+#pragma unroll
+    for (int e = 0; e < kRun; ++e) {
+        ls += w[e];
+        if (w[e] > 0.f) lp = start + e;
+    }
+    const float incl = warp_incl_scan(ls, lane);
+    lp = warp_max_int(lp);
+    if (lane == 31) s_wsum[wid] = incl;
+    if (lane == 0) s_wlast[wid] = lp;
+    __syncthreads();
+    PassScan r;
+    float off = 0.f, tot = 0.f;
+    int last = -1;
+#pragma unroll
+    for (int j = 0; j < kDrawWarps; ++j) {
+        if (j == wid) off = tot;
+        tot += s_wsum[j];
+        last = max(last, s_wlast[j]);
+    }
+    __syncthreads();   // s_wsum / s_wlast are reused by the next pass
+    // the last thread's incl is the pass total bit for bit (same additions)
+    r.incl = off + incl;
+    r.excl = r.incl - ls;
+    r.own = ls;
+    r.total = tot;
+    r.last = last;
+    return r;
+}
+
+template <typename T>
+__device__ __forceinline__ PassScan pass_scan(const DrawRow<T>& d, bool residual, int pass_start, int end,
+                                              float (&w)[kRunVecs * 16 / sizeof(T)], float (&s_wsum)[kDrawWarps],
+                                              int (&s_wlast)[kDrawWarps]) {
+    return residual ? pass_scan_t<T, true>(d, pass_start, end, w, s_wsum, s_wlast)
+                    : pass_scan_t<T, false>(d, pass_start, end, w, s_wsum, s_wlast);
+}
+
+// ------------------------------------------------------------ kernel 2
+template <typename T>
+__global__ void __launch_bounds__(kDrawThreads, 2) accept_draw_kernel(const AcceptParams p) {
+    constexpr int kPer = 16 / (int)sizeof(T);
+    constexpr int kRun = kRunVecs * kPer;
+    constexpr int kPass = kDrawThreads * kRun;
+    __shared__ float2 s_stat[kMaxRows];
+    __shared__ float s_pass[kMaxPasses];
+    __shared__ float s_wsum[kDrawWarps];
+    __shared__ int s_wlast[kDrawWarps];
+    __shared__ int s_first[kDrawWarps];
+    __shared__ int s_a;
+    __shared__ float2 s_x[2];   // (slice mass, last positive id) per exchange round
+
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const uint32_t rank = cluster_rank(), n_ranks = cluster_size();
+    const int b = p.b_base + blockIdx.y;
+    const int k = p.k, V = p.V;
+
+    // ---- the accept-test inputs of lane i < k of warp 0, loaded first
+    bool valid = false;
+    float zt = 0.f, zd = 0.f, ui = 1.f;
+    int xi = -1;
+    if (wid == 0 && lane < k) {
+        xi = __ldg(p.tokens + (size_t)b * k + lane);
+        ui = __ldg(p.uniforms + (size_t)b * (k + 1) + lane);
+        valid = xi >= 0 && xi < V;
+        if (valid) {
+            zt = to_f(row_ptr<T>(p, b, lane)[xi]);
+            zd = to_f(row_ptr<T>(p, b, k + 1 + lane)[xi]);
+        }
+    }
+    const float uk = __ldg(p.uniforms + (size_t)b * (k + 1) + k);
+
+    // ---- row statistics of the request (kernel 1's output), then the tests
+    wait_prior_grid();
+    fold_rows<false, kRowsPerDrawWarp>(p, b, wid, kDrawWarps, p.R, lane, s_stat);
+    __syncthreads();
+    if (wid == 0) {
+        bool rej = false;
+        if (lane < k) rej = rejects(valid, zt, zd, s_stat[lane], s_stat[k + 1 + lane], ui, p.c_hi, p.c_lo);
+        const unsigned m = __ballot_sync(0xffffffffu, rej);
+        if (lane == 0) s_a = m ? __ffs(m) - 1 : k;
+    }
+    __syncthreads();
+    const int a = s_a;
+
+    // ---- the draw: this CTA's slice [c0, c1) of row pair a
+    const int c0 = min(V, (int)rank * p.slice), c1 = min(V, c0 + p.slice);
+    const int n_pass = (c1 - c0 + kPass - 1) / kPass;
+    DrawRow<T> d;
+    d.rt = row_ptr<T>(p, b, a);
+    d.rd = a < k ? row_ptr<T>(p, b, k + 1 + a) : d.rt;
+    // a row without a finite entry (outside the contract) weighs zero everywhere
+    const float2 st = s_stat[a], sd = a < k ? s_stat[k + 1 + a] : make_float2(0.f, 0.f);
+    d.mt = st.x == kNegInf ? 0.f : st.x;
+    d.md = sd.x == kNegInf ? 0.f : sd.x;
+    d.rho = sd.y > 0.f ? st.y / sd.y : 0.f;
+    d.c_hi = p.c_hi;
+    d.at = aligned16(d.rt);
+    d.ad = aligned16(d.rd);
+
+    if (n_pass > 1) {
+        // several passes: ask L2 for the whole slice of the row pair now, so
+        // that the passes below find it there instead of waiting on DRAM
+        const char* bt = reinterpret_cast<const char*>(d.rt + c0);
+        const char* bd = reinterpret_cast<const char*>(d.rd + c0);
+        const int bytes = (c1 - c0) * (int)sizeof(T);
+        for (int off = tid * 128; off < bytes; off += kDrawThreads * 128) {
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(bt + off));
+            if (a < k) asm volatile("prefetch.global.L2 [%0];" ::"l"(bd + off));
+        }
+    }
+    bool residual = a < k;
+    float w[kRun];
+    int token = 0;
+    int writer = -1;   // the thread of this CTA that writes the emitted token
+    for (int round = 0; round < 2; ++round) {
+        float mass = 0.f;
+        int last = -1;
+        PassScan kept{0.f, 0.f, 0.f, 0.f, -1};   // the last pass, whose weights stay in w
+        for (int ps = 0; ps < n_pass; ++ps) {
+            const int nx = c0 + (ps + 1) * kPass + tid * kRun;
+            if (ps + 1 < n_pass && (tid & 3) == 0 && nx < c1) {
+                // the next pass into L1 while this one is reduced (a 128-byte
+                // line holds the runs of four threads); only addresses inside
+                // the slice are touched
+                asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rt + nx));
+                if (residual) asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rd + nx));
+            }
+            kept = pass_scan<T>(d, residual, c0 + ps * kPass, c1, w, s_wsum, s_wlast);
+            if (tid == 0) s_pass[ps] = kept.total;
+            mass += kept.total;
+            last = max(last, kept.last);
+        }
+        if (tid == 0) s_x[round] = make_float2(mass, __int_as_float(last));
+        cluster_arrive();
+        cluster_wait();
+        // every CTA folds the masses of ranks 0..n-1 in the same order
+        float2 x = make_float2(0.f, __int_as_float(-1));
+        if (lane < (int)n_ranks) x = ld_cluster_f2(&s_x[round], lane);
+        const float incl = warp_incl_scan(x.x, lane);
+        const float Z = __shfl_sync(0xffffffffu, incl, 31);
+        if (!(Z > 0.f) && residual && round == 0) {
+            // no positive residual (p == q up to rounding): draw from p instead
+            residual = false;
             continue;
         }
-        if (owner == rank) {
-            token = (int)draw_scan(rt, rd, c0, c1, w, c_hi, c_lo, true, base, t, &s_found, wsum);
+        const float t = uk * Z;
+        const float before = incl - x.x;
+        const unsigned own = __ballot_sync(0xffffffffu, lane < (int)n_ranks && x.x > 0.f && incl > t);
+        if (!own) {
+            // u_k * Z at or past the total through rounding: the last positive weight
+            const int lp = warp_max_int(__float_as_int(x.y));
+            token = lp >= 0 ? lp : 0;
+            if (rank == 0) writer = 0;
+            break;
         }
+        const int owner = __ffs(own) - 1;
+        if ((int)rank != owner) break;
+        float tt = t - __shfl_sync(0xffffffffu, before, owner);   // position within this slice
+        // the pass that holds the cell, in the order the mass was summed
+        int pj = -1;
+        float cum = 0.f;
+        for (int ps = 0; ps < n_pass; ++ps) {
+            const float m = s_pass[ps];
+            if (m > 0.f && cum + m > tt) {
+                pj = ps;
+                break;
+            }
+            cum += m;
+        }
+        if (pj < 0) {   // rounding: the slice's last positive weight
+            token = last;
+            writer = 0;
+            break;
+        }
+        tt -= cum;
+        // the weights of the last pass are still in registers; others are recomputed
+        const PassScan sc = pj == n_pass - 1 ? kept : pass_scan<T>(d, residual, c0 + pj * kPass, c1, w, s_wsum, s_wlast);
+        // the first run with positive mass whose prefix passes tt (a run of
+        // zero weights can come first through rounding; it never owns the draw)
+        const unsigned cross = __ballot_sync(0xffffffffu, sc.own > 0.f && sc.incl > tt);
+        if (lane == 0) s_first[wid] = cross ? wid * 32 + __ffs(cross) - 1 : INT_MAX;
+        __syncthreads();
+        int first = INT_MAX;
+#pragma unroll
+        for (int j = 0; j < kDrawWarps; ++j) first = min(first, s_first[j]);
+        if (first == INT_MAX) {   // rounding: the pass's last positive weight
+            token = sc.last;
+            writer = 0;
+            break;
+        }
+        if (tid == first) {
+            const int start = c0 + pj * kPass + tid * kRun;
+            float c = sc.excl;
+            int pick = -1, lastp = -1;
+#pragma unroll
+            for (int e = 0; e < kRun; ++e) {
+                c += w[e];
+                if (w[e] > 0.f) {   // only a token with positive weight can be drawn
+                    lastp = start + e;
+                    if (pick < 0 && c > tt) pick = start + e;
+                }
+            }
+            token = pick >= 0 ? pick : lastp;   // the run has a positive weight
+        }
+        writer = first;
         break;
     }
-    if (threadIdx.x == 0) {
-        int32_t* out = p.out_tokens + (size_t)b * (k + 1);
-        if (owner == rank) out[a] = token >= 0 ? token : c0;
-        if (rank == 0) {
-            for (int j = 0; j < a; ++j) out[j] = __ldg(x + j);
-            for (int j = a + 1; j <= k; ++j) out[j] = -1;
-            p.out_n[b] = a;
-            if (owner < 0) out[a] = 0;   // no positive weight anywhere (not a distribution)
-        }
+    if (tid == writer) p.out_tokens[(size_t)b * (k + 1) + a] = token >= 0 ? token : 0;
+    if (rank == 0 && tid <= k && tid != a) {
+        const int32_t x = tid < a ? __ldg(p.tokens + (size_t)b * k + tid) : -1;
+        p.out_tokens[(size_t)b * (k + 1) + tid] = x;
     }
-    cl.sync();   // shared memory of every rank stays alive until all reads are done
+    if (rank == 0 && tid == 0) p.out_n[b] = a;
+    // no CTA leaves while another may still read its exchange slots
+    cluster_arrive();
+    cluster_wait();
+}
+
+// ------------------------------------------------------------ greedy
+template <typename T>
+__global__ void __launch_bounds__(kThreads) accept_greedy_kernel(const AcceptParams p) {
+    __shared__ float2 s_stat[kWarps][kMaxRows];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int b = blockIdx.x * kWarps + wid;
+    if (b >= p.B) return;
+    const int k = p.k;
+    wait_prior_grid();
+    fold_rows<true, 4>(p, b, 0, 1, k + 1, lane, s_stat[wid]);
+    __syncwarp();
+    int g = 0, x = -1;
+    if (lane <= k) {
+        g = __float_as_int(s_stat[wid][lane].y);
+        if (g == INT_MAX) g = 0;   // a row with no finite entry
+    }
+    if (lane < k) x = __ldg(p.tokens + (size_t)b * k + lane);
+    const unsigned miss = __ballot_sync(0xffffffffu, lane < k && x != g);
+    const int a = miss ? __ffs(miss) - 1 : k;
+    const int emit = __shfl_sync(0xffffffffu, g, a);
+    if (lane <= k) p.out_tokens[(size_t)b * (k + 1) + lane] = lane < a ? x : (lane == a ? emit : -1);
+    if (lane == 0) p.out_n[b] = a;
+}
+
+// ------------------------------------------------------------------- host
+// Resident CTAs of `kern` on the current device (cached per device and slot).
+template <typename K>
+int resident_ctas(K kern, int slot, int threads, int smem) {
+    static int cache[64][8] = {};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    int occ = (dev >= 0 && dev < 64) ? cache[dev][slot] : 0;
+    if (!occ) {
+        if (smem > 48 * 1024) cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, threads, smem) != cudaSuccess || occ <= 0)
+            occ = 2;
+        cudaGetLastError();
+        if (dev >= 0 && dev < 64) cache[dev][slot] = occ;
+    }
+    return occ * current_sm_count();
 }
 
 int g_max_cluster[64] = {0};
 
-int max_cluster_size(int dev) {
+// The largest cluster (16, non-portable, or 8) the device schedules for the
+// draw kernel.
+int max_cluster_size() {
+    int dev = 0;
+    cudaGetDevice(&dev);
     if (dev < 0 || dev >= 64) return 8;
     if (g_max_cluster[dev]) return g_max_cluster[dev];
     int best = 8;
-    auto kern = spec_accept_kernel<__nv_bfloat16, false>;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+    auto kern = accept_draw_kernel<__nv_bfloat16>;
+    auto kern32 = accept_draw_kernel<float>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess &&
+        cudaFuncSetAttribute(kern32, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
         cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(16, 1, 1);
-        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.gridDim = dim3(kMaxCluster, 1, 1);
+        cfg.blockDim = dim3(kDrawThreads, 1, 1);
         cudaLaunchAttribute attr;
         attr.id = cudaLaunchAttributeClusterDimension;
-        attr.val.clusterDim.x = 16;
+        attr.val.clusterDim.x = kMaxCluster;
         attr.val.clusterDim.y = 1;
         attr.val.clusterDim.z = 1;
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
-        int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0) best = 16;
+        int n = 0, n32 = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0 &&
+            cudaOccupancyMaxActiveClusters(&n32, kern32, &cfg) == cudaSuccess && n32 > 0)
+            best = kMaxCluster;
     }
     cudaGetLastError();
     g_max_cluster[dev] = best;
     return best;
 }
 
+struct AcceptPlan {
+    int R, I, W, J, grid1;
+    long long N;
+    int cluster, slice;
+    size_t off_cnt, bytes;
+};
+
 template <typename T, bool G>
-cs_status launch_typed(AcceptParams p, int cluster, int batch, cudaStream_t stream) {
-    auto kern = spec_accept_kernel<T, G>;
-    if (cluster > 8) {
-        static bool done[64] = {};
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (dev < 0 || dev >= 64 || !done[dev]) {
-            const cudaError_t e =
-                cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-            if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(non-portable cluster)");
-            if (dev >= 0 && dev < 64) done[dev] = true;
-        }
+int stats_resident() {
+    const int slot = (G ? 1 : 0) + (sizeof(T) == 4 ? 2 : 0);
+    return resident_ctas(accept_stats_kernel<T, G>, slot, kThreads, 0);
+}
+
+AcceptPlan plan_accept(const cs_accept_dims& d, int n_draft, bool greedy, bool with_cluster) {
+    const bool f32 = d.logit_dtype == CS_F32;
+    AcceptPlan P{};
+    P.R = greedy ? n_draft + 1 : 2 * n_draft + 1;
+    const int item = kItemBytes / (f32 ? 4 : 2);
+    P.I = (d.vocab + item - 1) / item;
+    P.N = (long long)d.batch * P.R * P.I;
+    const int resident = f32 ? (greedy ? stats_resident<float, true>() : stats_resident<float, false>())
+                             : (greedy ? stats_resident<__nv_bfloat16, true>()
+                                       : stats_resident<__nv_bfloat16, false>());
+    long long g = (P.N + kWarps - 1) / kWarps;
+    if (g > resident) g = resident;
+    P.grid1 = (int)(g > 0 ? g : 1);
+    // every busy warp owns at least one item, so a row's segments come from
+    // consecutive warps
+    const long long warps = (long long)P.grid1 * kWarps;
+    P.W = (int)(warps < P.N ? warps : (P.N > 0 ? P.N : 1));
+    // a row meets at most (I-1)/q + 2 ranges of q >= 1 items, and at most I
+    const long long q = P.N / P.W > 0 ? P.N / P.W : 1;
+    const long long J = (P.I - 1) / q + 2;
+    P.J = (int)(J < P.I ? J : P.I);
+    const size_t rows = (size_t)d.batch * P.R;
+    P.off_cnt = (rows * P.J * sizeof(float2) + 255) / 256 * 256;
+    P.bytes = P.off_cnt + (rows * sizeof(int) + 255) / 256 * 256;
+    if (!greedy && with_cluster) {
+        // All clusters in one wave (two CTAs per SM), no CTA with an empty
+        // slice, at most kMaxPasses passes per CTA.
+        const int pass = kDrawThreads * kRunVecs * (f32 ? 4 : 8);
+        const int sms = current_sm_count();
+        int c = 2 * sms / (d.batch > 0 ? d.batch : 1);
+        const int by_vocab = (d.vocab + pass - 1) / pass;
+        if (c > by_vocab) c = by_vocab;
+        const int cmax = max_cluster_size();
+        if (c > cmax) c = cmax;
+        const int need = (int)(((long long)d.vocab + (long long)kMaxPasses * pass - 1) / ((long long)kMaxPasses * pass));
+        if (c < need) c = need;
+        if (c < 1) c = 1;
+        P.cluster = c;
+        const int per = (d.vocab + c - 1) / c;
+        P.slice = (per + 7) / 8 * 8;
     }
-    for (int b0 = 0; b0 < batch; b0 += 65535) {
+    return P;
+}
+
+template <typename T, bool G>
+cs_status launch_typed(AcceptParams p, const AcceptPlan& P, cudaStream_t stream) {
+    accept_stats_kernel<T, G><<<P.grid1, kThreads, 0, stream>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "accept_stats_kernel launch");
+    // the second kernel is launched as a programmatic dependent of the first:
+    // it may start early and waits (griddepcontrol.wait) before reading the
+    // partials
+    cudaLaunchAttribute attrs[2];
+    attrs[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attrs[0].val.programmaticStreamSerializationAllowed = 1;
+    if (G) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((p.B + kWarps - 1) / kWarps, 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.stream = stream;
+        cfg.attrs = attrs;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, accept_greedy_kernel<T>, p);
+        if (e != cudaSuccess) return cuda_fail(e, "accept_greedy_kernel launch");
+        return CS_OK;
+    }
+    auto kern = accept_draw_kernel<T>;
+    if (P.cluster > 8) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(non-portable cluster)");
+    }
+    attrs[1].id = cudaLaunchAttributeClusterDimension;
+    attrs[1].val.clusterDim.x = P.cluster;
+    attrs[1].val.clusterDim.y = 1;
+    attrs[1].val.clusterDim.z = 1;
+    for (int b0 = 0; b0 < p.B; b0 += 65535) {
         p.b_base = b0;
         cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(cluster, batch - b0 < 65535 ? batch - b0 : 65535, 1);
-        cfg.blockDim = dim3(kThreads, 1, 1);
-        cfg.dynamicSmemBytes = 0;
+        cfg.gridDim = dim3(P.cluster, p.B - b0 < 65535 ? p.B - b0 : 65535, 1);
+        cfg.blockDim = dim3(kDrawThreads, 1, 1);
         cfg.stream = stream;
-        cudaLaunchAttribute attr;
-        attr.id = cudaLaunchAttributeClusterDimension;
-        attr.val.clusterDim.x = cluster;
-        attr.val.clusterDim.y = 1;
-        attr.val.clusterDim.z = 1;
-        cfg.attrs = &attr;
-        cfg.numAttrs = 1;
-        const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p);
-        if (e != cudaSuccess) return cuda_fail(e, "spec_accept_kernel launch");
+        cfg.attrs = attrs;
+        cfg.numAttrs = 2;
+        e = cudaLaunchKernelEx(&cfg, kern, p);
+        if (e != cudaSuccess) return cuda_fail(e, "accept_draw_kernel launch");
     }
     return CS_OK;
 }
 
 }  // namespace
 
+size_t accept_workspace_bytes(const cs_accept_dims& d, int n_draft, float temperature) {
+    if (temperature == 0.f) return plan_accept(d, n_draft, true, false).bytes;
+    return plan_accept(d, n_draft, false, false).bytes;
+}
+
+size_t accept_workspace_bytes_any(const cs_accept_dims& d, int n_draft) {
+    const size_t a = plan_accept(d, n_draft, true, false).bytes;
+    const size_t b = plan_accept(d, n_draft, false, false).bytes;
+    return a > b ? a : b;
+}
+
 cs_status launch_spec_accept(const cs_accept_dims& d, const void* target, const void* draft,
                              const int32_t* tokens, const float* uniforms, int n_draft,
                              float temperature, int32_t* out_tokens, int32_t* out_n,
-                             cudaStream_t stream) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-    const int sms = current_sm_count();
-    // Enough CTAs to cover the SMs several times over, at least ~2K logits per
-    // CTA, at most the largest cluster the device schedules.
-    const int want = (4 * sms + d.batch - 1) / d.batch;
-    int cluster = 1;
-    while (cluster < want && cluster < 16) cluster <<= 1;
-    int by_vocab = 1;
-    while (by_vocab * 2 <= d.vocab / 2048 && by_vocab < 16) by_vocab <<= 1;
-    if (cluster > by_vocab) cluster = by_vocab;
-    const int cmax = max_cluster_size(dev);
-    if (cluster > cmax) cluster = cmax;
-
+                             void* workspace, cudaStream_t stream) {
+    const bool greedy = temperature == 0.f;
+    const AcceptPlan P = plan_accept(d, n_draft, greedy, true);
     AcceptParams p{};
     p.target = target;
     p.draft = draft;
@@ -704,19 +917,24 @@ cs_status launch_spec_accept(const cs_accept_dims& d, const void* target, const 
     p.uniforms = uniforms;
     p.out_tokens = out_tokens;
     p.out_n = out_n;
+    p.B = d.batch;
     p.V = d.vocab;
     p.k = n_draft;
-    const int per = (d.vocab + cluster - 1) / cluster;
-    p.chunk = (per + kGroup - 1) / kGroup * kGroup;
+    p.R = P.R;
+    p.I = P.I;
+    p.N = P.N;
+    p.W = P.W;
+    p.J = P.J;
+    p.slice = P.slice;
     const double c = temperature > 0.f ? 1.4426950408889634 / (double)temperature : 0.0;
     p.c_hi = (float)c;
     p.c_lo = (float)(c - (double)p.c_hi);
-    const bool greedy = temperature == 0.f;
+    p.part = static_cast<float2*>(workspace);
+    p.cnt = reinterpret_cast<int*>(static_cast<uint8_t*>(workspace) + P.off_cnt);
     if (d.logit_dtype == CS_F32)
-        return greedy ? launch_typed<float, true>(p, cluster, d.batch, stream)
-                      : launch_typed<float, false>(p, cluster, d.batch, stream);
-    return greedy ? launch_typed<__nv_bfloat16, true>(p, cluster, d.batch, stream)
-                  : launch_typed<__nv_bfloat16, false>(p, cluster, d.batch, stream);
+        return greedy ? launch_typed<float, true>(p, P, stream) : launch_typed<float, false>(p, P, stream);
+    return greedy ? launch_typed<__nv_bfloat16, true>(p, P, stream)
+                  : launch_typed<__nv_bfloat16, false>(p, P, stream);
 }
 
 }  // namespace cs

@@ -114,8 +114,9 @@ def test_empty_batch_is_a_no_op(lib):
                               None) == binding.CS_OK
 
 
-def accept(lib, dims, n_draft=4, T=1.0, t=FAKE, d=FAKE, x=FAKE, u=FAKE, out=FAKE, n=FAKE):
-    return lib.cs_spec_accept(ctypes.byref(dims), t, d, x, u, n_draft, T, out, n, None, 0, None)
+def accept(lib, dims, n_draft=4, T=1.0, t=FAKE, d=FAKE, x=FAKE, u=FAKE, out=FAKE, n=FAKE, ws=FAKE,
+           ws_bytes=1 << 40):
+    return lib.cs_spec_accept(ctypes.byref(dims), t, d, x, u, n_draft, T, out, n, ws, ws_bytes, None)
 
 
 @pytest.mark.parametrize("field,value", [("batch", -2), ("vocab", 0), ("logit_dtype", 7)])
@@ -123,6 +124,11 @@ def test_spec_accept_rejects_bad_dims(lib, field, value):
     dims = binding.AcceptDims(4, 32000, binding.CS_BF16)
     setattr(dims, field, value)
     assert accept(lib, dims) == binding.CS_ERR_INVALID_ARG
+
+
+def test_spec_accept_rejects_vocabularies_beyond_the_limit(lib):
+    assert accept(lib, binding.AcceptDims(2, (1 << 22) + 1, binding.CS_BF16)) == binding.CS_ERR_UNSUPPORTED
+    assert lib.cs_spec_accept_workspace_bytes(ctypes.byref(binding.AcceptDims(2, (1 << 22) + 1, binding.CS_BF16)), 4) == 0
 
 
 @pytest.mark.parametrize("T", [-0.5, float("nan"), float("inf")])
@@ -141,7 +147,10 @@ def test_spec_accept_null_and_alignment(lib):
         assert accept(lib, dims, **{arg: None}) == binding.CS_ERR_INVALID_ARG
     assert accept(lib, dims, d=None) == binding.CS_ERR_INVALID_ARG            # T > 0 needs the draft
     assert accept(lib, dims, t=FAKE + 2) == binding.CS_ERR_INVALID_ARG        # fp32 logits, 2-byte offset
-    assert lib.cs_spec_accept_workspace_bytes(ctypes.byref(dims), 4) == 0
+    need = lib.cs_spec_accept_workspace_bytes(ctypes.byref(dims), 4)
+    assert need >= 4 * 9 * 4 * 8             # one (max, sum) pair per chunk of each row
+    assert accept(lib, dims, ws=None) == binding.CS_ERR_WORKSPACE
+    assert accept(lib, dims, ws_bytes=need - 1) == binding.CS_ERR_WORKSPACE
 
 
 def test_binding_fails_loudly_without_library(tmp_path):

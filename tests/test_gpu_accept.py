@@ -139,6 +139,26 @@ def test_masked_minus_inf_logits():
     assert_parity(inp, 1.0, "-inf masked")
 
 
+@pytest.mark.parametrize("V,dtype", [(5000, "bf16"), (40000, "f32"), (300000, "bf16")])
+def test_draw_at_the_top_of_the_cdf(V, dtype):
+    # u_k just below 1 puts the draw at the end of the CDF, where the fp32
+    # running sums may stop short of u_k * Z (the rounding fallback: the last
+    # id with positive weight).  The last 100 ids are masked and the last
+    # unmasked one carries most of the target's mass, so both paths must
+    # emit exactly that id, for the residual and the bonus draw alike.
+    B, k = 24, 3
+    inp = custom(B, k, V, dtype, 1.0, cell=9)
+    last = V - 101
+    inp["target"][..., last + 1:] = float("-inf")
+    inp["draft"][..., last + 1:] = float("-inf")
+    inp["target"][..., last] = inp["target"].float().amax(dim=-1).to(inp["target"].dtype) + 6.0
+    inp["draft_tokens"].clamp_(max=last)
+    inp["uniforms"][:, k] = float(np.nextafter(np.float32(1.0), np.float32(0.0)))
+    out, n = gpu(inp, 1.0)
+    got = out[np.arange(B), n]
+    assert (got == last).all(), got
+
+
 def test_deterministic():
     inp = W.accept_inputs(W.WORKLOADS[3], 1.0, DEV)
     a = gpu(inp, 1.0)
