@@ -118,6 +118,9 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nw = p.row_warps;
     const int nb = p.n_batch;
+    // the merge kernel is a programmatic dependent: let it start (and work out
+    // its schedule) while this kernel runs
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     // ---- schedule: exclusive prefix of tiles per request (x heads), clamped L
     if (threadIdx.x == 0) {
@@ -492,6 +495,9 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     __syncthreads();
     const int n_p = s_np;
     if (n_p <= 1) return;   // written whole by the main kernel
+    // everything above depends only on the context lengths; the pieces are
+    // the main kernel's output
+    asm volatile("griddepcontrol.wait;" ::: "memory");
 
     const int bg = p.b_base + bl;
     for (int row = warp; row < p.n_rows; row += kMergeThreads / 32) {
@@ -669,8 +675,18 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
         verify_attention_kernel<<<pl.grid, block, kSmemBytes, stream>>>(tk, tv, p);
         e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_fail(e, "verify_attention_kernel launch");
-        verify_attention_merge_kernel<<<dim3(d.n_kv_heads, p.n_batch), kMergeThreads, 0, stream>>>(p, pl.grid);
-        e = cudaGetLastError();
+        // programmatic dependent launch: the merge kernel may start early and
+        // waits (griddepcontrol.wait) before it reads the partials
+        cudaLaunchAttribute attr;
+        attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr.val.programmaticStreamSerializationAllowed = 1;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(d.n_kv_heads, p.n_batch, 1);
+        cfg.blockDim = dim3(kMergeThreads, 1, 1);
+        cfg.stream = stream;
+        cfg.attrs = &attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, verify_attention_merge_kernel, (const AttnParams)p, (int)pl.grid);
         if (e != cudaSuccess) return cuda_fail(e, "verify_attention_merge_kernel launch");
     }
     return CS_OK;
