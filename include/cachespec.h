@@ -15,7 +15,9 @@
  *                          the drafted tokens;
  *   cs_spec_accept      -- the acceptance step: temperature softmax of target
  *                          and draft logits, accept test, residual / bonus
- *                          draw by inverse CDF, and its greedy variant.
+ *                          draw by inverse CDF, and its greedy variant;
+ *   cs_sample           -- the drafter's per-position sampling step (the same
+ *                          temperature softmax and inverse-CDF draw).
  *
  * Conventions for every entry point
  *   - All tensor arguments are DEVICE pointers owned by the caller, dense
@@ -198,6 +200,35 @@ cs_status cs_verify_attention_noalloc(const cs_attn_dims* dims, const void* q, c
                                       const void* v_pages, const int32_t* page_table,
                                       const int32_t* ctx_lens, int32_t n_draft, void* out,
                                       cs_stream_t stream);
+
+/*
+ * Draft-side sampling (the drafter's step before the verify pass: it
+ * proposes x_i ~ q_i one position at a time, Sec. 3.4), with the same
+ * conventions as the final draw of cs_spec_accept.
+ *
+ * For every request b:
+ *   T > 0: out_tokens[b] = the smallest token id whose running mass of
+ *          softmax(logits[b,:] / T) (ascending ids) exceeds uniforms[b]
+ *          times the total (if rounding leaves none, the largest id of
+ *          positive weight);
+ *   T == 0: out_tokens[b] = argmax logits[b,:] (lowest id on ties).
+ *
+ *   logits       [B, V] fp32 or bf16 (dims->logit_dtype), element-aligned
+ *   uniforms     fp32 [B] in [0, 1) (read only when T > 0)
+ *   temperature  T >= 0 and finite
+ *   out_tokens   int32 [B]
+ *   workspace    device scratch of at least cs_sample_workspace_bytes(dims)
+ *                bytes, 256-byte aligned, any initial contents; calls that
+ *                share one must be ordered.
+ *
+ * A logit of -inf marks a masked token; every row needs a finite entry.
+ * Returns CS_ERR_INVALID_ARG, CS_ERR_UNSUPPORTED (vocab above CS_MAX_VOCAB),
+ * CS_ERR_WORKSPACE or CS_ERR_CUDA.
+ */
+size_t cs_sample_workspace_bytes(const cs_accept_dims* dims);
+cs_status cs_sample(const cs_accept_dims* dims, const void* logits, const float* uniforms,
+                    float temperature, int32_t* out_tokens, void* workspace,
+                    size_t workspace_bytes, cs_stream_t stream);
 
 /*
  * Device status word of a verify-attention workspace: 0 when every call that

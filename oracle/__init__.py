@@ -59,6 +59,8 @@ def _load():
         lib.oracle_inverse_cdf.argtypes = [vp, f64, i32, f64, vp]
         lib.oracle_row_argmax.restype = i32
         lib.oracle_row_argmax.argtypes = [vp, i32, i32]
+        lib.oracle_sample.restype = ctypes.c_int
+        lib.oracle_sample.argtypes = [i32, i32, i32, vp, vp, f64, vp, vp]
         lib.oracle_max_threads.restype = ctypes.c_int
         lib.oracle_set_threads.argtypes = [ctypes.c_int]
         _lib = lib
@@ -152,6 +154,21 @@ def spec_accept(target, draft, draft_tokens, uniforms, temperature, with_draw_ma
     if with_draw_margin:
         return out, acc, margin, draw_margin
     return out, acc, margin
+
+
+def sample(logits, uniforms, temperature, with_margin=False):
+    """Draft-side sampling oracle: one token per row of ``logits`` [B, V] (bf16 bit
+    patterns or fp32); ``uniforms`` [B] (fp32 or fp64).  Returns tokens (and margins)."""
+    lib = _load()
+    z, code = _logit_array(np.asarray(logits))
+    B, V = z.shape
+    u = np.ascontiguousarray(np.asarray(uniforms, dtype=np.float64).reshape(B))
+    out = np.zeros(B, dtype=np.int32)
+    margin = np.zeros(B, dtype=np.float64)
+    rc = lib.oracle_sample(B, V, code, _ptr(z), _ptr(u), float(temperature), _ptr(out), _ptr(margin))
+    if rc != 0:
+        raise RuntimeError(f"oracle_sample failed with status {rc}")
+    return (out, margin) if with_margin else out
 
 
 def row_probs(row, temperature):

@@ -23,6 +23,9 @@
  *      the draw is the inverse CDF in ascending token id with uniform u_k.
  *   3. Greedy (T == 0): g_i = argmax z_t,i (lowest id on ties); accept x_i
  *      iff x_i == g_i; emit g_a.
+ *   4. Draft-side sampling (the drafter's per-position step before the
+ *      verify pass): x = inverse CDF of softmax(z / T) at u, ascending token
+ *      id, the computed total as the normaliser; T == 0 takes the argmax.
  *
  * Every floating-point step is fp64; inputs (bf16 bit patterns or fp32) are
  * widened exactly.  Loops run in the order the definition states (ascending
@@ -385,4 +388,44 @@ int oracle_spec_accept(int32_t batch, int32_t vocab, int32_t dtype,
                                            out_n_accepted, out_margin, out_draw_margin);
     free(u);
     return rc;
+}
+
+/* ------------------------------------------------------------------------
+ * 4. Draft-side sampling.
+ *
+ * For each row b: T > 0 draws out[b] = inverse CDF of p = softmax(z_b / T)
+ * at uniforms[b] (the total Z is the computed sum of p, as in the final draw
+ * of the acceptance step); T == 0 takes the argmax (lowest id on ties).
+ * out_margin[b] (may be NULL) is the distance of u from the two CDF values
+ * bracketing the drawn cell (+inf for greedy).
+ * ---------------------------------------------------------------------- */
+int oracle_sample(int32_t batch, int32_t vocab, int32_t dtype, const void* logits,
+                  const double* uniforms, double temperature, int32_t* out_tokens,
+                  double* out_margin) {
+    if (batch < 0 || vocab <= 0 || (dtype != 0 && dtype != 1)) return ORC_BAD_ARG;
+    if (!(temperature >= 0.0)) return ORC_BAD_ARG;
+    const size_t esz = dtype == 0 ? 4 : 2;
+    int status = ORC_OK;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t b = 0; b < batch; ++b) {
+        const char* row = (const char*)logits + (size_t)b * (size_t)vocab * esz;
+        double margin = INFINITY;
+        if (temperature == 0.0) {
+            out_tokens[b] = oracle_row_argmax(row, dtype, vocab);
+        } else {
+            double* p = (double*)malloc((size_t)vocab * sizeof(double));
+            if (!p) {
+#pragma omp atomic write
+                status = ORC_NO_MEM;
+                continue;
+            }
+            oracle_row_probs(row, dtype, vocab, temperature, p);
+            double Z = 0.0;
+            for (int64_t v = 0; v < vocab; ++v) Z += p[v];
+            out_tokens[b] = oracle_inverse_cdf(p, Z, vocab, uniforms[b], &margin);
+            free(p);
+        }
+        if (out_margin) out_margin[b] = margin;
+    }
+    return status;
 }

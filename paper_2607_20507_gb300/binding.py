@@ -22,7 +22,8 @@ STATUS_NAMES = {0: "CS_OK", 1: "CS_ERR_INVALID_ARG", 2: "CS_ERR_UNSUPPORTED", 3:
                 4: "CS_ERR_WORKSPACE"}
 EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_workspace_bytes",
                     "cs_verify_attention", "cs_spec_accept_workspace_bytes", "cs_spec_accept",
-                    "cs_read_device_status", "cs_verify_attention_noalloc")
+                    "cs_read_device_status", "cs_verify_attention_noalloc", "cs_sample_workspace_bytes",
+                    "cs_sample")
 
 
 class AttnDims(ctypes.Structure):
@@ -80,6 +81,10 @@ def load_library(path: str | None = None):
                                                     i32, vp, vp]
         lib.cs_read_device_status.restype = ctypes.c_int
         lib.cs_read_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_int32), vp]
+        lib.cs_sample_workspace_bytes.restype = sz
+        lib.cs_sample_workspace_bytes.argtypes = [ctypes.POINTER(AcceptDims)]
+        lib.cs_sample.restype = ctypes.c_int
+        lib.cs_sample.argtypes = [ctypes.POINTER(AcceptDims), vp, vp, ctypes.c_float, vp, vp, sz, vp]
         if path is None:
             _lib = lib
         return lib
@@ -215,6 +220,35 @@ def cs_spec_accept(target_logits, draft_logits, draft_tokens, uniforms, temperat
                             _stream(dev) if stream is None else stream)
     _check(lib, st)
     return out_tokens, out_n_accepted
+
+
+def cs_sample(logits, uniforms, temperature, out_tokens=None, workspace=None,
+              stream: int | None = None):
+    """Draft-side sampling, one token per row of ``logits`` [B, V]; returns out_tokens [B].
+    See include/cachespec.h."""
+    lib = load_library()
+    dev = logits.device
+    if logits.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("logits must be float32 or bfloat16")
+    _need(logits, "logits", logits.dtype, 2, dev)
+    B, V = logits.shape
+    _need(uniforms, "uniforms", torch.float32, 1, dev)
+    if out_tokens is None:
+        out_tokens = torch.empty((B,), dtype=torch.int32, device=dev)
+    _need(out_tokens, "out_tokens", torch.int32, 1, dev)
+    d = AcceptDims(B, V, CS_F32 if logits.dtype == torch.float32 else CS_BF16)
+    if workspace is None:
+        n = lib.cs_sample_workspace_bytes(ctypes.byref(d))
+        key = ("sample", str(dev), n)
+        workspace = _workspaces.get(key)
+        if workspace is None:
+            workspace = torch.zeros(max(n, 256), dtype=torch.uint8, device=dev)
+            _workspaces[key] = workspace
+    st = lib.cs_sample(ctypes.byref(d), _ptr(logits), _ptr(uniforms), float(temperature), _ptr(out_tokens),
+                       _ptr(workspace), workspace.numel() * workspace.element_size(),
+                       _stream(dev) if stream is None else stream)
+    _check(lib, st)
+    return out_tokens
 
 
 def cs_verify_attention_noalloc(q, k_pages, v_pages, page_table, ctx_lens, n_draft, out=None,

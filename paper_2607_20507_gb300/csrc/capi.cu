@@ -63,6 +63,20 @@ cs_status check_accept(const cs_accept_dims* d, int32_t n_draft, float temperatu
         return fail(CS_ERR_UNSUPPORTED, "vocab %d (this build implements up to %d)", d->vocab, CS_MAX_VOCAB);
     return CS_OK;
 }
+cs_status check_sample(const cs_accept_dims* d, float temperature) {
+    if (!d) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
+    if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
+    if (d->vocab <= 0) return fail(CS_ERR_INVALID_ARG, "vocab %d <= 0", d->vocab);
+    if (d->logit_dtype != CS_F32 && d->logit_dtype != CS_BF16)
+        return fail(CS_ERR_INVALID_ARG, "logit_dtype %d is neither CS_F32 nor CS_BF16", d->logit_dtype);
+    if (!(temperature >= 0.f) || isinf(temperature))
+        return fail(CS_ERR_INVALID_ARG, "temperature must be finite and >= 0");
+    if ((long long)d->batch * (long long)d->vocab > (1LL << 46))
+        return fail(CS_ERR_INVALID_ARG, "logit tensor too large");
+    if (d->vocab > CS_MAX_VOCAB)
+        return fail(CS_ERR_UNSUPPORTED, "vocab %d (this build implements up to %d)", d->vocab, CS_MAX_VOCAB);
+    return CS_OK;
+}
 }  // namespace
 
 cs_status fail(cs_status st, const char* fmt, ...) {
@@ -158,6 +172,32 @@ cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
     return launch_spec_accept(*dims, target_logits, temperature > 0.f ? draft_logits : nullptr,
                               draft_tokens, uniforms, n_draft, temperature, out_tokens,
                               out_n_accepted, workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t cs_sample_workspace_bytes(const cs_accept_dims* dims) {
+    if (check_sample(dims, 1.0f) != CS_OK) return 0;
+    return accept_workspace_bytes_any(*dims, 0);
+}
+
+cs_status cs_sample(const cs_accept_dims* dims, const void* logits, const float* uniforms,
+                    float temperature, int32_t* out_tokens, void* workspace, size_t workspace_bytes,
+                    cs_stream_t stream) {
+    cs_status st = check_sample(dims, temperature);
+    if (st != CS_OK) return st;
+    if (dims->batch == 0) return CS_OK;
+    if (!logits || !uniforms || !out_tokens) return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    const size_t esz = dims->logit_dtype == CS_F32 ? 4 : 2;
+    if (!aligned(logits, esz)) return fail(CS_ERR_INVALID_ARG, "logits must be aligned to their element size");
+    if (!aligned(uniforms, 4) || !aligned(out_tokens, 4))
+        return fail(CS_ERR_INVALID_ARG, "int32/fp32 pointers must be 4-byte aligned");
+    const size_t need = accept_workspace_bytes(*dims, 0, temperature);
+    if (!workspace || workspace_bytes < need)
+        return fail(CS_ERR_WORKSPACE, "workspace of %zu bytes given, %zu needed", workspace_bytes, need);
+    if (!aligned(workspace, 256)) return fail(CS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    // the acceptance path with no drafted positions: every request decides
+    // a = 0 and draws its token from p_0 (or takes its argmax when T == 0)
+    return launch_spec_accept(*dims, logits, nullptr, nullptr, uniforms, 0, temperature, out_tokens,
+                              nullptr, workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
 cs_status cs_read_device_status(const void* workspace, int32_t* status_out, cs_stream_t stream) {

@@ -56,7 +56,7 @@ struct AcceptParams {
     const int32_t* tokens;    // [B, k]
     const float* uniforms;    // [B, k+1]
     int32_t* out_tokens;      // [B, k+1]
-    int32_t* out_n;           // [B]
+    int32_t* out_n;           // [B], or null (the sampler)
     int B, V, k;
     int R;                    // rows per request: 2k+1 (sampling) or k+1 (greedy)
     int I;                    // 4 KB items per row
@@ -707,7 +707,7 @@ __global__ void __launch_bounds__(kDrawThreads, 2) accept_draw_kernel(const Acce
         const int32_t x = tid < a ? __ldg(p.tokens + (size_t)b * k + tid) : -1;
         p.out_tokens[(size_t)b * (k + 1) + tid] = x;
     }
-    if (rank == 0 && tid == 0) p.out_n[b] = a;
+    if (rank == 0 && tid == 0 && p.out_n) p.out_n[b] = a;
     // no CTA leaves while another may still read its exchange slots
     cluster_arrive();
     cluster_wait();
@@ -734,7 +734,7 @@ __global__ void __launch_bounds__(kThreads) accept_greedy_kernel(const AcceptPar
     const int a = miss ? __ffs(miss) - 1 : k;
     const int emit = __shfl_sync(0xffffffffu, g, a);
     if (lane <= k) p.out_tokens[(size_t)b * (k + 1) + lane] = lane < a ? x : (lane == a ? emit : -1);
-    if (lane == 0) p.out_n[b] = a;
+    if (lane == 0 && p.out_n) p.out_n[b] = a;
 }
 
 // ------------------------------------------------------------------- host

@@ -153,6 +153,26 @@ def test_spec_accept_null_and_alignment(lib):
     assert accept(lib, dims, ws_bytes=need - 1) == binding.CS_ERR_WORKSPACE
 
 
+def sample(lib, dims, T=1.0, z=FAKE, u=FAKE, out=FAKE, ws=FAKE, ws_bytes=1 << 40):
+    return lib.cs_sample(ctypes.byref(dims), z, u, T, out, ws, ws_bytes, None)
+
+
+def test_sample_argument_checks(lib):
+    dims = binding.AcceptDims(4, 32000, binding.CS_BF16)
+    for arg in ("z", "u", "out"):
+        assert sample(lib, dims, **{arg: None}) == binding.CS_ERR_INVALID_ARG
+    for T in (-1.0, float("nan"), float("inf")):
+        assert sample(lib, dims, T=T) == binding.CS_ERR_INVALID_ARG
+    assert sample(lib, binding.AcceptDims(4, 32000, 9)) == binding.CS_ERR_INVALID_ARG
+    assert sample(lib, binding.AcceptDims(4, (1 << 22) + 1, binding.CS_BF16)) == binding.CS_ERR_UNSUPPORTED
+    need = lib.cs_sample_workspace_bytes(ctypes.byref(dims))
+    assert need >= 4 * 16 * 8                 # one pair per 4 KB item of each row
+    assert sample(lib, dims, ws=None) == binding.CS_ERR_WORKSPACE
+    assert sample(lib, dims, ws_bytes=need - 1) == binding.CS_ERR_WORKSPACE
+    assert sample(lib, dims, ws=FAKE + 64) == binding.CS_ERR_INVALID_ARG
+    assert sample(lib, binding.AcceptDims(0, 100, binding.CS_F32), z=None, u=None, out=None, ws=None) == binding.CS_OK
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     with pytest.raises(RuntimeError, match="not found"):
         binding.load_library(str(tmp_path / "missing.so"))
