@@ -17,7 +17,11 @@
  *                          and draft logits, accept test, residual / bonus
  *                          draw by inverse CDF, and its greedy variant;
  *   cs_sample           -- the drafter's per-position sampling step (the same
- *                          temperature softmax and inverse-CDF draw).
+ *                          temperature softmax and inverse-CDF draw);
+ *   cs_kv_append,
+ *   cs_kv_commit        -- the paged KV cache around the verify pass: append
+ *                          the verify positions' K/V rows, then keep the
+ *                          accepted prefix.
  *
  * Conventions for every entry point
  *   - All tensor arguments are DEVICE pointers owned by the caller, dense
@@ -200,6 +204,40 @@ cs_status cs_verify_attention_noalloc(const cs_attn_dims* dims, const void* q, c
                                       const void* v_pages, const int32_t* page_table,
                                       const int32_t* ctx_lens, int32_t n_draft, void* out,
                                       cs_stream_t stream);
+
+/*
+ * Paged KV cache around the verify pass (Sec. 3.4's draft-and-verify step).
+ *
+ * cs_kv_append writes the K and V rows of the n_new newest positions of
+ * every request into its pages before verify attention (n_new = k+1: the
+ * last committed token and the k drafts).  ctx_lens[b] = L_b already counts
+ * them (clamped to [0, max_pages_per_seq*page_size], as in
+ * cs_verify_attention), so row i of request b, KV head h lands at key
+ * position L_b - n_new + i: slot (L_b - n_new + i) % ps of page
+ * page_table[b][(L_b - n_new + i) / ps].  A row whose position is negative
+ * or whose page id lies outside [0, num_pages) is not written.
+ *
+ *   dims        the pool geometry (head_dim 128; n_q_heads and sm_scale unused)
+ *   new_k/new_v bf16 [B, n_new, Hkv, 128], 16-byte aligned
+ *   k_pages/v_pages bf16 [P, Hkv, ps, 128], 16-byte aligned, updated in place
+ *   page_table  int32 [B, max_pages_per_seq]; ctx_lens int32 [B]
+ *   n_new       in [1, 4096]
+ * Requests must not share the page slots they write (the writes would race).
+ *
+ * cs_kv_commit shortens every context after the acceptance step to the rows
+ * that stay valid: the prefix, the last committed token and the accepted
+ * drafts, ctx_lens[b] <- max(0, ctx_lens[b] - n_draft + n_accepted[b]).
+ * The emitted token (residual or bonus draw) has no row yet: it is the first
+ * input of the next step.  Pages past the new length are not released.
+ *
+ * Both return CS_ERR_INVALID_ARG (null pointer, misalignment, bad dimension
+ * or count), CS_ERR_UNSUPPORTED (head_dim != 128) or CS_ERR_CUDA.
+ */
+cs_status cs_kv_append(const cs_attn_dims* dims, const void* new_k, const void* new_v, void* k_pages,
+                       void* v_pages, const int32_t* page_table, const int32_t* ctx_lens, int32_t n_new,
+                       cs_stream_t stream);
+cs_status cs_kv_commit(int32_t batch, int32_t* ctx_lens, const int32_t* n_accepted, int32_t n_draft,
+                       cs_stream_t stream);
 
 /*
  * Draft-side sampling (the drafter's step before the verify pass: it

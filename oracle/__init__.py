@@ -59,6 +59,10 @@ def _load():
         lib.oracle_inverse_cdf.argtypes = [vp, f64, i32, f64, vp]
         lib.oracle_row_argmax.restype = i32
         lib.oracle_row_argmax.argtypes = [vp, i32, i32]
+        lib.oracle_kv_append.restype = ctypes.c_int
+        lib.oracle_kv_append.argtypes = [i32] * 6 + [vp] * 6 + [i32]
+        lib.oracle_kv_commit.restype = ctypes.c_int
+        lib.oracle_kv_commit.argtypes = [i32, vp, vp, i32]
         lib.oracle_sample.restype = ctypes.c_int
         lib.oracle_sample.argtypes = [i32, i32, i32, vp, vp, f64, vp, vp]
         lib.oracle_max_threads.restype = ctypes.c_int
@@ -169,6 +173,33 @@ def sample(logits, uniforms, temperature, with_margin=False):
     if rc != 0:
         raise RuntimeError(f"oracle_sample failed with status {rc}")
     return (out, margin) if with_margin else out
+
+
+def kv_append(new_k, new_v, k_pages, v_pages, page_table, ctx_lens):
+    """Paged append in place on numpy uint16 (bf16 bit) pools; new rows [B, n_new, Hkv, D]."""
+    lib = _load()
+    nk = np.ascontiguousarray(new_k, dtype=np.uint16)
+    nv = np.ascontiguousarray(new_v, dtype=np.uint16)
+    assert k_pages.dtype == np.uint16 and k_pages.flags.c_contiguous and v_pages.flags.c_contiguous
+    B, n_new, Hkv, D = nk.shape
+    P, _, ps, _ = k_pages.shape
+    pt = np.ascontiguousarray(page_table, dtype=np.int32)
+    cl = np.ascontiguousarray(ctx_lens, dtype=np.int32)
+    rc = lib.oracle_kv_append(B, Hkv, D, ps, pt.shape[1], P, _ptr(nk), _ptr(nv), _ptr(k_pages),
+                              _ptr(v_pages), _ptr(pt), _ptr(cl), n_new)
+    if rc != 0:
+        raise RuntimeError(f"oracle_kv_append failed with status {rc}")
+
+
+def kv_commit(ctx_lens, n_accepted, n_draft):
+    """New context lengths after the acceptance step (returns a new int32 array)."""
+    lib = _load()
+    cl = np.array(ctx_lens, dtype=np.int32)
+    na = np.ascontiguousarray(n_accepted, dtype=np.int32)
+    rc = lib.oracle_kv_commit(cl.shape[0], _ptr(cl), _ptr(na), int(n_draft))
+    if rc != 0:
+        raise RuntimeError(f"oracle_kv_commit failed with status {rc}")
+    return cl
 
 
 def row_probs(row, temperature):

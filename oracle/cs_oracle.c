@@ -26,6 +26,11 @@
  *   4. Draft-side sampling (the drafter's per-position step before the
  *      verify pass): x = inverse CDF of softmax(z / T) at u, ascending token
  *      id, the computed total as the normaliser; T == 0 takes the argmax.
+ *   5. Paged KV cache: the k+1 verify positions' K/V rows go to key
+ *      positions L_b-(k+1) .. L_b-1 of their request (slot pos % ps of page
+ *      page_table[b][pos / ps]); after the acceptance step the context keeps
+ *      L_b - k + a rows (the prefix, the verify input token and the a
+ *      accepted drafts).
  *
  * Every floating-point step is fp64; inputs (bf16 bit patterns or fp32) are
  * widened exactly.  Loops run in the order the definition states (ascending
@@ -428,4 +433,51 @@ int oracle_sample(int32_t batch, int32_t vocab, int32_t dtype, const void* logit
         if (out_margin) out_margin[b] = margin;
     }
     return status;
+}
+
+/* ------------------------------------------------------------------------
+ * 5. Paged KV cache.
+ *
+ * Append: rows are bf16 bit patterns.  For request b, new row i, KV head h:
+ * pos = L_b - n_new + i with L_b clamped to [0, max_pages * ps]; when
+ * pos >= 0 and the page id is in [0, num_pages), copy the D values into
+ * pool[page][h][pos % ps].  Commit: L_b <- max(0, L_b - n_draft + a_b).
+ * ---------------------------------------------------------------------- */
+int oracle_kv_append(int32_t batch, int32_t n_kv_heads, int32_t head_dim, int32_t page_size,
+                     int32_t max_pages, int32_t num_pages, const uint16_t* new_k,
+                     const uint16_t* new_v, uint16_t* k_pages, uint16_t* v_pages,
+                     const int32_t* page_table, const int32_t* ctx_lens, int32_t n_new) {
+    if (batch < 0 || n_kv_heads <= 0 || head_dim <= 0 || page_size <= 0 || max_pages <= 0 ||
+        num_pages <= 0 || n_new < 1)
+        return ORC_BAD_ARG;
+    const int64_t cap = (int64_t)max_pages * page_size;
+    for (int64_t b = 0; b < batch; ++b) {
+        int64_t L = ctx_lens[b];
+        if (L < 0) L = 0;
+        if (L > cap) L = cap;
+        for (int64_t i = 0; i < n_new; ++i) {
+            const int64_t pos = L - n_new + i;
+            if (pos < 0) continue;
+            const int64_t page = page_table[b * max_pages + pos / page_size];
+            if (page < 0 || page >= num_pages) continue;
+            for (int64_t h = 0; h < n_kv_heads; ++h) {
+                const int64_t src = ((b * n_new + i) * n_kv_heads + h) * head_dim;
+                const int64_t dst = ((page * n_kv_heads + h) * page_size + pos % page_size) * head_dim;
+                for (int64_t e = 0; e < head_dim; ++e) {
+                    k_pages[dst + e] = new_k[src + e];
+                    v_pages[dst + e] = new_v[src + e];
+                }
+            }
+        }
+    }
+    return ORC_OK;
+}
+
+int oracle_kv_commit(int32_t batch, int32_t* ctx_lens, const int32_t* n_accepted, int32_t n_draft) {
+    if (batch < 0 || n_draft < 0) return ORC_BAD_ARG;
+    for (int64_t b = 0; b < batch; ++b) {
+        const int64_t L = (int64_t)ctx_lens[b] - n_draft + n_accepted[b];
+        ctx_lens[b] = (int32_t)(L > 0 ? L : 0);
+    }
+    return ORC_OK;
 }

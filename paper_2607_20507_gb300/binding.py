@@ -23,7 +23,7 @@ STATUS_NAMES = {0: "CS_OK", 1: "CS_ERR_INVALID_ARG", 2: "CS_ERR_UNSUPPORTED", 3:
 EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_workspace_bytes",
                     "cs_verify_attention", "cs_spec_accept_workspace_bytes", "cs_spec_accept",
                     "cs_read_device_status", "cs_verify_attention_noalloc", "cs_sample_workspace_bytes",
-                    "cs_sample")
+                    "cs_sample", "cs_kv_append", "cs_kv_commit")
 
 
 class AttnDims(ctypes.Structure):
@@ -81,6 +81,10 @@ def load_library(path: str | None = None):
                                                     i32, vp, vp]
         lib.cs_read_device_status.restype = ctypes.c_int
         lib.cs_read_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_int32), vp]
+        lib.cs_kv_append.restype = ctypes.c_int
+        lib.cs_kv_append.argtypes = [ctypes.POINTER(AttnDims), vp, vp, vp, vp, vp, vp, i32, vp]
+        lib.cs_kv_commit.restype = ctypes.c_int
+        lib.cs_kv_commit.argtypes = [i32, vp, vp, i32, vp]
         lib.cs_sample_workspace_bytes.restype = sz
         lib.cs_sample_workspace_bytes.argtypes = [ctypes.POINTER(AcceptDims)]
         lib.cs_sample.restype = ctypes.c_int
@@ -220,6 +224,38 @@ def cs_spec_accept(target_logits, draft_logits, draft_tokens, uniforms, temperat
                             _stream(dev) if stream is None else stream)
     _check(lib, st)
     return out_tokens, out_n_accepted
+
+
+def cs_kv_append(new_k, new_v, k_pages, v_pages, page_table, ctx_lens, stream: int | None = None):
+    """Append the K/V rows of the newest positions into the page pools (in place).
+    new_k / new_v bf16 [B, n_new, Hkv, D]; pools [P, Hkv, ps, D].  See include/cachespec.h."""
+    lib = load_library()
+    dev = k_pages.device
+    _need(new_k, "new_k", torch.bfloat16, 4, dev)
+    _need(new_v, "new_v", torch.bfloat16, 4, dev)
+    _need(k_pages, "k_pages", torch.bfloat16, 4, dev)
+    _need(v_pages, "v_pages", torch.bfloat16, 4, dev)
+    _need(page_table, "page_table", torch.int32, 2, dev)
+    _need(ctx_lens, "ctx_lens", torch.int32, 1, dev)
+    B, n_new, Hkv, D = new_k.shape
+    P, Hkv2, ps, D2 = k_pages.shape
+    if tuple(new_v.shape) != tuple(new_k.shape) or Hkv2 != Hkv or D2 != D or k_pages.shape != v_pages.shape:
+        raise ValueError("new rows and pools do not match")
+    d = AttnDims(B, Hkv, Hkv, D, ps, page_table.shape[1], P, 0.0)
+    st = lib.cs_kv_append(ctypes.byref(d), _ptr(new_k), _ptr(new_v), _ptr(k_pages), _ptr(v_pages),
+                          _ptr(page_table), _ptr(ctx_lens), int(n_new), _stream(dev) if stream is None else stream)
+    _check(lib, st)
+
+
+def cs_kv_commit(ctx_lens, n_accepted, n_draft: int, stream: int | None = None):
+    """Keep the accepted prefix: ctx_lens <- max(0, ctx_lens - k + n_accepted), in place."""
+    lib = load_library()
+    dev = ctx_lens.device
+    _need(ctx_lens, "ctx_lens", torch.int32, 1, dev)
+    _need(n_accepted, "n_accepted", torch.int32, 1, dev)
+    st = lib.cs_kv_commit(int(ctx_lens.shape[0]), _ptr(ctx_lens), _ptr(n_accepted), int(n_draft),
+                          _stream(dev) if stream is None else stream)
+    _check(lib, st)
 
 
 def cs_sample(logits, uniforms, temperature, out_tokens=None, workspace=None,

@@ -174,6 +174,40 @@ cs_status cs_spec_accept(const cs_accept_dims* dims, const void* target_logits,
                               out_n_accepted, workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
+cs_status cs_kv_append(const cs_attn_dims* dims, const void* new_k, const void* new_v, void* k_pages,
+                       void* v_pages, const int32_t* page_table, const int32_t* ctx_lens, int32_t n_new,
+                       cs_stream_t stream) {
+    if (!dims) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
+    const cs_attn_dims* d = dims;
+    if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
+    if (d->n_kv_heads <= 0 || d->page_size <= 0 || d->max_pages_per_seq <= 0 || d->num_pages <= 0)
+        return fail(CS_ERR_INVALID_ARG, "n_kv_heads, page_size, max_pages_per_seq and num_pages must be positive");
+    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this build implements 128)", d->head_dim);
+    if (n_new < 1 || n_new > 4096) return fail(CS_ERR_INVALID_ARG, "n_new %d not in [1, 4096]", n_new);
+    if ((long long)d->max_pages_per_seq * d->page_size > (1LL << 30))
+        return fail(CS_ERR_INVALID_ARG, "max_pages_per_seq * page_size exceeds 2^30 keys");
+    if (d->batch == 0) return CS_OK;
+    if (!new_k || !new_v || !k_pages || !v_pages || !page_table || !ctx_lens)
+        return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (!aligned(new_k, 16) || !aligned(new_v, 16) || !aligned(k_pages, 16) || !aligned(v_pages, 16))
+        return fail(CS_ERR_INVALID_ARG, "new rows and page pools must be 16-byte aligned");
+    if (!aligned(page_table, 4) || !aligned(ctx_lens, 4))
+        return fail(CS_ERR_INVALID_ARG, "page_table and ctx_lens must be 4-byte aligned");
+    return launch_kv_append(*d, new_k, new_v, k_pages, v_pages, page_table, ctx_lens, n_new,
+                            reinterpret_cast<cudaStream_t>(stream));
+}
+
+cs_status cs_kv_commit(int32_t batch, int32_t* ctx_lens, const int32_t* n_accepted, int32_t n_draft,
+                       cs_stream_t stream) {
+    if (batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", batch);
+    if (n_draft < 0 || n_draft > 16) return fail(CS_ERR_INVALID_ARG, "n_draft %d not in [0, 16]", n_draft);
+    if (batch == 0) return CS_OK;
+    if (!ctx_lens || !n_accepted) return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (!aligned(ctx_lens, 4) || !aligned(n_accepted, 4))
+        return fail(CS_ERR_INVALID_ARG, "ctx_lens and n_accepted must be 4-byte aligned");
+    return launch_kv_commit(ctx_lens, n_accepted, batch, n_draft, reinterpret_cast<cudaStream_t>(stream));
+}
+
 size_t cs_sample_workspace_bytes(const cs_accept_dims* dims) {
     if (check_sample(dims, 1.0f) != CS_OK) return 0;
     return accept_workspace_bytes_any(*dims, 0);

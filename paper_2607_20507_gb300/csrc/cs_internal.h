@@ -42,4 +42,11 @@ cs_status launch_spec_accept(const cs_accept_dims& d, const void* target, const 
                              float temperature, int32_t* out_tokens, int32_t* out_n,
                              void* workspace, cudaStream_t stream);
 
+// ------------------------------------------------------------- KV cache
+cs_status launch_kv_append(const cs_attn_dims& d, const void* new_k, const void* new_v, void* k_pages,
+                           void* v_pages, const int32_t* page_table, const int32_t* ctx_lens, int n_new,
+                           cudaStream_t stream);
+cs_status launch_kv_commit(int32_t* ctx_lens, const int32_t* n_accepted, int batch, int n_draft,
+                           cudaStream_t stream);
+
 }  // namespace cs

@@ -173,6 +173,26 @@ def test_sample_argument_checks(lib):
     assert sample(lib, binding.AcceptDims(0, 100, binding.CS_F32), z=None, u=None, out=None, ws=None) == binding.CS_OK
 
 
+def test_kv_argument_checks(lib):
+    d = good_attn_dims()
+    append = lambda dims=d, n=6, **kw: lib.cs_kv_append(ctypes.byref(dims), kw.get("nk", FAKE), kw.get("nv", FAKE),
+                                                        kw.get("kp", FAKE), kw.get("vp", FAKE), kw.get("pt", FAKE),
+                                                        kw.get("cl", FAKE), n, None)
+    for arg in ("nk", "nv", "kp", "vp", "pt", "cl"):
+        assert append(**{arg: None}) == binding.CS_ERR_INVALID_ARG
+    assert append(nk=FAKE + 8) == binding.CS_ERR_INVALID_ARG
+    assert append(n=0) == binding.CS_ERR_INVALID_ARG
+    bad = good_attn_dims()
+    bad.head_dim = 64
+    assert append(dims=bad) == binding.CS_ERR_UNSUPPORTED
+    empty = good_attn_dims()
+    empty.batch = 0
+    assert append(dims=empty, nk=None, nv=None, kp=None, vp=None, pt=None, cl=None) == binding.CS_OK
+    assert lib.cs_kv_commit(4, None, FAKE, 5, None) == binding.CS_ERR_INVALID_ARG
+    assert lib.cs_kv_commit(4, FAKE, FAKE, 17, None) == binding.CS_ERR_INVALID_ARG
+    assert lib.cs_kv_commit(0, None, None, 5, None) == binding.CS_OK
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     with pytest.raises(RuntimeError, match="not found"):
         binding.load_library(str(tmp_path / "missing.so"))
