@@ -364,6 +364,19 @@ def run_gb300(args) -> dict | None:
                                "rows": int(B * (k + 1) * Hkv_)},
                  "draft_sample": {"us": 1e6 * t_smp, "bytes": smp_bytes, "gbs": smp_bytes / t_smp / 1e9,
                                   "rows": B, "vocab": int(d_logits.shape[1])}}
+    # the front end's semantic routing (one batch of request embeddings
+    # against the group centroids), at two group-index sizes
+    for rw in (W.ROUTE_WORKLOADS[2], W.ROUTE_WORKLOADS[3]):
+        rx = W.route_inputs(rw, dev)
+        r_inv = binding.cs_route_norms(rx["centroids"])
+        r_out = [torch.empty(rw.batch, dtype=dt, device=dev) for dt in (torch.int32, torch.int32, torch.float32)]
+        t_rt = timed_graph(lambda: binding.cs_route(rx["emb"], rx["centroids"], r_inv, W.ROUTE_TAU, *r_out))
+        flops = 2.0 * rw.batch * rw.n_groups * rw.dim
+        r_bytes = (rw.batch + rw.n_groups) * rw.dim * 2 + rw.n_groups * 4 + rw.batch * 12
+        next_rows[f"route_b{rw.batch}_g{rw.n_groups}"] = {
+            "us": 1e6 * t_rt, "tflops": flops / t_rt / 1e12, "flops": flops, "bytes": r_bytes,
+            "hit_rate": float((r_out[0] >= 0).float().mean().item())}
+        del rx, r_inv, r_out
 
     # end to end through the public API: inputs start in pinned host memory
     host = {name: t.cpu().pin_memory() for name, t in

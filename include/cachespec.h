@@ -21,7 +21,9 @@
  *   cs_kv_append,
  *   cs_kv_commit        -- the paged KV cache around the verify pass: append
  *                          the verify positions' K/V rows, then keep the
- *                          accepted prefix.
+ *                          accepted prefix;
+ *   cs_route            -- the front end's batched semantic routing: cosine
+ *                          scores against group centroids, arg max, threshold.
  *
  * Conventions for every entry point
  *   - All tensor arguments are DEVICE pointers owned by the caller, dense
@@ -77,6 +79,14 @@ typedef struct {
     int32_t vocab;              /* V > 0 */
     int32_t logit_dtype;        /* cs_dtype of target and draft logits */
 } cs_accept_dims;
+
+/* Geometry of one routing call. */
+typedef struct {
+    int32_t batch;              /* B >= 0 requests */
+    int32_t n_groups;           /* N >= 0 groups (0: every request misses) */
+    int32_t dim;                /* embedding width, a multiple of 64 up to CS_MAX_ROUTE_DIM */
+} cs_route_dims;
+#define CS_MAX_ROUTE_DIM 384
 
 /* ABI version of this header (bumped on any incompatible change). */
 #define CS_ABI_VERSION 1
@@ -238,6 +248,43 @@ cs_status cs_kv_append(const cs_attn_dims* dims, const void* new_k, const void* 
                        cs_stream_t stream);
 cs_status cs_kv_commit(int32_t batch, int32_t* ctx_lens, const int32_t* n_accepted, int32_t n_draft,
                        cs_stream_t stream);
+
+/*
+ * Batched semantic routing (the paper's front end, Sec. 3.1): the score of
+ * request b against group i is the cosine similarity of their embeddings,
+ *     S(b, i) = (e_b . c_i) / (|e_b| |c_i|)   (0 when either norm is 0);
+ * out_best[b] = argmax_i S(b, i) (the lowest i on ties; -1 when N == 0),
+ * out_score[b] = that score (-inf when N == 0), and
+ * out_group[b] = out_best[b] when out_score[b] >= tau, else -1 (the request
+ * goes to the cache-miss branch).
+ *
+ *   emb        bf16 [B, dim], 16-byte aligned
+ *   centroids  bf16 [N, dim], 16-byte aligned (may be NULL when N == 0)
+ *   inv_norms  fp32 [N]: 1/|c_i| (0 for a zero row), as written by
+ *              cs_route_norms for the same centroids (may be NULL when N == 0)
+ *   tau        the matching threshold, finite
+ *   out_*      int32 / fp32 [B]
+ *   workspace  at least cs_route_workspace_bytes(dims) bytes, 256-byte
+ *              aligned, any initial contents; calls sharing one must be
+ *              ordered.  Its first 4 bytes are the device status word
+ *              (cs_read_device_status); zero-fill the workspace before its
+ *              first use.
+ * The scores are fp32 sums of exact bf16 products: they differ from exact
+ * cosines by at most ~dim * 2^-24 relative.
+ *
+ * cs_route_norms writes inv_norms for N centroids (run it whenever the
+ * centroids change).
+ *
+ * Return CS_ERR_INVALID_ARG (null pointer, misalignment, bad count or
+ * threshold), CS_ERR_UNSUPPORTED (dim not a multiple of 64 in
+ * [64, CS_MAX_ROUTE_DIM]), CS_ERR_WORKSPACE or CS_ERR_CUDA.
+ */
+size_t cs_route_workspace_bytes(const cs_route_dims* dims);
+cs_status cs_route_norms(int32_t n_groups, int32_t dim, const void* centroids, float* inv_norms,
+                         cs_stream_t stream);
+cs_status cs_route(const cs_route_dims* dims, const void* emb, const void* centroids,
+                   const float* inv_norms, float tau, int32_t* out_group, int32_t* out_best,
+                   float* out_score, void* workspace, size_t workspace_bytes, cs_stream_t stream);
 
 /*
  * Draft-side sampling (the drafter's step before the verify pass: it

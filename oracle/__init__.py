@@ -63,6 +63,8 @@ def _load():
         lib.oracle_kv_append.argtypes = [i32] * 6 + [vp] * 6 + [i32]
         lib.oracle_kv_commit.restype = ctypes.c_int
         lib.oracle_kv_commit.argtypes = [i32, vp, vp, i32]
+        lib.oracle_route.restype = ctypes.c_int
+        lib.oracle_route.argtypes = [i32, i32, i32, vp, vp, f64, vp, vp, vp, vp, vp]
         lib.oracle_sample.restype = ctypes.c_int
         lib.oracle_sample.argtypes = [i32, i32, i32, vp, vp, f64, vp, vp]
         lib.oracle_max_threads.restype = ctypes.c_int
@@ -200,6 +202,25 @@ def kv_commit(ctx_lens, n_accepted, n_draft):
     if rc != 0:
         raise RuntimeError(f"oracle_kv_commit failed with status {rc}")
     return cl
+
+
+def route(emb_bits, centroid_bits, tau):
+    """fp64 semantic routing.  emb [B, d] and centroids [N, d] as uint16 bf16 bits.
+    Returns dict(group, best, score, margin, tau_margin)."""
+    lib = _load()
+    e = np.ascontiguousarray(emb_bits, dtype=np.uint16)
+    c = np.ascontiguousarray(centroid_bits, dtype=np.uint16)
+    B, d = e.shape
+    N = c.shape[0] if c.size else 0
+    if N:
+        assert c.shape[1] == d
+    out = {k: np.zeros(B, dtype=np.int32) for k in ("group", "best")}
+    out.update({k: np.zeros(B, dtype=np.float64) for k in ("score", "margin", "tau_margin")})
+    rc = lib.oracle_route(B, N, d, _ptr(e), _ptr(c) if N else None, float(tau), _ptr(out["group"]),
+                          _ptr(out["best"]), _ptr(out["score"]), _ptr(out["margin"]), _ptr(out["tau_margin"]))
+    if rc != 0:
+        raise RuntimeError(f"oracle_route failed with status {rc}")
+    return out
 
 
 def row_probs(row, temperature):

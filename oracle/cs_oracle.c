@@ -26,6 +26,10 @@
  *   4. Draft-side sampling (the drafter's per-position step before the
  *      verify pass): x = inverse CDF of softmax(z / T) at u, ascending token
  *      id, the computed total as the normaliser; T == 0 takes the argmax.
+ *   6. Semantic routing (Sec. 3.1): the score of request x against group G_i
+ *      is the cosine similarity of its embedding with the group's centroid;
+ *      i* = argmax_i (lowest i on ties); a score below tau sends x to the
+ *      cache-miss branch (group -1).
  *   5. Paged KV cache: the k+1 verify positions' K/V rows go to key
  *      positions L_b-(k+1) .. L_b-1 of their request (slot pos % ps of page
  *      page_table[b][pos / ps]); after the acceptance step the context keeps
@@ -479,5 +483,64 @@ int oracle_kv_commit(int32_t batch, int32_t* ctx_lens, const int32_t* n_accepted
         const int64_t L = (int64_t)ctx_lens[b] - n_draft + n_accepted[b];
         ctx_lens[b] = (int32_t)(L > 0 ? L : 0);
     }
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------
+ * 6. Semantic routing.
+ *
+ * emb [B, d] and centroids [N, d] are bf16 bit patterns, widened exactly.
+ * S(b, i) = (e_b . c_i) / (|e_b| |c_i|), 0 when either norm is 0; every
+ * product and sum in fp64, ascending index.  out_best[b] = argmax_i S (the
+ * lowest i on ties; -1 when N == 0), out_score[b] = that S (-inf when
+ * N == 0), out_group[b] = out_best[b] if out_score[b] >= tau else -1.
+ * out_margin[b] (may be NULL) = best score minus the runner-up (+inf when
+ * N < 2); out_tau_margin[b] (may be NULL) = |best score - tau|.
+ * ---------------------------------------------------------------------- */
+static double bf16_at(const uint16_t* p, int64_t i) { return bf16_bits_to_double(p[i]); }
+
+int oracle_route(int32_t batch, int32_t n_groups, int32_t dim, const uint16_t* emb,
+                 const uint16_t* centroids, double tau, int32_t* out_group, int32_t* out_best,
+                 double* out_score, double* out_margin, double* out_tau_margin) {
+    if (batch < 0 || n_groups < 0 || dim <= 0) return ORC_BAD_ARG;
+    double* cn = (double*)malloc(((size_t)n_groups + 1) * sizeof(double));
+    if (!cn) return ORC_NO_MEM;
+    for (int64_t i = 0; i < n_groups; ++i) {
+        double s = 0.0;
+        for (int64_t k = 0; k < dim; ++k) {
+            const double c = bf16_at(centroids, i * dim + k);
+            s += c * c;
+        }
+        cn[i] = sqrt(s);
+    }
+#pragma omp parallel for schedule(dynamic, 16)
+    for (int64_t b = 0; b < batch; ++b) {
+        double en = 0.0;
+        for (int64_t k = 0; k < dim; ++k) {
+            const double e = bf16_at(emb, b * dim + k);
+            en += e * e;
+        }
+        en = sqrt(en);
+        double best = -INFINITY, second = -INFINITY;
+        int32_t arg = -1;
+        for (int64_t i = 0; i < n_groups; ++i) {
+            double dot = 0.0;
+            for (int64_t k = 0; k < dim; ++k) dot += bf16_at(emb, b * dim + k) * bf16_at(centroids, i * dim + k);
+            const double s = (en > 0.0 && cn[i] > 0.0) ? dot / (en * cn[i]) : 0.0;
+            if (s > best) {
+                second = best;
+                best = s;
+                arg = (int32_t)i;
+            } else if (s > second) {
+                second = s;
+            }
+        }
+        out_best[b] = arg;
+        out_score[b] = best;
+        out_group[b] = (arg >= 0 && best >= tau) ? arg : -1;
+        if (out_margin) out_margin[b] = n_groups >= 2 ? best - second : INFINITY;
+        if (out_tau_margin) out_tau_margin[b] = fabs(best - tau);
+    }
+    free(cn);
     return ORC_OK;
 }

@@ -23,7 +23,12 @@ STATUS_NAMES = {0: "CS_OK", 1: "CS_ERR_INVALID_ARG", 2: "CS_ERR_UNSUPPORTED", 3:
 EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_workspace_bytes",
                     "cs_verify_attention", "cs_spec_accept_workspace_bytes", "cs_spec_accept",
                     "cs_read_device_status", "cs_verify_attention_noalloc", "cs_sample_workspace_bytes",
-                    "cs_sample", "cs_kv_append", "cs_kv_commit")
+                    "cs_sample", "cs_kv_append", "cs_kv_commit", "cs_route_workspace_bytes",
+                    "cs_route_norms", "cs_route")
+
+
+class RouteDims(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("n_groups", ctypes.c_int32), ("dim", ctypes.c_int32)]
 
 
 class AttnDims(ctypes.Structure):
@@ -85,6 +90,12 @@ def load_library(path: str | None = None):
         lib.cs_kv_append.argtypes = [ctypes.POINTER(AttnDims), vp, vp, vp, vp, vp, vp, i32, vp]
         lib.cs_kv_commit.restype = ctypes.c_int
         lib.cs_kv_commit.argtypes = [i32, vp, vp, i32, vp]
+        lib.cs_route_workspace_bytes.restype = sz
+        lib.cs_route_workspace_bytes.argtypes = [ctypes.POINTER(RouteDims)]
+        lib.cs_route_norms.restype = ctypes.c_int
+        lib.cs_route_norms.argtypes = [i32, i32, vp, vp, vp]
+        lib.cs_route.restype = ctypes.c_int
+        lib.cs_route.argtypes = [ctypes.POINTER(RouteDims), vp, vp, vp, ctypes.c_float, vp, vp, vp, vp, sz, vp]
         lib.cs_sample_workspace_bytes.restype = sz
         lib.cs_sample_workspace_bytes.argtypes = [ctypes.POINTER(AcceptDims)]
         lib.cs_sample.restype = ctypes.c_int
@@ -256,6 +267,51 @@ def cs_kv_commit(ctx_lens, n_accepted, n_draft: int, stream: int | None = None):
     st = lib.cs_kv_commit(int(ctx_lens.shape[0]), _ptr(ctx_lens), _ptr(n_accepted), int(n_draft),
                           _stream(dev) if stream is None else stream)
     _check(lib, st)
+
+
+def cs_route_norms(centroids, inv_norms=None, stream: int | None = None):
+    """Inverse L2 norms of the group centroids (bf16 [N, d]); returns fp32 [N]."""
+    lib = load_library()
+    dev = centroids.device
+    _need(centroids, "centroids", torch.bfloat16, 2, dev)
+    N, d = centroids.shape
+    if inv_norms is None:
+        inv_norms = torch.empty((N,), dtype=torch.float32, device=dev)
+    _need(inv_norms, "inv_norms", torch.float32, 1, dev)
+    st = lib.cs_route_norms(int(N), int(d), _ptr(centroids) if N else None, _ptr(inv_norms) if N else None,
+                            _stream(dev) if stream is None else stream)
+    _check(lib, st)
+    return inv_norms
+
+
+def cs_route(emb, centroids, inv_norms, tau, out_group=None, out_best=None, out_score=None, workspace=None,
+             stream: int | None = None):
+    """Batched semantic routing; returns (group [B], best [B], score [B]).  See include/cachespec.h."""
+    lib = load_library()
+    dev = emb.device
+    _need(emb, "emb", torch.bfloat16, 2, dev)
+    _need(centroids, "centroids", torch.bfloat16, 2, dev)
+    _need(inv_norms, "inv_norms", torch.float32, 1, dev)
+    B, d = emb.shape
+    N = centroids.shape[0]
+    if N and centroids.shape[1] != d:
+        raise ValueError("emb and centroids differ in width")
+    out_group = torch.empty((B,), dtype=torch.int32, device=dev) if out_group is None else out_group
+    out_best = torch.empty((B,), dtype=torch.int32, device=dev) if out_best is None else out_best
+    out_score = torch.empty((B,), dtype=torch.float32, device=dev) if out_score is None else out_score
+    dims = RouteDims(B, N, d)
+    if workspace is None:
+        n = lib.cs_route_workspace_bytes(ctypes.byref(dims))
+        key = ("route", str(dev), n)
+        workspace = _workspaces.get(key)
+        if workspace is None:
+            workspace = torch.zeros(max(n, 256), dtype=torch.uint8, device=dev)
+            _workspaces[key] = workspace
+    st = lib.cs_route(ctypes.byref(dims), _ptr(emb), _ptr(centroids) if N else None, _ptr(inv_norms) if N else None,
+                      float(tau), _ptr(out_group), _ptr(out_best), _ptr(out_score), _ptr(workspace),
+                      workspace.numel() * workspace.element_size(), _stream(dev) if stream is None else stream)
+    _check(lib, st)
+    return out_group, out_best, out_score
 
 
 def cs_sample(logits, uniforms, temperature, out_tokens=None, workspace=None,

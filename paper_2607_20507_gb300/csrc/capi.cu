@@ -63,6 +63,15 @@ cs_status check_accept(const cs_accept_dims* d, int32_t n_draft, float temperatu
         return fail(CS_ERR_UNSUPPORTED, "vocab %d (this build implements up to %d)", d->vocab, CS_MAX_VOCAB);
     return CS_OK;
 }
+cs_status check_route(const cs_route_dims* d) {
+    if (!d) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
+    if (d->batch < 0 || d->n_groups < 0) return fail(CS_ERR_INVALID_ARG, "batch and n_groups must be >= 0");
+    if (d->dim <= 0 || d->dim % 64 != 0 || d->dim > CS_MAX_ROUTE_DIM)
+        return fail(CS_ERR_UNSUPPORTED, "dim %d (supported: multiples of 64 up to %d)", d->dim, CS_MAX_ROUTE_DIM);
+    if ((d->batch + 127) / 128 > 65535) return fail(CS_ERR_UNSUPPORTED, "batch %d too large for one call", d->batch);
+    return CS_OK;
+}
+
 cs_status check_sample(const cs_accept_dims* d, float temperature) {
     if (!d) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
     if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
@@ -206,6 +215,46 @@ cs_status cs_kv_commit(int32_t batch, int32_t* ctx_lens, const int32_t* n_accept
     if (!aligned(ctx_lens, 4) || !aligned(n_accepted, 4))
         return fail(CS_ERR_INVALID_ARG, "ctx_lens and n_accepted must be 4-byte aligned");
     return launch_kv_commit(ctx_lens, n_accepted, batch, n_draft, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t cs_route_workspace_bytes(const cs_route_dims* dims) {
+    if (check_route(dims) != CS_OK) return 0;
+    return plan_route(*dims, current_sm_count()).bytes;
+}
+
+cs_status cs_route_norms(int32_t n_groups, int32_t dim, const void* centroids, float* inv_norms,
+                         cs_stream_t stream) {
+    if (n_groups < 0) return fail(CS_ERR_INVALID_ARG, "n_groups %d < 0", n_groups);
+    if (dim <= 0 || dim % 64 != 0 || dim > CS_MAX_ROUTE_DIM)
+        return fail(CS_ERR_UNSUPPORTED, "dim %d (supported: multiples of 64 up to %d)", dim, CS_MAX_ROUTE_DIM);
+    if (n_groups == 0) return CS_OK;
+    if (!centroids || !inv_norms) return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (!aligned(centroids, 16) || !aligned(inv_norms, 4))
+        return fail(CS_ERR_INVALID_ARG, "centroids must be 16-byte and inv_norms 4-byte aligned");
+    return launch_route_norms(n_groups, dim, centroids, inv_norms, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cs_status cs_route(const cs_route_dims* dims, const void* emb, const void* centroids, const float* inv_norms,
+                   float tau, int32_t* out_group, int32_t* out_best, float* out_score, void* workspace,
+                   size_t workspace_bytes, cs_stream_t stream) {
+    cs_status st = check_route(dims);
+    if (st != CS_OK) return st;
+    if (isnan(tau) || isinf(tau)) return fail(CS_ERR_INVALID_ARG, "tau is not finite");
+    if (dims->batch == 0) return CS_OK;
+    if (!emb || !out_group || !out_best || !out_score) return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (dims->n_groups > 0 && (!centroids || !inv_norms))
+        return fail(CS_ERR_INVALID_ARG, "centroids and inv_norms are NULL with n_groups > 0");
+    if (!aligned(emb, 16) || (centroids && !aligned(centroids, 16)))
+        return fail(CS_ERR_INVALID_ARG, "emb and centroids must be 16-byte aligned");
+    if ((inv_norms && !aligned(inv_norms, 4)) || !aligned(out_group, 4) || !aligned(out_best, 4) ||
+        !aligned(out_score, 4))
+        return fail(CS_ERR_INVALID_ARG, "int32/fp32 pointers must be 4-byte aligned");
+    const RoutePlan pl = plan_route(*dims, current_sm_count());
+    if (!workspace || workspace_bytes < pl.bytes)
+        return fail(CS_ERR_WORKSPACE, "workspace of %zu bytes given, %zu needed", workspace_bytes, pl.bytes);
+    if (!aligned(workspace, 256)) return fail(CS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    return launch_route(*dims, pl, emb, centroids, inv_norms, tau, out_group, out_best, out_score, workspace,
+                        reinterpret_cast<cudaStream_t>(stream));
 }
 
 size_t cs_sample_workspace_bytes(const cs_accept_dims* dims) {

@@ -49,4 +49,16 @@ cs_status launch_kv_append(const cs_attn_dims& d, const void* new_k, const void*
 cs_status launch_kv_commit(int32_t* ctx_lens, const int32_t* n_accepted, int batch, int n_draft,
                            cudaStream_t stream);
 
+// -------------------------------------------------------------- routing
+constexpr int kMaxRouteDim = CS_MAX_ROUTE_DIM;
+struct RoutePlan {
+    int m_tiles, n_tiles, tiles_per_split, n_splits;
+    size_t bytes;   // workspace: status word (256 B), then [n_splits, B] partials
+};
+RoutePlan plan_route(const cs_route_dims& d, int sm_count);
+cs_status launch_route(const cs_route_dims& d, const RoutePlan& pl, const void* emb, const void* centroids,
+                       const float* inv_norms, float tau, int32_t* out_group, int32_t* out_best,
+                       float* out_score, void* workspace, cudaStream_t stream);
+cs_status launch_route_norms(int n_groups, int dim, const void* centroids, float* inv_norms, cudaStream_t stream);
+
 }  // namespace cs

@@ -268,3 +268,44 @@ def attention_subset(inp: dict, idx) -> dict:
 def accept_subset(inp: dict, idx) -> dict:
     idx = torch.as_tensor(list(idx), dtype=torch.int64, device=inp["target"].device)
     return {k: v[idx].contiguous() for k, v in inp.items()}
+
+
+# --------------------------------------------------------------------------
+# routing (the front end's semantic matching): synthetic embeddings
+# --------------------------------------------------------------------------
+ROUTE_TAU = 0.85   # the paper's semantic matching threshold
+
+
+@dataclasses.dataclass(frozen=True)
+class RouteWorkload:
+    wid: int
+    name: str
+    batch: int          # requests per routing call
+    n_groups: int       # existing request groups (centroids)
+    dim: int = 384      # all-MiniLM-L6-v2 embedding width
+    hit_fraction: float = 0.7
+
+
+ROUTE_WORKLOADS = {
+    1: RouteWorkload(1, "route-b64-g1000-d384", 64, 1000),
+    2: RouteWorkload(2, "route-b1024-g16384-d384", 1024, 16384),
+    3: RouteWorkload(3, "route-b4096-g100000-d384", 4096, 100000),
+}
+
+
+def route_inputs(w: RouteWorkload, device="cpu", seed: int | None = None) -> dict:
+    """Centroids with random directions and scales; a `hit_fraction` of the
+    requests are a centroid's direction plus isotropic noise of a spread that
+    puts their cosine with it around the 0.85 threshold (about 0.75-0.93),
+    the rest are random directions; request scales vary too.  bf16."""
+    g = torch.Generator().manual_seed(seed if seed is not None else 7_000_000 + 1000 * w.wid)
+    d, N, B = w.dim, w.n_groups, w.batch
+    cent = torch.randn(N, d, generator=g) * (0.5 + 1.5 * torch.rand(N, 1, generator=g))
+    hit = torch.rand(B, generator=g) < w.hit_fraction
+    pick = torch.randint(0, max(N, 1), (B,), generator=g)
+    sigma = 0.02 + 0.025 * torch.rand(B, 1, generator=g)
+    unit = cent / cent.norm(dim=1, keepdim=True).clamp_min(1e-30) if N else torch.zeros(1, d)
+    near = unit[pick] + sigma * torch.randn(B, d, generator=g)
+    far = torch.randn(B, d, generator=g) / math.sqrt(d)
+    emb = torch.where(hit[:, None], near, far) * (0.3 + 3.0 * torch.rand(B, 1, generator=g))
+    return dict(emb=emb.to(torch.bfloat16).to(device), centroids=cent.to(torch.bfloat16).to(device))

@@ -193,6 +193,37 @@ def test_kv_argument_checks(lib):
     assert lib.cs_kv_commit(0, None, None, 5, None) == binding.CS_OK
 
 
+def test_route_argument_checks(lib):
+    def route(dims, e=FAKE, c=FAKE, inv=FAKE, tau=0.85, g=FAKE, b=FAKE, s=FAKE, ws=FAKE, ws_bytes=1 << 40):
+        return lib.cs_route(ctypes.byref(dims), e, c, inv, tau, g, b, s, ws, ws_bytes, None)
+    d = binding.RouteDims(1024, 16384, 384)
+    for dim in (0, 100, 448, -64):
+        assert route(binding.RouteDims(4, 10, dim)) == binding.CS_ERR_UNSUPPORTED
+    assert route(binding.RouteDims(-1, 10, 64)) == binding.CS_ERR_INVALID_ARG
+    assert route(binding.RouteDims(4, -1, 64)) == binding.CS_ERR_INVALID_ARG
+    assert route(binding.RouteDims(128 * 65535 + 1, 10, 64)) == binding.CS_ERR_UNSUPPORTED
+    for tau in (float("nan"), float("inf"), -float("inf")):
+        assert route(d, tau=tau) == binding.CS_ERR_INVALID_ARG
+    for arg in ("e", "c", "inv", "g", "b", "s"):
+        assert route(d, **{arg: None}) == binding.CS_ERR_INVALID_ARG
+    assert route(d, e=FAKE + 8) == binding.CS_ERR_INVALID_ARG
+    assert route(d, c=FAKE + 2) == binding.CS_ERR_INVALID_ARG
+    assert route(d, s=FAKE + 1) == binding.CS_ERR_INVALID_ARG
+    need = lib.cs_route_workspace_bytes(ctypes.byref(d))
+    assert need >= 256 + 1024 * 8             # status word + at least one partial per request
+    assert lib.cs_route_workspace_bytes(ctypes.byref(binding.RouteDims(4, 10, 100))) == 0
+    assert route(d, ws=None) == binding.CS_ERR_WORKSPACE
+    assert route(d, ws_bytes=need - 1) == binding.CS_ERR_WORKSPACE
+    assert route(d, ws=FAKE + 64) == binding.CS_ERR_INVALID_ARG
+    assert route(binding.RouteDims(0, 10, 64), e=None, c=None, inv=None, g=None, b=None, s=None,
+                 ws=None) == binding.CS_OK
+    assert lib.cs_route_norms(5, 100, FAKE, FAKE, None) == binding.CS_ERR_UNSUPPORTED
+    assert lib.cs_route_norms(-1, 64, FAKE, FAKE, None) == binding.CS_ERR_INVALID_ARG
+    assert lib.cs_route_norms(5, 64, None, FAKE, None) == binding.CS_ERR_INVALID_ARG
+    assert lib.cs_route_norms(5, 64, FAKE + 8, FAKE, None) == binding.CS_ERR_INVALID_ARG
+    assert lib.cs_route_norms(0, 64, None, None, None) == binding.CS_OK
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     with pytest.raises(RuntimeError, match="not found"):
         binding.load_library(str(tmp_path / "missing.so"))
