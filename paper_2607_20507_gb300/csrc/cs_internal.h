@@ -52,8 +52,11 @@ cs_status launch_kv_commit(int32_t* ctx_lens, const int32_t* n_accepted, int bat
 // -------------------------------------------------------------- routing
 constexpr int kMaxRouteDim = CS_MAX_ROUTE_DIM;
 struct RoutePlan {
-    int m_tiles, n_tiles, tiles_per_split, n_splits;
-    size_t bytes;   // workspace: status word (256 B), then [n_splits, B] partials
+    int m_tiles, n_tiles;   // 128-request and 128-group tiles
+    long long items;        // m_tiles * n_tiles (request tile, group tile) pairs
+    int grid;               // persistent CTAs, each an equal contiguous item range
+    int seg_slots;          // partial slots per request tile
+    size_t bytes;           // workspace: status word (256 B), then [m_tiles, seg_slots, 128] partials
 };
 RoutePlan plan_route(const cs_route_dims& d, int sm_count);
 cs_status launch_route(const cs_route_dims& d, const RoutePlan& pl, const void* emb, const void* centroids,

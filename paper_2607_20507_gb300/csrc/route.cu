@@ -27,22 +27,39 @@
 namespace cs {
 namespace {
 
-constexpr int kRM = 128;                  // requests per CTA (MMA M)
+constexpr int kRM = 128;                  // requests per tile (MMA M)
 constexpr int kRN = 128;                  // groups per tile (MMA N)
 constexpr int kKC = 64;                   // dims per chunk: one 128-byte swizzle row
 constexpr int kChunkBytes = kRM * 128;    // 128 rows x 64 dims x 2 B
-constexpr int kMaxChunks = kMaxRouteDim / kKC;
-constexpr int kRSlots = 6;                // centroid-chunk ring
+constexpr int kMaxSlots = 12;             // centroid-chunk ring, at most
 constexpr int kRThreads = 256;            // warp 0 TMA, warp 1 MMA, warp 2 TMEM, warps 4-7 epilogue
 constexpr int kRTmemCols = 2 * kRN;
-constexpr int kRSmem = kMaxChunks * kChunkBytes + kRSlots * kChunkBytes + 256 /*barriers*/ + 1024;
+constexpr int kRBarBytes = 256;
+constexpr int kRStaticSmem = 2 * kRN * 4 + 64;   // inverse-norm double buffer, TMEM address
+constexpr int kRSmemLimit = 232448;              // opt-in shared memory per block on sm_103a
+
+__host__ __device__ constexpr int route_slots(int n_chunks) {
+    return (kRSmemLimit - kRStaticSmem - 1024 - kRBarBytes - n_chunks * kChunkBytes) / kChunkBytes < kMaxSlots
+               ? (kRSmemLimit - kRStaticSmem - 1024 - kRBarBytes - n_chunks * kChunkBytes) / kChunkBytes
+               : kMaxSlots;
+}
+__host__ __device__ constexpr int route_smem_bytes(int n_chunks) {
+    return 1024 + n_chunks * kChunkBytes + route_slots(n_chunks) * kChunkBytes + kRBarBytes;
+}
+static_assert(route_slots(kMaxRouteDim / kKC) >= 6, "ring too shallow for the widest embedding");
 
 struct RouteParams {
-    int B, N, d, n_chunks, n_tiles, tiles_per_split;
+    int B, N, d, n_chunks, n_tiles, slots, grid, seg_slots;
+    long long items;              // m_tiles * n_tiles work items, split evenly over the grid
     const float* inv_norm_c;      // [N]
-    float2* part;                 // [n_splits, B]: (max of dot * inv_norm_c, index as int bits)
+    float2* part;                 // [m_tiles, seg_slots, 128]: (max of dot * inv_norm_c, index as int bits)
     int* status;
 };
+
+// The CTA whose item range holds item x: ranges are [c*I/G, (c+1)*I/G).
+__host__ __device__ __forceinline__ int route_owner(long long x, long long items, int grid) {
+    return (int)(((x + 1) * grid + items - 1) / items) - 1;
+}
 
 __host__ __device__ constexpr uint32_t route_idesc() {
     // kind::f16: bf16 A and B (both K-major), fp32 D, M = 128, N = 128
@@ -63,33 +80,64 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
         : "memory");
 }
 
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(done)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return done != 0;
+}
+
+// Spins (no suspend) on the phase; about one second at most, then records
+// the timeout in the status word and returns false.
 __device__ __forceinline__ bool wait_bar(uint64_t* bar, uint32_t parity, int* status) {
-    if (mbar_wait_bounded(bar, parity)) return true;
+    if (mbar_test(bar, parity)) return true;
+    const uint64_t t0 = global_timer_ns();
+    for (uint32_t it = 0; it < (1u << 28); ++it) {
+        if (mbar_test(bar, parity)) return true;
+        if ((it & 1023u) == 1023u && global_timer_ns() - t0 > 1000000000ull) break;
+    }
     atomicOr(status, CS_DEVICE_WAIT_TIMEOUT);
     return false;
 }
 
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ void epi_bar_sync() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// Persistent: CTA c owns the work items [c*I/G, (c+1)*I/G) of the m-major
+// sequence (request tile m, group tile t).  The request tile stays resident
+// in shared memory while t advances and is reloaded when m changes.
 __global__ void __launch_bounds__(kRThreads, 1)
 route_gemm_kernel(const __grid_constant__ CUtensorMap tmap_e, const __grid_constant__ CUtensorMap tmap_c,
                   const RouteParams p) {
     extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sa = smem;                                   // [n_chunks][128 rows][128 B]
-    uint8_t* sb = smem + kMaxChunks * kChunkBytes;        // [kRSlots][128 groups][128 B]
-    uint64_t* bars = reinterpret_cast<uint64_t*>(sb + kRSlots * kChunkBytes);
-    uint64_t* a_full = bars;
-    uint64_t* full = bars + 1;               // [kRSlots]
-    uint64_t* empty = full + kRSlots;        // [kRSlots]
-    uint64_t* d_full = empty + kRSlots;      // [2]
-    uint64_t* d_free = d_full + 2;           // [2]
-    uint64_t* mma_done = d_free + 2;
+    __shared__ __align__(16) float s_inv[2 * kRN];
     __shared__ uint32_t s_tmem;
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int slots = p.slots;
+    uint8_t* sa = smem;                                   // [n_chunks][128 rows][128 B]
+    uint8_t* sb = smem + p.n_chunks * kChunkBytes;        // [slots][128 groups][128 B]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sb + slots * kChunkBytes);
+    uint64_t* a_full = bars;
+    uint64_t* a_free = bars + 1;
+    uint64_t* d_full = bars + 2;             // [2]
+    uint64_t* d_free = bars + 4;             // [2]
+    uint64_t* mma_done = bars + 6;
+    uint64_t* full = bars + 7;               // [slots]
+    uint64_t* empty = full + kMaxSlots;      // [slots]
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m = blockIdx.y;
-    const int t0 = blockIdx.x * p.tiles_per_split;
-    const int t1 = min(p.n_tiles, t0 + p.tiles_per_split);
-    const int nt = t1 - t0;
+    const long long it0 = (long long)blockIdx.x * p.items / p.grid;
+    const long long it1 = (long long)(blockIdx.x + 1) * p.items / p.grid;
+    const int nt = (int)(it1 - it0);
     if (warp == 2) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s_tmem)),
                      "n"(kRTmemCols)
@@ -98,15 +146,16 @@ route_gemm_kernel(const __grid_constant__ CUtensorMap tmap_e, const __grid_const
     }
     if (threadIdx.x == 0) {
         mbar_init(a_full, 1);
-        for (int i = 0; i < kRSlots; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&empty[i], 1);
-        }
+        mbar_init(a_free, 1);
         for (int i = 0; i < 2; ++i) {
             mbar_init(&d_full[i], 1);
             mbar_init(&d_free[i], 4);
         }
         mbar_init(mma_done, 1);
+        for (int i = 0; i < slots; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
         fence_barrier_init();
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -114,17 +163,23 @@ route_gemm_kernel(const __grid_constant__ CUtensorMap tmap_e, const __grid_const
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = s_tmem;
 
-    if (warp == 0 && lane == 0 && nt > 0) {
+    if (warp == 0 && lane == 0) {
         // ---------------------------------------------------------- TMA
         tma_prefetch_desc(&tmap_e);
         tma_prefetch_desc(&tmap_c);
-        mbar_arrive_expect_tx(a_full, (uint32_t)(p.n_chunks * kChunkBytes));
-        for (int kc = 0; kc < p.n_chunks; ++kc)
-            tma_load_2d(smem_u32(sa + kc * kChunkBytes), &tmap_e, a_full, kc * kKC, m * kRM);
-        int s = 0;
-        uint32_t use = 0;
+        int s = 0, cur_m = -1;
+        uint32_t use = 0, a_loads = 0;
         bool ok = true;
-        for (int t = t0; t < t1 && ok; ++t) {
+        for (long long it = it0; it < it1 && ok; ++it) {
+            const int m = (int)(it / p.n_tiles), t = (int)(it - (long long)m * p.n_tiles);
+            if (m != cur_m) {
+                if (a_loads > 0 && !wait_bar(a_free, (a_loads - 1) & 1, p.status)) break;
+                mbar_arrive_expect_tx(a_full, (uint32_t)(p.n_chunks * kChunkBytes));
+                for (int kc = 0; kc < p.n_chunks; ++kc)
+                    tma_load_2d(smem_u32(sa + kc * kChunkBytes), &tmap_e, a_full, kc * kKC, m * kRM);
+                ++a_loads;
+                cur_m = m;
+            }
             for (int kc = 0; kc < p.n_chunks; ++kc) {
                 if (use > 0 && !wait_bar(&empty[s], (use - 1) & 1, p.status)) {
                     ok = false;
@@ -132,26 +187,35 @@ route_gemm_kernel(const __grid_constant__ CUtensorMap tmap_e, const __grid_const
                 }
                 mbar_arrive_expect_tx(&full[s], (uint32_t)kChunkBytes);
                 tma_load_2d(smem_u32(sb + s * kChunkBytes), &tmap_c, &full[s], kc * kKC, t * kRN);
-                if (++s == kRSlots) {
+                if (++s == slots) {
                     s = 0;
                     ++use;
                 }
             }
         }
-        // no copy in flight at exit: the last fill of every slot has landed
-        const int total = nt * p.n_chunks;
-        for (int f = total - kRSlots > 0 ? total - kRSlots : 0; f < total; ++f)
-            if (!mbar_wait_bounded(&full[f % kRSlots], (uint32_t)(f / kRSlots) & 1)) atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-        if (!mbar_wait_bounded(a_full, 0)) atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-    } else if (warp == 1 && lane == 0 && nt > 0) {
+        // no copy in flight at exit: the last fill of every slot and the last
+        // request tile have landed
+        const long long total = (long long)nt * p.n_chunks;
+        for (long long f = total > slots ? total - slots : 0; f < total; ++f)
+            if (!mbar_wait_bounded(&full[f % slots], (uint32_t)(f / slots) & 1))
+                atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+        if (a_loads > 0 && !mbar_wait_bounded(a_full, (a_loads - 1) & 1)) atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+    } else if (warp == 1 && lane == 0) {
         // ---------------------------------------------------------- MMA
-        bool ok = wait_bar(a_full, 0, p.status);
-        int s = 0;
-        uint32_t use = 0;
+        int s = 0, cur_m = -1;
+        uint32_t use = 0, a_loads = 0;
+        bool ok = true;
         for (int tl = 0; tl < nt && ok; ++tl) {
+            const int m = (int)((it0 + tl) / p.n_tiles);
+            if (m != cur_m) {
+                if (a_loads > 0) umma_commit(a_free);   // the previous request tile may be overwritten
+                if (!wait_bar(a_full, a_loads & 1, p.status)) break;
+                ++a_loads;
+                cur_m = m;
+            }
             const int db = tl & 1;
             if (tl >= 2 && !wait_bar(&d_free[db], (uint32_t)((tl >> 1) - 1) & 1, p.status)) break;
-            for (int kc = 0; kc < p.n_chunks && ok; ++kc) {
+            for (int kc = 0; kc < p.n_chunks; ++kc) {
                 if (!wait_bar(&full[s], use & 1, p.status)) {
                     ok = false;
                     break;
@@ -167,36 +231,60 @@ route_gemm_kernel(const __grid_constant__ CUtensorMap tmap_e, const __grid_const
                         "l"(sw128_desc(a0 + ks * 32)), "l"(sw128_desc(b0 + ks * 32)), "r"(route_idesc()), "r"(acc)
                         : "memory");
                 }
-                asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                                 smem_u32(&empty[s]))
-                             : "memory");
-                if (++s == kRSlots) {
+                umma_commit(&empty[s]);
+                if (++s == slots) {
                     s = 0;
                     ++use;
                 }
             }
-            asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                             smem_u32(&d_full[db]))
-                         : "memory");
+            if (ok) umma_commit(&d_full[db]);
         }
-        asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                         smem_u32(mma_done))
-                     : "memory");
+        umma_commit(mma_done);
         if (!mbar_wait_bounded(mma_done, 0)) atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-    } else if (warp >= 4 && nt > 0) {
+    } else if (warp >= 4) {
         // ------------------------------------------------------ epilogue
         const int sub = warp & 3;
         const int row = sub * 32 + lane;
         const uint32_t t_lane = tmem + ((uint32_t)(sub * 32) << 16);
+        const float kNaN = __int_as_float(0x7fffffff);   // excluded by fmaxf and by ==
+        auto inv_of = [&](long long it) {
+            const int t = (int)(it % p.n_tiles);
+            const int j = t * kRN + row;
+            return j < p.N ? __ldg(p.inv_norm_c + j) : kNaN;
+        };
+        auto flush = [&](int m, float best, int idx) {
+            const int b = m * kRM + row;
+            if (b < p.B) {
+                const int slot = blockIdx.x - route_owner((long long)m * p.n_tiles, p.items, p.grid);
+                p.part[((size_t)m * p.seg_slots + slot) * kRM + row] = make_float2(best, __int_as_float(idx));
+            }
+        };
+        float inv_next = nt > 0 ? inv_of(it0) : 0.f;
         float best = kNegInf;
-        int idx = -1;
+        int idx = -1, cur_m = nt > 0 ? (int)(it0 / p.n_tiles) : -1;
+        bool dead = false;
         for (int tl = 0; tl < nt; ++tl) {
-            const int db = tl & 1, t = t0 + tl;
+            const long long it = it0 + tl;
+            const int m = (int)(it / p.n_tiles), t = (int)(it - (long long)m * p.n_tiles);
+            if (m != cur_m) {
+                flush(cur_m, best, idx);
+                best = kNegInf;
+                idx = -1;
+                cur_m = m;
+            }
+            const int db = tl & 1;
+            s_inv[db * kRN + row] = inv_next;
+            epi_bar_sync();
+            if (tl + 1 < nt) inv_next = inv_of(it + 1);
+            // after a timed-out wait the warp keeps taking part in the named
+            // barrier (every epilogue warp passes it nt times) but skips the rest
             int ok = 0;
-            if (lane == 0) ok = wait_bar(&d_full[db], (uint32_t)(tl >> 1) & 1, p.status) ? 1 : 0;
+            if (lane == 0 && !dead) ok = wait_bar(&d_full[db], (uint32_t)(tl >> 1) & 1, p.status) ? 1 : 0;
             ok = __shfl_sync(0xffffffffu, ok, 0);
-            __syncwarp();
-            if (!ok) break;
+            if (!ok) {
+                dead = true;
+                continue;
+            }
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 #pragma unroll 1
             for (int c0 = 0; c0 < kRN; c0 += 32) {
@@ -211,25 +299,34 @@ route_gemm_kernel(const __grid_constant__ CUtensorMap tmap_e, const __grid_const
                       "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
                     : "r"(t_lane + db * kRN + c0));
                 asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-                const int j0 = t * kRN + c0;
+                const float4* sv = reinterpret_cast<const float4*>(s_inv + db * kRN + c0);
+                float sc[32];
+                float mx = kNegInf;
 #pragma unroll
-                for (int e = 0; e < 32; ++e) {
-                    // ascending group ids: strict > keeps the lowest id of the maximum
-                    if (j0 + e < p.N) {
-                        const float sc = __uint_as_float(r[e]) * __ldg(p.inv_norm_c + j0 + e);
-                        if (sc > best) {
-                            best = sc;
-                            idx = j0 + e;
-                        }
-                    }
+                for (int q4 = 0; q4 < 8; ++q4) {
+                    const float4 v = sv[q4];
+                    sc[4 * q4 + 0] = __uint_as_float(r[4 * q4 + 0]) * v.x;
+                    sc[4 * q4 + 1] = __uint_as_float(r[4 * q4 + 1]) * v.y;
+                    sc[4 * q4 + 2] = __uint_as_float(r[4 * q4 + 2]) * v.z;
+                    sc[4 * q4 + 3] = __uint_as_float(r[4 * q4 + 3]) * v.w;
+                    mx = fmaxf(mx, fmaxf(fmaxf(sc[4 * q4], sc[4 * q4 + 1]), fmaxf(sc[4 * q4 + 2], sc[4 * q4 + 3])));
+                }
+                // ascending group ids and a strict > across chunks keep the
+                // lowest id of the maximum; inside the chunk, its first hit
+                if (mx > best) {
+                    int e0 = 31;
+#pragma unroll
+                    for (int e = 31; e >= 0; --e)
+                        if (sc[e] == mx) e0 = e;
+                    best = mx;
+                    idx = t * kRN + c0 + e0;
                 }
             }
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             __syncwarp();
             if (lane == 0) mbar_arrive(&d_free[db]);
         }
-        const int b = m * kRM + row;
-        if (b < p.B) p.part[(size_t)blockIdx.x * p.B + b] = make_float2(best, __int_as_float(idx));
+        if (cur_m >= 0) flush(cur_m, best, idx);
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
@@ -238,11 +335,13 @@ route_gemm_kernel(const __grid_constant__ CUtensorMap tmap_e, const __grid_const
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(kRTmemCols) : "memory");
 }
 
-// One warp per request: fold the splits (higher score, then lower index),
-// scale by the request's own inverse norm, apply the threshold.
-__global__ void __launch_bounds__(256) route_merge_kernel(const __nv_bfloat16* emb, const float2* part, int n_splits,
-                                                           int B, int d, float tau, int32_t* out_group,
-                                                           int32_t* out_best, float* out_score) {
+// One warp per request: fold the partials of the CTAs that covered its
+// request tile (higher score, then lower index), scale by the request's own
+// inverse norm, apply the threshold.
+__global__ void __launch_bounds__(256) route_merge_kernel(const __nv_bfloat16* emb, const float2* part, int B, int d,
+                                                           int n_tiles, long long items, int grid, int seg_slots,
+                                                           float tau, int32_t* out_group, int32_t* out_best,
+                                                           float* out_score) {
     const int b = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
     if (b >= B) return;
     float ss = 0.f;
@@ -254,12 +353,17 @@ __global__ void __launch_bounds__(256) route_merge_kernel(const __nv_bfloat16* e
     for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
     float best = kNegInf;
     int idx = -1;
-    for (int sp = lane; sp < n_splits; sp += 32) {
-        const float2 v = part[(size_t)sp * B + b];
-        const int vi = __float_as_int(v.y);
-        if (vi >= 0 && (v.x > best || (v.x == best && vi < idx) || idx < 0)) {
-            best = v.x;
-            idx = vi;
+    if (n_tiles > 0) {
+        const int m = b / kRM;
+        const int n_seg = route_owner((long long)(m + 1) * n_tiles - 1, items, grid) -
+                          route_owner((long long)m * n_tiles, items, grid) + 1;
+        for (int j = lane; j < n_seg; j += 32) {
+            const float2 v = part[((size_t)m * seg_slots + j) * kRM + (b % kRM)];
+            const int vi = __float_as_int(v.y);
+            if (vi >= 0 && (idx < 0 || v.x > best || (v.x == best && vi < idx))) {
+                best = v.x;
+                idx = vi;
+            }
         }
     }
 #pragma unroll
@@ -328,12 +432,13 @@ RoutePlan plan_route(const cs_route_dims& d, int sm_count) {
     RoutePlan pl{};
     pl.m_tiles = (d.batch + kRM - 1) / kRM;
     pl.n_tiles = (d.n_groups + kRN - 1) / kRN;
-    int splits = pl.m_tiles > 0 ? (sm_count > 0 ? sm_count : 148) / pl.m_tiles : 1;
-    if (splits < 1) splits = 1;
-    if (splits > pl.n_tiles) splits = pl.n_tiles;
-    pl.tiles_per_split = splits > 0 ? (pl.n_tiles + splits - 1) / splits : 0;
-    pl.n_splits = pl.tiles_per_split > 0 ? (pl.n_tiles + pl.tiles_per_split - 1) / pl.tiles_per_split : 0;
-    pl.bytes = 256 + ((size_t)pl.n_splits * d.batch * sizeof(float2) + 255) / 256 * 256;
+    pl.items = (long long)pl.m_tiles * pl.n_tiles;
+    const int sms = sm_count > 0 ? sm_count : 148;
+    pl.grid = (int)(pl.items < sms ? pl.items : sms);
+    // CTAs covering one request tile: its n_tiles items meet at most
+    // floor((n_tiles - 1) * G / I) + 2 of the G ranges
+    pl.seg_slots = pl.items > 0 ? (int)(((long long)(pl.n_tiles - 1) * pl.grid) / pl.items) + 2 : 0;
+    pl.bytes = 256 + ((size_t)pl.m_tiles * pl.seg_slots * kRM * sizeof(float2) + 255) / 256 * 256;
     return pl;
 }
 
@@ -342,37 +447,42 @@ cs_status launch_route(const cs_route_dims& d, const RoutePlan& pl, const void* 
                        float* out_score, void* workspace, cudaStream_t stream) {
     uint8_t* ws = static_cast<uint8_t*>(workspace);
     cudaError_t e;
-    if (pl.n_splits > 0) {
+    if (pl.grid > 0) {
         CUtensorMap te, tc;
         cs_status st = encode_rows_map(&te, emb, d.batch, d.dim);
         if (st != CS_OK) return st;
         st = encode_rows_map(&tc, centroids, d.n_groups, d.dim);
         if (st != CS_OK) return st;
-        static bool attr_done[64] = {};
+        const int n_chunks = d.dim / kKC;
+        const int smem = route_smem_bytes(n_chunks);
+        static int attr_smem[64] = {};
         int dev = 0;
         cudaGetDevice(&dev);
-        if (dev < 0 || dev >= 64 || !attr_done[dev]) {
-            e = cudaFuncSetAttribute(route_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kRSmem);
+        if (dev < 0 || dev >= 64 || attr_smem[dev] < smem) {
+            e = cudaFuncSetAttribute(route_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
             if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(route_gemm_kernel)");
-            if (dev >= 0 && dev < 64) attr_done[dev] = true;
+            if (dev >= 0 && dev < 64) attr_smem[dev] = smem;
         }
         RouteParams p{};
         p.B = d.batch;
         p.N = d.n_groups;
         p.d = d.dim;
-        p.n_chunks = d.dim / kKC;
+        p.n_chunks = n_chunks;
         p.n_tiles = pl.n_tiles;
-        p.tiles_per_split = pl.tiles_per_split;
+        p.slots = route_slots(n_chunks);
+        p.grid = pl.grid;
+        p.seg_slots = pl.seg_slots;
+        p.items = pl.items;
         p.inv_norm_c = inv_norms;
         p.status = reinterpret_cast<int*>(ws);
         p.part = reinterpret_cast<float2*>(ws + 256);
-        route_gemm_kernel<<<dim3(pl.n_splits, pl.m_tiles), kRThreads, kRSmem, stream>>>(te, tc, p);
+        route_gemm_kernel<<<pl.grid, kRThreads, smem, stream>>>(te, tc, p);
         e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_fail(e, "route_gemm_kernel launch");
     }
     route_merge_kernel<<<(d.batch + 7) / 8, 256, 0, stream>>>(
-        static_cast<const __nv_bfloat16*>(emb), reinterpret_cast<const float2*>(ws + 256), pl.n_splits, d.batch,
-        d.dim, tau, out_group, out_best, out_score);
+        static_cast<const __nv_bfloat16*>(emb), reinterpret_cast<const float2*>(ws + 256), d.batch, d.dim,
+        pl.n_tiles, pl.items, pl.grid, pl.seg_slots, tau, out_group, out_best, out_score);
     e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "route_merge_kernel launch");
     return CS_OK;
