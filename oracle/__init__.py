@@ -67,6 +67,14 @@ def _load():
         lib.oracle_route.argtypes = [i32, i32, i32, vp, vp, f64, vp, vp, vp, vp, vp]
         lib.oracle_sample.restype = ctypes.c_int
         lib.oracle_sample.argtypes = [i32, i32, i32, vp, vp, f64, vp, vp]
+        lib.oracle_tree_attention.restype = ctypes.c_int
+        lib.oracle_tree_attention.argtypes = [i32] * 7 + [f64] + [vp] * 6 + [i32, vp]
+        lib.oracle_tree_accept.restype = ctypes.c_int
+        lib.oracle_tree_accept.argtypes = [i32, i32, i32, vp, vp, vp, vp, vp, i32, f64] + [vp] * 5
+        lib.oracle_tree_accept_f64u.restype = ctypes.c_int
+        lib.oracle_tree_accept_f64u.argtypes = [i32, i32, i32, vp, vp, vp, vp, vp, i32, f64] + [vp] * 5
+        lib.oracle_kv_commit_tree.restype = ctypes.c_int
+        lib.oracle_kv_commit_tree.argtypes = [i32] * 6 + [vp] * 6 + [i32]
         lib.oracle_max_threads.restype = ctypes.c_int
         lib.oracle_set_threads.argtypes = [ctypes.c_int]
         _lib = lib
@@ -255,3 +263,80 @@ def row_argmax(row):
     lib = _load()
     r, code = _logit_array(np.asarray(row).reshape(-1))
     return int(lib.oracle_row_argmax(_ptr(r), code, r.shape[0]))
+
+
+def tree_attention(q_bits, k_bits, v_bits, page_table, ctx_lens, parents, scale=0.0):
+    """fp64 token-tree verify attention.
+
+    q_bits [B, n, Hq, D] uint16 (bf16 bits), one query row per tree node;
+    parents [B, n] int32 (node 0 is the root; parents[c] in [0, c)).  The other
+    arguments as for ``verify_attention``.  Returns fp64 [B, n, Hq, D].
+    """
+    lib = _load()
+    q = np.ascontiguousarray(q_bits, dtype=np.uint16)
+    kp = np.ascontiguousarray(k_bits, dtype=np.uint16)
+    vp = np.ascontiguousarray(v_bits, dtype=np.uint16)
+    pt = np.ascontiguousarray(page_table, dtype=np.int32)
+    cl = np.ascontiguousarray(ctx_lens, dtype=np.int32)
+    B, n, Hq, D = q.shape
+    par = np.ascontiguousarray(parents, dtype=np.int32).reshape(B, n)
+    P, Hkv, ps, D2 = kp.shape
+    assert D2 == D and vp.shape == kp.shape and pt.shape[0] == B and cl.shape == (B,)
+    out = np.zeros((B, n, Hq, D), dtype=np.float64)
+    rc = lib.oracle_tree_attention(B, Hq, Hkv, D, ps, pt.shape[1], P, float(scale), _ptr(q), _ptr(kp),
+                                   _ptr(vp), _ptr(pt), _ptr(cl), _ptr(par), n, _ptr(out))
+    if rc != 0:
+        raise RuntimeError(f"oracle_tree_attention failed with status {rc}")
+    return out
+
+
+def tree_accept(target, draft, parents, node_tokens, uniforms, temperature):
+    """fp64 token-tree acceptance (multi-candidate speculative sampling).
+
+    target, draft [B, n, V] (float32 or uint16 bf16 bits; draft may be None when
+    temperature == 0); parents, node_tokens [B, n] int32; uniforms [B, n]
+    float32 (or float64 for the pins).  Returns dict(tokens [B, n], path [B, n],
+    n_accepted [B], margin [B], draw_margin [B]).
+    """
+    lib = _load()
+    t, code = _logit_array(target)
+    B, n, V = t.shape
+    d = None
+    if draft is not None:
+        d, code_d = _logit_array(draft)
+        assert code_d == code and d.shape == (B, n, V)
+    par = np.ascontiguousarray(parents, dtype=np.int32).reshape(B, n)
+    x = np.ascontiguousarray(node_tokens, dtype=np.int32).reshape(B, n)
+    u = np.asarray(uniforms)
+    if u.dtype == np.float64:
+        fn = lib.oracle_tree_accept_f64u
+        u = np.ascontiguousarray(u).reshape(B, n)
+    else:
+        fn = lib.oracle_tree_accept
+        u = np.ascontiguousarray(u, dtype=np.float32).reshape(B, n)
+    res = {"tokens": np.zeros((B, n), np.int32), "path": np.zeros((B, n), np.int32),
+           "n_accepted": np.zeros(B, np.int32), "margin": np.zeros(B), "draw_margin": np.zeros(B)}
+    rc = fn(B, V, code, _ptr(t), _ptr(d), _ptr(par), _ptr(x), _ptr(u), n, float(temperature),
+            _ptr(res["tokens"]), _ptr(res["path"]), _ptr(res["n_accepted"]), _ptr(res["margin"]),
+            _ptr(res["draw_margin"]))
+    if rc != 0:
+        raise RuntimeError(f"oracle_tree_accept failed with status {rc}")
+    return res
+
+
+def kv_commit_tree(k_pages, v_pages, page_table, ctx_lens, path, n_accepted, n_nodes):
+    """Moves the accepted path's K/V rows next to the root, in place on numpy uint16
+    pools; returns the new context lengths (a new int32 array)."""
+    lib = _load()
+    assert k_pages.dtype == np.uint16 and k_pages.flags.c_contiguous and v_pages.flags.c_contiguous
+    P, Hkv, ps, D = k_pages.shape
+    pt = np.ascontiguousarray(page_table, dtype=np.int32)
+    cl = np.array(ctx_lens, dtype=np.int32)
+    B = cl.shape[0]
+    pa = np.ascontiguousarray(path, dtype=np.int32).reshape(B, n_nodes)
+    na = np.ascontiguousarray(n_accepted, dtype=np.int32)
+    rc = lib.oracle_kv_commit_tree(B, Hkv, D, ps, pt.shape[1], P, _ptr(k_pages), _ptr(v_pages), _ptr(pt),
+                                   _ptr(cl), _ptr(pa), _ptr(na), int(n_nodes))
+    if rc != 0:
+        raise RuntimeError(f"oracle_kv_commit_tree failed with status {rc}")
+    return cl

@@ -35,6 +35,12 @@
  *      page_table[b][pos / ps]); after the acceptance step the context keeps
  *      L_b - k + a rows (the prefix, the verify input token and the a
  *      accepted drafts).
+ *   7. Token-tree verification (Sec. 2's multi-candidate variants): the
+ *      attention of section 1 with each node seeing the prefix and its own
+ *      ancestors; the walk that tests the children of each node in turn
+ *      against the running residual (multi-candidate speculative
+ *      sampling); the commit that moves the accepted path's K/V rows next
+ *      to the root.
  *
  * Every floating-point step is fp64; inputs (bf16 bit patterns or fp32) are
  * widened exactly.  Loops run in the order the definition states (ascending
@@ -542,5 +548,323 @@ int oracle_route(int32_t batch, int32_t n_groups, int32_t dim, const uint16_t* e
         if (out_tau_margin) out_tau_margin[b] = fabs(best - tau);
     }
     free(cn);
+    return ORC_OK;
+}
+
+/* ------------------------------------------------------------------------
+ * 7. Token-tree verification (the multi-candidate variant of the
+ *    draft-and-verify step that the paper cites among the SpecDec variants
+ *    in Sec. 2: a tree of drafted candidates verified in one target pass,
+ *    then a walk that keeps one root-to-node path).
+ *
+ * A request's tree has n nodes in topological order.  Node 0 is the root,
+ * the last committed token, which is not verified; node c >= 1 holds the
+ * drafted token tokens[c] and its parent parents[c], which must lie in
+ * [0, c) -- a node whose parent does not is detached: it is never reached
+ * by the walk and its ancestry stops at itself.  anc(c) = {c} plus anc of
+ * its parent.  The K/V rows of node m sit at key position L_b - n + m.
+ *
+ * Attention: node i of request b, query head h, sees every prefix key
+ * j < L_b - n and the tree keys L_b - n + m for m in anc(i); the same
+ * softmax(q.K*scale).V as section 1 over that key set, in ascending key
+ * order.  Keys at negative positions (L_b < n) do not exist.  A node that
+ * sees no key outputs zeros.
+ *
+ * Acceptance (T > 0): the walk starts at the root with the target
+ * distribution p_u = softmax(z_t,u / T) of the current node u as its
+ * running distribution r.  The children of u (the nodes whose parent is u,
+ * ascending index) are tested in turn against the draft distribution
+ * q_u = softmax(z_d,u / T) that drafted them: child c with token x is
+ * accepted iff u_{c-1} < r(x) / q_u(x) (+inf when q_u(x) == 0, 0 when x is
+ * not a token id).  A rejection replaces r by max(0, r - q_u) normalised and
+ * the next sibling is tested against it; if that residual has no positive
+ * mass (r == q_u up to rounding) the remaining siblings are skipped and r
+ * falls back to p_u.  An accepted child is emitted and becomes u; when no
+ * child is accepted (or u is a leaf) one token is drawn from r by the
+ * inverse CDF of section 2 at u_{n-1}, and the step ends.  When every
+ * node's children are independent draws from that node's q_u, the emitted
+ * tokens follow the target's law exactly (each test is one speculative
+ * sampling step whose fallback is again such a step).  A chain
+ * (parents[c] = c - 1) is exactly the rule of section 2 with k = n - 1.
+ * Greedy (T == 0): at node u, g = argmax z_t,u (lowest id on ties); the
+ * first child whose token equals g is accepted, else g is emitted.
+ *
+ * target [B, n, V], draft [B, n, V] (row u = the distribution node u's
+ * children were drafted from; rows of leaves are not read; draft may be
+ * NULL when T == 0), parents / tokens [B, n] int32, uniforms [B, n] fp64
+ * (u_{c-1} tests node c, u_{n-1} is the draw).  out_tokens [B, n]: the
+ * accepted tokens, the emitted token, then -1; out_path [B, n]: the
+ * accepted nodes in walk order, then -1; out_n [B]: accepted count.
+ * out_margin / out_draw_margin as in section 2 (over the tests performed).
+ * ---------------------------------------------------------------------- */
+static int tree_parent(const int32_t* par, int64_t c) {
+    if (c <= 0) return -1;
+    const int32_t p = par[c];
+    return (p >= 0 && p < c) ? p : -1;
+}
+
+int oracle_tree_attention(int32_t batch, int32_t n_q_heads, int32_t n_kv_heads,
+                          int32_t head_dim, int32_t page_size, int32_t max_pages_per_seq,
+                          int32_t num_pages, double scale, const uint16_t* q,
+                          const uint16_t* k_pages, const uint16_t* v_pages,
+                          const int32_t* page_table, const int32_t* ctx_lens,
+                          const int32_t* parents, int32_t n_nodes, double* out) {
+    if (batch < 0 || n_q_heads <= 0 || n_kv_heads <= 0 || head_dim <= 0 ||
+        page_size <= 0 || max_pages_per_seq <= 0 || num_pages < 0 || n_nodes < 1)
+        return ORC_BAD_ARG;
+    if (n_q_heads % n_kv_heads != 0) return ORC_BAD_ARG;
+    if (batch == 0) return ORC_OK;
+    const int64_t n = n_nodes, group = n_q_heads / n_kv_heads, D = head_dim, ps = page_size;
+    const int64_t l_cap = (int64_t)max_pages_per_seq * ps;
+    if (scale <= 0.0) scale = 1.0 / sqrt((double)head_dim);
+
+    int status = ORC_OK;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
+    for (int64_t b = 0; b < batch; ++b) {
+        for (int64_t h = 0; h < n_q_heads; ++h) {
+            int64_t L = ctx_lens[b];
+            if (L < 0) L = 0;
+            if (L > l_cap) L = l_cap;
+            const int64_t kvh = h / group;
+            const int32_t* par = parents + b * n;
+            int64_t* keys = (int64_t*)malloc((size_t)(L + 1) * sizeof(int64_t));
+            double* s = (double*)malloc((size_t)(L + 1) * sizeof(double));
+            char* in_anc = (char*)malloc((size_t)n);
+            double* o = (double*)malloc((size_t)D * sizeof(double));
+            if (!keys || !s || !in_anc || !o) {
+#pragma omp atomic write
+                status = ORC_NO_MEM;
+                free(keys);
+                free(s);
+                free(in_anc);
+                free(o);
+                continue;
+            }
+            for (int64_t i = 0; i < n; ++i) {
+                const uint16_t* qv = q + ((b * n + i) * n_q_heads + h) * D;
+                double* dst = out + ((b * n + i) * n_q_heads + h) * D;
+                /* the key set of node i, ascending */
+                for (int64_t m = 0; m < n; ++m) in_anc[m] = 0;
+                for (int64_t m = i; m >= 0; m = tree_parent(par, m)) in_anc[m] = 1;
+                int64_t nk = 0;
+                for (int64_t j = 0; j < L; ++j) {
+                    const int64_t m = j - (L - n);
+                    if (m < 0 || in_anc[m]) keys[nk++] = j;
+                }
+                if (nk == 0) {
+                    for (int64_t d = 0; d < D; ++d) dst[d] = 0.0;
+                    continue;
+                }
+                for (int64_t t = 0; t < nk; ++t) {
+                    const int64_t j = keys[t];
+                    const int64_t page = page_table[b * max_pages_per_seq + j / ps];
+                    double dot = 0.0;
+                    if (page >= 0 && page < num_pages) {
+                        const uint16_t* kr = k_pages + ((page * n_kv_heads + kvh) * ps + j % ps) * D;
+                        for (int64_t d = 0; d < D; ++d)
+                            dot += bf16_bits_to_double(qv[d]) * bf16_bits_to_double(kr[d]);
+                    }
+                    s[t] = scale * dot;
+                }
+                double m = s[0];
+                for (int64_t t = 1; t < nk; ++t)
+                    if (s[t] > m) m = s[t];
+                double l = 0.0;
+                for (int64_t t = 0; t < nk; ++t) {
+                    s[t] = exp(s[t] - m);
+                    l += s[t];
+                }
+                for (int64_t d = 0; d < D; ++d) o[d] = 0.0;
+                for (int64_t t = 0; t < nk; ++t) {
+                    const int64_t j = keys[t];
+                    const int64_t page = page_table[b * max_pages_per_seq + j / ps];
+                    if (page < 0 || page >= num_pages) continue;
+                    const uint16_t* vr = v_pages + ((page * n_kv_heads + kvh) * ps + j % ps) * D;
+                    for (int64_t d = 0; d < D; ++d) o[d] += s[t] * bf16_bits_to_double(vr[d]);
+                }
+                for (int64_t d = 0; d < D; ++d) dst[d] = o[d] / l;
+            }
+            free(keys);
+            free(s);
+            free(in_anc);
+            free(o);
+        }
+    }
+    return status;
+}
+
+int oracle_tree_accept_f64u(int32_t batch, int32_t vocab, int32_t dtype, const void* target,
+                            const void* draft, const int32_t* parents, const int32_t* tokens,
+                            const double* uniforms, int32_t n_nodes, double temperature,
+                            int32_t* out_tokens, int32_t* out_path, int32_t* out_n,
+                            double* out_margin, double* out_draw_margin) {
+    if (batch < 0 || vocab <= 0 || n_nodes < 1 || (dtype != 0 && dtype != 1)) return ORC_BAD_ARG;
+    if (!(temperature >= 0.0)) return ORC_BAD_ARG;
+    if (temperature > 0.0 && n_nodes > 1 && !draft) return ORC_BAD_ARG;
+    const int64_t n = n_nodes, V = vocab;
+    const size_t esz = dtype == 0 ? 4 : 2;
+    int status = ORC_OK;
+
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t b = 0; b < batch; ++b) {
+        const char* trow0 = (const char*)target + (size_t)(b * n * V) * esz;
+        const char* drow0 = draft ? (const char*)draft + (size_t)(b * n * V) * esz : NULL;
+        const int32_t* par = parents + b * n;
+        const int32_t* x = tokens + b * n;
+        const double* u = uniforms + b * n;
+        int32_t* out = out_tokens + b * n;
+        int32_t* path = out_path + b * n;
+        int64_t depth = 0, node = 0;
+        double margin = INFINITY, draw_margin = INFINITY;
+        int32_t emit = 0;
+
+        if (temperature == 0.0) {
+            for (;;) {
+                const int32_t g = oracle_row_argmax(trow0 + (size_t)(node * V) * esz, dtype, vocab);
+                int64_t next = -1;
+                for (int64_t c = node + 1; c < n; ++c)
+                    if (tree_parent(par, c) == node && x[c] == g) {
+                        next = c;
+                        break;
+                    }
+                if (next < 0) {
+                    emit = g;
+                    break;
+                }
+                out[depth] = x[next];
+                path[depth] = (int32_t)next;
+                ++depth;
+                node = next;
+            }
+        } else {
+            double* p = (double*)malloc((size_t)V * sizeof(double));
+            double* qd = (double*)malloc((size_t)V * sizeof(double));
+            double* r = (double*)malloc((size_t)V * sizeof(double));
+            if (!p || !qd || !r) {
+#pragma omp atomic write
+                status = ORC_NO_MEM;
+                free(p);
+                free(qd);
+                free(r);
+                continue;
+            }
+            for (;;) {
+                oracle_row_probs(trow0 + (size_t)(node * V) * esz, dtype, vocab, temperature, p);
+                for (int64_t v = 0; v < V; ++v) r[v] = p[v];
+                int have_q = 0;
+                int64_t next = -1;
+                for (int64_t c = node + 1; c < n; ++c) {
+                    if (tree_parent(par, c) != node) continue;
+                    if (!have_q) {
+                        oracle_row_probs(drow0 + (size_t)(node * V) * esz, dtype, vocab, temperature, qd);
+                        have_q = 1;
+                    }
+                    double ratio = 0.0;
+                    if (x[c] >= 0 && x[c] < vocab)
+                        ratio = qd[x[c]] > 0.0 ? r[x[c]] / qd[x[c]] : INFINITY;
+                    const double gap = fabs(u[c - 1] - ratio);
+                    if (gap < margin) margin = gap;
+                    if (u[c - 1] < ratio) {
+                        next = c;
+                        break;
+                    }
+                    /* rejected: the next sibling is tested against the residual */
+                    double Z = 0.0;
+                    for (int64_t v = 0; v < V; ++v) {
+                        const double d = r[v] - qd[v];
+                        r[v] = d > 0.0 ? d : 0.0;
+                        Z += r[v];
+                    }
+                    if (!(Z > 0.0)) {
+                        for (int64_t v = 0; v < V; ++v) r[v] = p[v];
+                        break;
+                    }
+                    for (int64_t v = 0; v < V; ++v) r[v] /= Z;
+                }
+                if (next < 0) {
+                    double Z = 0.0;
+                    for (int64_t v = 0; v < V; ++v) Z += r[v];
+                    emit = oracle_inverse_cdf(r, Z, vocab, u[n - 1], &draw_margin);
+                    break;
+                }
+                out[depth] = x[next];
+                path[depth] = (int32_t)next;
+                ++depth;
+                node = next;
+            }
+            free(p);
+            free(qd);
+            free(r);
+        }
+        out[depth] = emit;
+        for (int64_t i = depth + 1; i < n; ++i) out[i] = -1;
+        for (int64_t i = depth; i < n; ++i) path[i] = -1;
+        out_n[b] = (int32_t)depth;
+        if (out_margin) out_margin[b] = margin;
+        if (out_draw_margin) out_draw_margin[b] = draw_margin;
+    }
+    return status;
+}
+
+int oracle_tree_accept(int32_t batch, int32_t vocab, int32_t dtype, const void* target,
+                       const void* draft, const int32_t* parents, const int32_t* tokens,
+                       const float* uniforms, int32_t n_nodes, double temperature,
+                       int32_t* out_tokens, int32_t* out_path, int32_t* out_n,
+                       double* out_margin, double* out_draw_margin) {
+    if (batch < 0 || n_nodes < 1) return ORC_BAD_ARG;
+    const size_t cnt = (size_t)batch * (size_t)n_nodes;
+    double* u = (double*)malloc((cnt ? cnt : 1) * sizeof(double));
+    if (!u) return ORC_NO_MEM;
+    for (size_t i = 0; i < cnt; ++i) u[i] = (double)uniforms[i];
+    const int rc = oracle_tree_accept_f64u(batch, vocab, dtype, target, draft, parents, tokens, u,
+                                           n_nodes, temperature, out_tokens, out_path, out_n,
+                                           out_margin, out_draw_margin);
+    free(u);
+    return rc;
+}
+
+/* Commit of an accepted tree path: the K/V rows of the accepted nodes
+ * path[0..a) move, in walk order, to the key positions right after the
+ * root, L_b - n + 1 + i (node path[i] sat at L_b - n + path[i] >= that
+ * position, so an ascending copy never overwrites a row it still needs),
+ * and L_b becomes L_b - n + 1 + a.  Rows with a negative position or a
+ * page id outside [0, num_pages) are skipped, as in the append. */
+int oracle_kv_commit_tree(int32_t batch, int32_t n_kv_heads, int32_t head_dim, int32_t page_size,
+                          int32_t max_pages, int32_t num_pages, uint16_t* k_pages,
+                          uint16_t* v_pages, const int32_t* page_table, int32_t* ctx_lens,
+                          const int32_t* path, const int32_t* n_accepted, int32_t n_nodes) {
+    if (batch < 0 || n_kv_heads <= 0 || head_dim <= 0 || page_size <= 0 || max_pages <= 0 ||
+        num_pages <= 0 || n_nodes < 1)
+        return ORC_BAD_ARG;
+    const int64_t cap = (int64_t)max_pages * page_size;
+    for (int64_t b = 0; b < batch; ++b) {
+        int64_t L = ctx_lens[b];
+        if (L < 0) L = 0;
+        if (L > cap) L = cap;
+        int64_t a = n_accepted[b];
+        if (a < 0) a = 0;
+        if (a > n_nodes - 1) a = n_nodes - 1;
+        const int64_t base = L - n_nodes;
+        for (int64_t i = 0; i < a; ++i) {
+            const int64_t node = path[b * n_nodes + i];
+            if (node < 1 || node >= n_nodes) continue;
+            const int64_t src = base + node, dst = base + 1 + i;
+            if (src == dst || src < 0 || dst < 0) continue;
+            const int64_t ps_ = page_size;
+            const int64_t sp = page_table[b * max_pages + src / ps_];
+            const int64_t dp = page_table[b * max_pages + dst / ps_];
+            if (sp < 0 || sp >= num_pages || dp < 0 || dp >= num_pages) continue;
+            for (int64_t h = 0; h < n_kv_heads; ++h) {
+                const int64_t so = ((sp * n_kv_heads + h) * ps_ + src % ps_) * head_dim;
+                const int64_t d0 = ((dp * n_kv_heads + h) * ps_ + dst % ps_) * head_dim;
+                for (int64_t e = 0; e < head_dim; ++e) {
+                    k_pages[d0 + e] = k_pages[so + e];
+                    v_pages[d0 + e] = v_pages[so + e];
+                }
+            }
+        }
+        const int64_t nl = base + 1 + a;
+        ctx_lens[b] = (int32_t)(nl > 0 ? nl : 0);
+    }
     return ORC_OK;
 }
