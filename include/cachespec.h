@@ -23,7 +23,15 @@
  *                          the verify positions' K/V rows, then keep the
  *                          accepted prefix;
  *   cs_route            -- the front end's batched semantic routing: cosine
- *                          scores against group centroids, arg max, threshold.
+ *                          scores against group centroids, arg max, threshold;
+ *   cs_tree_verify_attention,
+ *   cs_tree_accept,
+ *   cs_kv_commit_tree   -- token-tree verification, the multi-candidate
+ *                          variant of the step among those Sec. 2 cites: a
+ *                          tree of drafted candidates is scored in one pass
+ *                          (each node sees the prefix and its ancestors), one
+ *                          root-to-node path is accepted, and its K/V rows
+ *                          are moved next to the root.
  *
  * Conventions for every entry point
  *   - All tensor arguments are DEVICE pointers owned by the caller, dense
@@ -314,6 +322,87 @@ size_t cs_sample_workspace_bytes(const cs_accept_dims* dims);
 cs_status cs_sample(const cs_accept_dims* dims, const void* logits, const float* uniforms,
                     float temperature, int32_t* out_tokens, void* workspace,
                     size_t workspace_bytes, cs_stream_t stream);
+
+/*
+ * Token-tree verification (the tree-structured, multi-candidate variants of
+ * speculative decoding that Sec. 2 cites beside the chain of Sec. 3.4).
+ *
+ * A request's tree has n nodes in topological order, described by
+ * parents int32 [B, n]: node 0 is the root (the last committed token; its
+ * entry is ignored), node c >= 1 is a drafted token whose parent must lie in
+ * [0, c).  A node whose parent does not is detached: it sees only the prefix
+ * and itself, and the walk never reaches it.  Node m's K/V rows sit at key
+ * position L_b - n + m (ctx_lens counts the n tree positions, as for the
+ * chain; cs_kv_append with n_new = n writes them).
+ *
+ * cs_tree_verify_attention: for every node i, query head h,
+ *     out[b,i,h,:] = softmax_j( sm_scale * q[b,i,h,:] . K_j ) V_j
+ * over the prefix keys j < L_b - n and the tree keys L_b - n + m for every
+ * ancestor m of i and i itself.  Arguments, layouts (q and out are
+ * [B, n, Hq, D]), workspace rules and defined behaviour as for
+ * cs_verify_attention, with n_nodes in [1, 64] in place of n_draft + 1.
+ * Trees with n * G > 144 query rows per KV head are processed as row blocks
+ * of at most 144 rows, each reading that head's keys again.
+ *
+ * cs_tree_accept: the walk of multi-candidate speculative sampling.  At the
+ * current node u (the root first) the running distribution r starts as
+ * p_u = softmax(target[b,u,:] / T); the children of u are tested in
+ * ascending index against q_u = softmax(draft[b,u,:] / T), the distribution
+ * they were drafted from: child c with token x is accepted iff
+ * u_{c-1} < r(x) / q_u(x); a rejection replaces r by max(0, r - q_u)
+ * normalised (if that has no positive mass the remaining children are
+ * skipped and r is p_u again).  An accepted child is emitted and becomes u;
+ * when no child is accepted (or u is a leaf) one token is drawn from r by
+ * the inverse CDF of cs_spec_accept at u_{n-1}, and the walk ends.  When the
+ * children of every node are independent draws from its q_u, the emitted
+ * tokens follow the target distribution.  A chain (parents[c] = c - 1) is
+ * the rule of cs_spec_accept with k = n - 1.  T == 0: at node u the first
+ * child whose token is argmax target[b,u,:] (lowest id on ties) is accepted,
+ * else that argmax is emitted.
+ *
+ *   target_logits  [B, n, V] fp32 or bf16; row u is node u's next-token
+ *                  distribution
+ *   draft_logits   [B, n, V] same dtype; row u is the distribution u's
+ *                  children were drafted from (rows of leaves are not read);
+ *                  may be NULL when temperature == 0
+ *   node_tokens    int32 [B, n]: the token of each node (entry 0 unused); an
+ *                  id outside [0, V) is never accepted
+ *   uniforms       fp32 [B, n] in [0, 1): u_{c-1} tests node c, u_{n-1} is
+ *                  the draw
+ *   out_tokens     int32 [B, n]: the accepted tokens in walk order, the
+ *                  emitted token, then -1
+ *   out_path       int32 [B, n]: the accepted nodes in walk order, then -1
+ *   out_n_accepted int32 [B]: the number of accepted nodes a
+ *   workspace      at least cs_tree_accept_workspace_bytes(dims, n) bytes,
+ *                  256-byte aligned, any initial contents; calls sharing one
+ *                  must be ordered.
+ * Logit conventions as for cs_spec_accept.
+ *
+ * cs_kv_commit_tree: after the walk, moves the K and V rows of the accepted
+ * nodes path[0..a) (out_path, out_n_accepted) to the positions right after
+ * the root, L_b - n + 1 + i, and sets ctx_lens[b] = L_b - n + 1 + a (L_b
+ * clamped to [0, max_pages_per_seq * ps], a to [0, n-1]).  Rows whose page
+ * id lies outside [0, num_pages) are not moved.  The emitted token has no
+ * row yet: it is the first input of the next step.
+ *
+ * Return CS_ERR_INVALID_ARG (null pointer, misalignment, bad dimension,
+ * n_nodes outside [1, 64], bad temperature), CS_ERR_UNSUPPORTED (as for the
+ * chain calls), CS_ERR_WORKSPACE or CS_ERR_CUDA.
+ */
+#define CS_MAX_TREE_NODES 64
+size_t cs_tree_verify_attention_workspace_bytes(const cs_attn_dims* dims, int32_t n_nodes);
+cs_status cs_tree_verify_attention(const cs_attn_dims* dims, const void* q, const void* k_pages,
+                                   const void* v_pages, const int32_t* page_table, const int32_t* ctx_lens,
+                                   const int32_t* parents, int32_t n_nodes, void* out, void* workspace,
+                                   size_t workspace_bytes, cs_stream_t stream);
+size_t cs_tree_accept_workspace_bytes(const cs_accept_dims* dims, int32_t n_nodes);
+cs_status cs_tree_accept(const cs_accept_dims* dims, const void* target_logits, const void* draft_logits,
+                         const int32_t* parents, const int32_t* node_tokens, const float* uniforms,
+                         int32_t n_nodes, float temperature, int32_t* out_tokens, int32_t* out_path,
+                         int32_t* out_n_accepted, void* workspace, size_t workspace_bytes, cs_stream_t stream);
+cs_status cs_kv_commit_tree(const cs_attn_dims* dims, void* k_pages, void* v_pages, const int32_t* page_table,
+                            int32_t* ctx_lens, const int32_t* path, const int32_t* n_accepted, int32_t n_nodes,
+                            cs_stream_t stream);
 
 /*
  * Device status word of a verify-attention workspace: 0 when every call that

@@ -24,7 +24,9 @@ EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_work
                     "cs_verify_attention", "cs_spec_accept_workspace_bytes", "cs_spec_accept",
                     "cs_read_device_status", "cs_verify_attention_noalloc", "cs_sample_workspace_bytes",
                     "cs_sample", "cs_kv_append", "cs_kv_commit", "cs_route_workspace_bytes",
-                    "cs_route_norms", "cs_route")
+                    "cs_route_norms", "cs_route", "cs_tree_verify_attention_workspace_bytes",
+                    "cs_tree_verify_attention", "cs_tree_accept_workspace_bytes", "cs_tree_accept",
+                    "cs_kv_commit_tree")
 
 
 class RouteDims(ctypes.Structure):
@@ -100,6 +102,18 @@ def load_library(path: str | None = None):
         lib.cs_sample_workspace_bytes.argtypes = [ctypes.POINTER(AcceptDims)]
         lib.cs_sample.restype = ctypes.c_int
         lib.cs_sample.argtypes = [ctypes.POINTER(AcceptDims), vp, vp, ctypes.c_float, vp, vp, sz, vp]
+        lib.cs_tree_verify_attention_workspace_bytes.restype = sz
+        lib.cs_tree_verify_attention_workspace_bytes.argtypes = [ctypes.POINTER(AttnDims), i32]
+        lib.cs_tree_verify_attention.restype = ctypes.c_int
+        lib.cs_tree_verify_attention.argtypes = [ctypes.POINTER(AttnDims), vp, vp, vp, vp, vp, vp, i32, vp,
+                                                 vp, sz, vp]
+        lib.cs_tree_accept_workspace_bytes.restype = sz
+        lib.cs_tree_accept_workspace_bytes.argtypes = [ctypes.POINTER(AcceptDims), i32]
+        lib.cs_tree_accept.restype = ctypes.c_int
+        lib.cs_tree_accept.argtypes = [ctypes.POINTER(AcceptDims), vp, vp, vp, vp, vp, i32, ctypes.c_float,
+                                       vp, vp, vp, vp, sz, vp]
+        lib.cs_kv_commit_tree.restype = ctypes.c_int
+        lib.cs_kv_commit_tree.argtypes = [ctypes.POINTER(AttnDims), vp, vp, vp, vp, vp, vp, i32, vp]
         if path is None:
             _lib = lib
         return lib
@@ -341,6 +355,105 @@ def cs_sample(logits, uniforms, temperature, out_tokens=None, workspace=None,
                        _stream(dev) if stream is None else stream)
     _check(lib, st)
     return out_tokens
+
+
+def _cached_workspace(kind: str, device, n: int) -> torch.Tensor:
+    key = (kind, str(device), n)
+    ws = _workspaces.get(key)
+    if ws is None:
+        ws = torch.zeros(max(n, 256), dtype=torch.uint8, device=device)
+        _workspaces[key] = ws
+    return ws
+
+
+def cs_tree_verify_attention(q, k_pages, v_pages, page_table, ctx_lens, parents, out=None, workspace=None,
+                             sm_scale: float = 0.0, stream: int | None = None):
+    """Token-tree verify attention; q / out bf16 [B, n, Hq, D], parents int32 [B, n].
+    Returns ``out``.  See include/cachespec.h."""
+    lib = load_library()
+    dev = q.device
+    _need(q, "q", torch.bfloat16, 4, dev)
+    _need(k_pages, "k_pages", torch.bfloat16, 4, dev)
+    _need(v_pages, "v_pages", torch.bfloat16, 4, dev)
+    _need(page_table, "page_table", torch.int32, 2, dev)
+    _need(ctx_lens, "ctx_lens", torch.int32, 1, dev)
+    _need(parents, "parents", torch.int32, 2, dev)
+    if v_pages.shape != k_pages.shape:
+        raise ValueError("k_pages and v_pages must have the same shape")
+    B, n = q.shape[0], q.shape[1]
+    if tuple(parents.shape) != (B, n):
+        raise ValueError(f"parents must be [{B}, {n}]")
+    d = attn_dims(q, k_pages, page_table, sm_scale)
+    if out is None:
+        out = torch.empty_like(q)
+    _need(out, "out", torch.bfloat16, 4, dev)
+    if workspace is None:
+        workspace = _cached_workspace("tree_attn", dev,
+                                      lib.cs_tree_verify_attention_workspace_bytes(ctypes.byref(d), int(n)))
+    st = lib.cs_tree_verify_attention(ctypes.byref(d), _ptr(q), _ptr(k_pages), _ptr(v_pages), _ptr(page_table),
+                                      _ptr(ctx_lens), _ptr(parents), int(n), _ptr(out), _ptr(workspace),
+                                      workspace.numel() * workspace.element_size(),
+                                      _stream(dev) if stream is None else stream)
+    _check(lib, st)
+    return out
+
+
+def cs_tree_accept(target_logits, draft_logits, parents, node_tokens, uniforms, temperature, out_tokens=None,
+                   out_path=None, out_n_accepted=None, workspace=None, stream: int | None = None):
+    """Token-tree acceptance walk; target / draft logits [B, n, V], parents / node_tokens int32 [B, n],
+    uniforms fp32 [B, n].  Returns (tokens [B, n], path [B, n], n_accepted [B]).  See include/cachespec.h."""
+    lib = load_library()
+    dev = target_logits.device
+    if target_logits.dtype not in (torch.float32, torch.bfloat16):
+        raise TypeError("logits must be float32 or bfloat16")
+    dtype = target_logits.dtype
+    _need(target_logits, "target_logits", dtype, 3, dev)
+    B, n, V = target_logits.shape
+    if draft_logits is not None:
+        _need(draft_logits, "draft_logits", dtype, 3, dev)
+        if tuple(draft_logits.shape) != (B, n, V):
+            raise ValueError(f"draft_logits must be [{B}, {n}, {V}]")
+    for name, t in (("parents", parents), ("node_tokens", node_tokens)):
+        _need(t, name, torch.int32, 2, dev)
+        if tuple(t.shape) != (B, n):
+            raise ValueError(f"{name} must be [{B}, {n}]")
+    _need(uniforms, "uniforms", torch.float32, 2, dev)
+    out_tokens = torch.empty((B, n), dtype=torch.int32, device=dev) if out_tokens is None else out_tokens
+    out_path = torch.empty((B, n), dtype=torch.int32, device=dev) if out_path is None else out_path
+    out_n_accepted = torch.empty((B,), dtype=torch.int32, device=dev) if out_n_accepted is None else out_n_accepted
+    _need(out_tokens, "out_tokens", torch.int32, 2, dev)
+    _need(out_path, "out_path", torch.int32, 2, dev)
+    _need(out_n_accepted, "out_n_accepted", torch.int32, 1, dev)
+    d = AcceptDims(B, V, CS_F32 if dtype == torch.float32 else CS_BF16)
+    if workspace is None:
+        workspace = _cached_workspace("tree_accept", dev, lib.cs_tree_accept_workspace_bytes(ctypes.byref(d), int(n)))
+    st = lib.cs_tree_accept(ctypes.byref(d), _ptr(target_logits), _ptr(draft_logits), _ptr(parents),
+                            _ptr(node_tokens), _ptr(uniforms), int(n), float(temperature), _ptr(out_tokens),
+                            _ptr(out_path), _ptr(out_n_accepted), _ptr(workspace),
+                            workspace.numel() * workspace.element_size(), _stream(dev) if stream is None else stream)
+    _check(lib, st)
+    return out_tokens, out_path, out_n_accepted
+
+
+def cs_kv_commit_tree(k_pages, v_pages, page_table, ctx_lens, path, n_accepted, stream: int | None = None):
+    """Move the accepted tree path's K/V rows next to the root and shorten ctx_lens (in place);
+    path int32 [B, n] and n_accepted [B] as returned by cs_tree_accept."""
+    lib = load_library()
+    dev = k_pages.device
+    _need(k_pages, "k_pages", torch.bfloat16, 4, dev)
+    _need(v_pages, "v_pages", torch.bfloat16, 4, dev)
+    _need(page_table, "page_table", torch.int32, 2, dev)
+    _need(ctx_lens, "ctx_lens", torch.int32, 1, dev)
+    _need(path, "path", torch.int32, 2, dev)
+    _need(n_accepted, "n_accepted", torch.int32, 1, dev)
+    if k_pages.shape != v_pages.shape:
+        raise ValueError("k_pages and v_pages must have the same shape")
+    P, Hkv, ps, D = k_pages.shape
+    B, n = path.shape
+    d = AttnDims(B, Hkv, Hkv, D, ps, page_table.shape[1], P, 0.0)
+    st = lib.cs_kv_commit_tree(ctypes.byref(d), _ptr(k_pages), _ptr(v_pages), _ptr(page_table), _ptr(ctx_lens),
+                               _ptr(path), _ptr(n_accepted), int(n), _stream(dev) if stream is None else stream)
+    _check(lib, st)
 
 
 def cs_verify_attention_noalloc(q, k_pages, v_pages, page_table, ctx_lens, n_draft, out=None,

@@ -21,7 +21,8 @@ bool pow2_page(int ps) {
     return ps == 8 || ps == 16 || ps == 32 || ps == 64 || ps == 128 || ps == 256;
 }
 
-cs_status check_attn(const cs_attn_dims* d, int32_t n_draft) {
+// Geometry checks shared by the chain and tree attention calls.
+cs_status check_attn_geometry(const cs_attn_dims* d) {
     if (!d) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
     if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
     if (d->n_q_heads <= 0 || d->n_kv_heads <= 0)
@@ -37,14 +38,42 @@ cs_status check_attn(const cs_attn_dims* d, int32_t n_draft) {
     if (d->num_pages <= 0) return fail(CS_ERR_INVALID_ARG, "num_pages %d <= 0", d->num_pages);
     if (isnan(d->sm_scale) || isinf(d->sm_scale))
         return fail(CS_ERR_INVALID_ARG, "sm_scale is not finite");
-    if (n_draft < 1 || n_draft > 16) return fail(CS_ERR_INVALID_ARG, "n_draft %d not in [1, 16]", n_draft);
     if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this build implements 128)", d->head_dim);
     if (!pow2_page(d->page_size))
         return fail(CS_ERR_UNSUPPORTED, "page_size %d (supported: 8..256, powers of two)", d->page_size);
-    const long long rows = (long long)(n_draft + 1) * (d->n_q_heads / d->n_kv_heads);
-    if (rows > 144) return fail(CS_ERR_UNSUPPORTED, "(k+1)*G = %lld query rows per KV head (max 144)", rows);
     if ((long long)d->max_pages_per_seq * d->page_size > (1LL << 30))
         return fail(CS_ERR_INVALID_ARG, "max_pages_per_seq * page_size exceeds 2^30 keys");
+    return CS_OK;
+}
+
+cs_status check_attn(const cs_attn_dims* d, int32_t n_draft) {
+    if (!d) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
+    if (n_draft < 1 || n_draft > 16) return fail(CS_ERR_INVALID_ARG, "n_draft %d not in [1, 16]", n_draft);
+    const cs_status st = check_attn_geometry(d);
+    if (st != CS_OK) return st;
+    const long long rows = (long long)(n_draft + 1) * (d->n_q_heads / d->n_kv_heads);
+    if (rows > 144) return fail(CS_ERR_UNSUPPORTED, "(k+1)*G = %lld query rows per KV head (max 144)", rows);
+    return CS_OK;
+}
+
+cs_status check_tree_attn(const cs_attn_dims* d, int32_t n_nodes) {
+    if (!d) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
+    if (n_nodes < 1 || n_nodes > CS_MAX_TREE_NODES)
+        return fail(CS_ERR_INVALID_ARG, "n_nodes %d not in [1, %d]", n_nodes, CS_MAX_TREE_NODES);
+    return check_attn_geometry(d);
+}
+
+// Pointer checks shared by the chain and tree attention calls.
+cs_status check_attn_pointers(const void* q, const void* k_pages, const void* v_pages, const int32_t* page_table,
+                              const int32_t* ctx_lens, const void* out) {
+    if (!q || !k_pages || !v_pages || !page_table || !ctx_lens || !out)
+        return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (!aligned(k_pages, 16) || !aligned(v_pages, 16))
+        return fail(CS_ERR_INVALID_ARG, "k_pages and v_pages must be 16-byte aligned");
+    if (!aligned(q, 4) || !aligned(out, 8))
+        return fail(CS_ERR_INVALID_ARG, "q must be 4-byte and out 8-byte aligned");
+    if (!aligned(page_table, 4) || !aligned(ctx_lens, 4))
+        return fail(CS_ERR_INVALID_ARG, "page_table and ctx_lens must be 4-byte aligned");
     return CS_OK;
 }
 
@@ -134,21 +163,98 @@ cs_status cs_verify_attention(const cs_attn_dims* dims, const void* q, const voi
     cs_status st = check_attn(dims, n_draft);
     if (st != CS_OK) return st;
     if (dims->batch == 0) return CS_OK;
-    if (!q || !k_pages || !v_pages || !page_table || !ctx_lens || !out)
-        return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
-    if (!aligned(k_pages, 16) || !aligned(v_pages, 16))
-        return fail(CS_ERR_INVALID_ARG, "k_pages and v_pages must be 16-byte aligned");
-    if (!aligned(q, 4) || !aligned(out, 8))
-        return fail(CS_ERR_INVALID_ARG, "q must be 4-byte and out 8-byte aligned");
-    if (!aligned(page_table, 4) || !aligned(ctx_lens, 4))
-        return fail(CS_ERR_INVALID_ARG, "page_table and ctx_lens must be 4-byte aligned");
+    st = check_attn_pointers(q, k_pages, v_pages, page_table, ctx_lens, out);
+    if (st != CS_OK) return st;
     const AttnPlan plan = plan_verify_attention(*dims, n_draft, current_sm_count());
     if (!workspace || workspace_bytes < plan.bytes)
         return fail(CS_ERR_WORKSPACE, "workspace of %zu bytes given, %zu needed", workspace_bytes,
                     plan.bytes);
     if (!aligned(workspace, 256)) return fail(CS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
-    return launch_verify_attention(*dims, plan, q, k_pages, v_pages, page_table, ctx_lens, out,
+    return launch_verify_attention(*dims, plan, q, k_pages, v_pages, page_table, ctx_lens, nullptr, out,
                                    workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t cs_tree_verify_attention_workspace_bytes(const cs_attn_dims* dims, int32_t n_nodes) {
+    if (check_tree_attn(dims, n_nodes) != CS_OK) return 0;
+    return plan_tree_attention(*dims, n_nodes, current_sm_count()).bytes;
+}
+
+cs_status cs_tree_verify_attention(const cs_attn_dims* dims, const void* q, const void* k_pages,
+                                   const void* v_pages, const int32_t* page_table, const int32_t* ctx_lens,
+                                   const int32_t* parents, int32_t n_nodes, void* out, void* workspace,
+                                   size_t workspace_bytes, cs_stream_t stream) {
+    cs_status st = check_tree_attn(dims, n_nodes);
+    if (st != CS_OK) return st;
+    if (dims->batch == 0) return CS_OK;
+    st = check_attn_pointers(q, k_pages, v_pages, page_table, ctx_lens, out);
+    if (st != CS_OK) return st;
+    if (!parents) return fail(CS_ERR_INVALID_ARG, "parents is NULL");
+    if (!aligned(parents, 4)) return fail(CS_ERR_INVALID_ARG, "parents must be 4-byte aligned");
+    const AttnPlan plan = plan_tree_attention(*dims, n_nodes, current_sm_count());
+    if (!workspace || workspace_bytes < plan.bytes)
+        return fail(CS_ERR_WORKSPACE, "workspace of %zu bytes given, %zu needed", workspace_bytes, plan.bytes);
+    if (!aligned(workspace, 256)) return fail(CS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    return launch_verify_attention(*dims, plan, q, k_pages, v_pages, page_table, ctx_lens, parents, out,
+                                   workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+size_t cs_tree_accept_workspace_bytes(const cs_accept_dims* dims, int32_t n_nodes) {
+    if (check_sample(dims, 1.0f) != CS_OK || n_nodes < 1 || n_nodes > CS_MAX_TREE_NODES) return 0;
+    return tree_accept_workspace_bytes(*dims, n_nodes);
+}
+
+cs_status cs_tree_accept(const cs_accept_dims* dims, const void* target_logits, const void* draft_logits,
+                         const int32_t* parents, const int32_t* node_tokens, const float* uniforms,
+                         int32_t n_nodes, float temperature, int32_t* out_tokens, int32_t* out_path,
+                         int32_t* out_n_accepted, void* workspace, size_t workspace_bytes, cs_stream_t stream) {
+    cs_status st = check_sample(dims, temperature);
+    if (st != CS_OK) return st;
+    if (n_nodes < 1 || n_nodes > CS_MAX_TREE_NODES)
+        return fail(CS_ERR_INVALID_ARG, "n_nodes %d not in [1, %d]", n_nodes, CS_MAX_TREE_NODES);
+    if ((long long)dims->batch * n_nodes * (long long)dims->vocab > (1LL << 46))
+        return fail(CS_ERR_INVALID_ARG, "logit tensor too large");
+    if (dims->batch == 0) return CS_OK;
+    if (!target_logits || !parents || !node_tokens || !uniforms || !out_tokens || !out_path || !out_n_accepted)
+        return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (temperature > 0.f && !draft_logits)
+        return fail(CS_ERR_INVALID_ARG, "draft_logits is NULL with temperature > 0");
+    const size_t esz = dims->logit_dtype == CS_F32 ? 4 : 2;
+    if (!aligned(target_logits, esz) || (draft_logits && !aligned(draft_logits, esz)))
+        return fail(CS_ERR_INVALID_ARG, "logit pointers must be aligned to their element size");
+    if (!aligned(parents, 4) || !aligned(node_tokens, 4) || !aligned(uniforms, 4) || !aligned(out_tokens, 4) ||
+        !aligned(out_path, 4) || !aligned(out_n_accepted, 4))
+        return fail(CS_ERR_INVALID_ARG, "int32/fp32 pointers must be 4-byte aligned");
+    const size_t need = tree_accept_workspace_bytes(*dims, n_nodes);
+    if (!workspace || workspace_bytes < need)
+        return fail(CS_ERR_WORKSPACE, "workspace of %zu bytes given, %zu needed", workspace_bytes, need);
+    if (!aligned(workspace, 256)) return fail(CS_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    return launch_tree_accept(*dims, target_logits, temperature > 0.f ? draft_logits : nullptr, parents, node_tokens,
+                              uniforms, n_nodes, temperature, out_tokens, out_path, out_n_accepted, workspace,
+                              reinterpret_cast<cudaStream_t>(stream));
+}
+
+cs_status cs_kv_commit_tree(const cs_attn_dims* dims, void* k_pages, void* v_pages, const int32_t* page_table,
+                            int32_t* ctx_lens, const int32_t* path, const int32_t* n_accepted, int32_t n_nodes,
+                            cs_stream_t stream) {
+    if (!dims) return fail(CS_ERR_INVALID_ARG, "dims is NULL");
+    const cs_attn_dims* d = dims;
+    if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
+    if (d->n_kv_heads <= 0 || d->page_size <= 0 || d->max_pages_per_seq <= 0 || d->num_pages <= 0)
+        return fail(CS_ERR_INVALID_ARG, "n_kv_heads, page_size, max_pages_per_seq and num_pages must be positive");
+    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this build implements 128)", d->head_dim);
+    if (n_nodes < 1 || n_nodes > CS_MAX_TREE_NODES)
+        return fail(CS_ERR_INVALID_ARG, "n_nodes %d not in [1, %d]", n_nodes, CS_MAX_TREE_NODES);
+    if ((long long)d->max_pages_per_seq * d->page_size > (1LL << 30))
+        return fail(CS_ERR_INVALID_ARG, "max_pages_per_seq * page_size exceeds 2^30 keys");
+    if (d->batch == 0) return CS_OK;
+    if (!k_pages || !v_pages || !page_table || !ctx_lens || !path || !n_accepted)
+        return fail(CS_ERR_INVALID_ARG, "a tensor pointer is NULL");
+    if (!aligned(k_pages, 16) || !aligned(v_pages, 16))
+        return fail(CS_ERR_INVALID_ARG, "page pools must be 16-byte aligned");
+    if (!aligned(page_table, 4) || !aligned(ctx_lens, 4) || !aligned(path, 4) || !aligned(n_accepted, 4))
+        return fail(CS_ERR_INVALID_ARG, "int32 pointers must be 4-byte aligned");
+    return launch_kv_commit_tree(*d, k_pages, v_pages, page_table, ctx_lens, path, n_accepted, n_nodes,
+                                 reinterpret_cast<cudaStream_t>(stream));
 }
 
 size_t cs_spec_accept_workspace_bytes(const cs_accept_dims* dims, int32_t n_draft) {

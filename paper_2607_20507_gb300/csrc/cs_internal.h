@@ -20,18 +20,25 @@ int current_sm_count();
 // ------------------------------------------------------------- attention
 struct AttnPlan {
     int group;        // G = Hq / Hkv
-    int rows;         // k + 1
-    int n_rows;       // (k+1) * G query rows per KV head
+    int rows;         // k + 1 (chain) or the tree's node count
+    bool tree;        // tree mask (parents given) instead of the causal chain
+    int n_rows_all;   // rows * G query rows per KV head
+    int n_rb;         // row blocks per KV head (each one span of the schedule)
+    int n_rows;       // query rows per row block (n_rows_all when n_rb == 1)
     int row_warps;    // ceil(n_rows / 16) consumer warps
     int grid;         // persistent CTAs (resident capacity of the device)
     size_t off_part_o, off_part_ml, bytes;   // workspace layout (status word at 0)
 };
 AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count);
+AttnPlan plan_tree_attention(const cs_attn_dims& d, int n_nodes, int sm_count);
 
+// parents: NULL for the causal chain, the [B, rows] parent array for a tree
+// (must match plan.tree)
 cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& plan, const void* q,
                                   const void* k_pages, const void* v_pages,
-                                  const int32_t* page_table, const int32_t* ctx_lens, void* out,
-                                  void* workspace, cudaStream_t stream);
+                                  const int32_t* page_table, const int32_t* ctx_lens,
+                                  const int32_t* parents, void* out, void* workspace,
+                                  cudaStream_t stream);
 
 // ------------------------------------------------------------ acceptance
 size_t accept_workspace_bytes(const cs_accept_dims& d, int n_draft, float temperature);
@@ -42,12 +49,23 @@ cs_status launch_spec_accept(const cs_accept_dims& d, const void* target, const 
                              float temperature, int32_t* out_tokens, int32_t* out_n,
                              void* workspace, cudaStream_t stream);
 
+// token trees: target and draft rows [B, n, V], parents / tokens /
+// uniforms [B, n]; outputs tokens and path [B, n], accepted count [B]
+size_t tree_accept_workspace_bytes(const cs_accept_dims& d, int n_nodes);
+cs_status launch_tree_accept(const cs_accept_dims& d, const void* target, const void* draft,
+                             const int32_t* parents, const int32_t* tokens, const float* uniforms, int n_nodes,
+                             float temperature, int32_t* out_tokens, int32_t* out_path, int32_t* out_n,
+                             void* workspace, cudaStream_t stream);
+
 // ------------------------------------------------------------- KV cache
 cs_status launch_kv_append(const cs_attn_dims& d, const void* new_k, const void* new_v, void* k_pages,
                            void* v_pages, const int32_t* page_table, const int32_t* ctx_lens, int n_new,
                            cudaStream_t stream);
 cs_status launch_kv_commit(int32_t* ctx_lens, const int32_t* n_accepted, int batch, int n_draft,
                            cudaStream_t stream);
+cs_status launch_kv_commit_tree(const cs_attn_dims& d, void* k_pages, void* v_pages, const int32_t* page_table,
+                                int32_t* ctx_lens, const int32_t* path, const int32_t* n_accepted, int n_nodes,
+                                cudaStream_t stream);
 
 // -------------------------------------------------------------- routing
 constexpr int kMaxRouteDim = CS_MAX_ROUTE_DIM;

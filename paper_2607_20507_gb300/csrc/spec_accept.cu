@@ -27,6 +27,14 @@
 //      finds the token within its slice.
 //   Greedy mode replaces kernel 2 by accept_greedy_kernel (one warp per
 //   request: argmax agreement).
+// Token trees (multi-candidate verification) reuse kernel 1 over the target
+// rows of every node and the draft rows of the nodes that have children
+// (a leaf's draft row is not read), and walk the tree in tree_draw_kernel
+// (one cluster per request): the children of the current node are tested in
+// turn, each rejection turning the running distribution into the residual
+// max(p - kappa q, 0) / Z, whose mass Z takes one cluster-wide pass over the
+// row pair; the walk ends with the draw of section 2 at that kappa.  The
+// greedy walk is tree_greedy_kernel.
 // No probability is written to memory; the scratch holds the row-segment
 // pairs and one count per row.
 #include <limits.h>
@@ -49,16 +57,20 @@ constexpr int kMaxRows = 33;                   // 2k+1 rows of a request, k <= 1
 constexpr int kRowsPerDrawWarp = (kMaxRows + kDrawWarps - 1) / kDrawWarps;
 constexpr int kMaxPasses = 128;                // passes of one CTA over its vocabulary slice
 constexpr int kMaxCluster = 16;
+constexpr int kMaxTreeNodes = 64;
 
 struct AcceptParams {
-    const void* target;       // [B, k+1, V]
-    const void* draft;        // [B, k, V]
-    const int32_t* tokens;    // [B, k]
-    const float* uniforms;    // [B, k+1]
-    int32_t* out_tokens;      // [B, k+1]
+    const void* target;       // [B, n_t, V]: chain n_t = k+1, tree n_t = nodes
+    const void* draft;        // [B, d_rows, V]: chain d_rows = k, tree d_rows = nodes
+    const int32_t* tokens;    // chain [B, k]; tree [B, n_t] (node tokens)
+    const float* uniforms;    // chain [B, k+1]; tree [B, n_t]
+    int32_t* out_tokens;      // chain [B, k+1]; tree [B, n_t]
     int32_t* out_n;           // [B], or null (the sampler)
+    const int32_t* parents;   // tree [B, n_t] (null for the chain)
+    int32_t* out_path;        // tree [B, n_t]: accepted nodes in walk order
     int B, V, k;
-    int R;                    // rows per request: 2k+1 (sampling) or k+1 (greedy)
+    int n_t, d_rows;          // target rows and draft rows per request
+    int R;                    // rows per request streamed by kernel 1: n_t + d_rows, or n_t (greedy)
     int I;                    // 4 KB items per row
     long long N;              // B * R * I items in all
     int W;                    // busy warps of kernel 1 (warp w owns items [w*N/W, (w+1)*N/W)), W <= N
@@ -165,11 +177,29 @@ __device__ __forceinline__ float2 warp_fold_argmax(float2 acc) {
     return acc;
 }
 
+// Row r of request b: target rows 0 .. n_t-1, then draft rows.
 template <typename T>
 __device__ __forceinline__ const T* row_ptr(const AcceptParams& p, int b, int r) {
-    const int V = p.V, k = p.k;
-    return r <= k ? static_cast<const T*>(p.target) + ((size_t)b * (k + 1) + r) * V
-                  : static_cast<const T*>(p.draft) + ((size_t)b * k + (r - k - 1)) * V;
+    const int V = p.V, nt = p.n_t;
+    return r < nt ? static_cast<const T*>(p.target) + ((size_t)b * nt + r) * V
+                  : static_cast<const T*>(p.draft) + ((size_t)b * p.d_rows + (r - nt)) * V;
+}
+
+// Bit u set iff tree node u of the parent array `par` (n <= 64 nodes) has a
+// child; every lane of the warp returns the same mask.
+__device__ __forceinline__ uint64_t tree_child_mask(const int32_t* par, int n, int lane) {
+    uint64_t m = 0;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = lane + 32 * h;
+        if (c > 0 && c < n) {
+            const int q = __ldg(par + c);
+            if (q >= 0 && q < c) m |= 1ull << q;
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) m |= __shfl_xor_sync(0xffffffffu, m, off);
+    return m;
 }
 
 // x / d for x >= 0, d > 0: one 32-bit division whenever both fit (every
@@ -262,10 +292,33 @@ __global__ void __launch_bounds__(kThreads, 2) accept_stats_kernel(const AcceptP
     if (w >= p.W) return;
     const long long lo = range_lo(p, w), hi = range_lo(p, w + 1);
     const int I = p.I, V = p.V, R = p.R;
+    // tree: the draft row of a node without children is never used; its
+    // items are skipped (read as -inf).  The child mask is cached per request.
+    long long kids_b = -1;
+    uint64_t kids = 0;
+    auto unused_row = [&](long long row) -> bool {
+        if (kGreedy || !p.parents) return false;
+        const int r = (int)(row % R);
+        if (r < p.n_t) return false;
+        const long long b = row / R;
+        if (b != kids_b) {
+            kids = tree_child_mask(p.parents + (size_t)b * p.n_t, p.n_t, lane);
+            kids_b = b;
+        }
+        return !((kids >> (r - p.n_t)) & 1ull);
+    };
 
     // One item into registers: lane l holds vectors u*32 + l; entries past
     // the row's end read as -inf.
     auto load = [&](long long row, int item, uint4 (&v)[kVecs]) {
+        if (unused_row(row)) {
+            Vec16<T> ninf;
+#pragma unroll
+            for (int e = 0; e < 16 / (int)sizeof(T); ++e) ninf.t[e] = (T)kNegInf;
+#pragma unroll
+            for (int u = 0; u < kVecs; ++u) v[u] = ninf.q;
+            return;
+        }
         const T* rp = row_ptr<T>(p, (int)(row / R), (int)(row % R));
         const int e0 = item * kItem, e1 = min(V, e0 + kItem);
         if (aligned16(rp) && e1 - e0 == kItem) {
@@ -379,11 +432,13 @@ __device__ __forceinline__ void fold_rows(const AcceptParams& p, int b, int firs
 }
 
 // ------------------------------------------------------------ accept test
-// Whether position i rejects: u_i < p_i(x_i) / q_i(x_i) fails.  zt, zd are
-// the target and draft logits of x_i, st, sd the rows' statistics.
-__device__ __forceinline__ bool rejects(bool valid, float zt, float zd, float2 st, float2 sd, float u,
-                                        float c_hi, float c_lo) {
-    if (!valid || zt == kNegInf) return true;
+// p(x) / q(x) of a drafted token: zt, zd are its target and draft logits,
+// st, sd the rows' statistics; 0 for an invalid token or p(x) == 0, +inf
+// when q(x) == 0.
+__device__ __forceinline__ float accept_ratio(bool valid, float zt, float zd, float2 st, float2 sd,
+                                              float c_hi, float c_lo) {
+    if (!valid || zt == kNegInf) return 0.f;
+    if (zd == kNegInf) return __int_as_float(0x7f800000);
     // log2 p(x)/q(x) = ((zt - mt) - (zd - md)) c + log2 Sd - log2 St, carried
     // as an unevaluated float pair
     const float dz = (zt - st.x) - (zd - sd.x);
@@ -393,8 +448,13 @@ __device__ __forceinline__ bool rejects(bool valid, float zt, float zd, float2 s
     const float H = A + Bl;
     const float bb = H - A;
     E += (A - (H - bb)) + (Bl - bb);
-    const float ratio = ex2(H) * fmaf(E, kLn2, 1.f);
-    return !(u < ratio);
+    return ex2(H) * fmaf(E, kLn2, 1.f);
+}
+
+// Whether position i rejects: u_i < p_i(x_i) / q_i(x_i) fails.
+__device__ __forceinline__ bool rejects(bool valid, float zt, float zd, float2 st, float2 sd, float u,
+                                        float c_hi, float c_lo) {
+    return !(u < accept_ratio(valid, zt, zd, st, sd, c_hi, c_lo));
 }
 
 // ------------------------------------------------------------ cluster PTX
@@ -532,6 +592,125 @@ __device__ __forceinline__ PassScan pass_scan(const DrawRow<T>& d, bool residual
                     : pass_scan_t<T, false>(d, pass_start, end, w, s_wsum, s_wlast);
 }
 
+// ------------------------------------------------------------ the draw
+// Inverse-CDF draw of one token from the weights of row pair d -- p, or
+// max(p - rho q, 0) when `residual` (rho as folded into d) -- over the
+// vocabulary slices of the cluster: this CTA owns [c0, c1) in n_pass passes.
+// Round 0 sums the slice masses and swaps them through distributed shared
+// memory; a residual without positive mass falls back to p in round 1.  On
+// return `writer` is the thread of this CTA that stores `token` (-1: another
+// CTA does).  Exchange slots alternate with the round counter xr, so one
+// cluster barrier per round keeps a slot from being rewritten while a peer
+// may still read it.
+template <typename T>
+__device__ __forceinline__ void cluster_draw(const DrawRow<T>& d, bool residual, float uk, int c0, int c1,
+                                             int n_pass, uint32_t rank, uint32_t n_ranks, float* s_pass,
+                                             float (&s_wsum)[kDrawWarps], int (&s_wlast)[kDrawWarps],
+                                             int (&s_first)[kDrawWarps], float2* s_x, int& xr, int& token,
+                                             int& writer) {
+    constexpr int kPer = 16 / (int)sizeof(T);
+    constexpr int kRun = kRunVecs * kPer;
+    constexpr int kPass = kDrawThreads * kRun;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    float w[kRun];
+    token = 0;
+    writer = -1;
+    for (int round = 0; round < 2; ++round) {
+        float mass = 0.f;
+        int last = -1;
+        PassScan kept{0.f, 0.f, 0.f, 0.f, -1};   // the last pass, whose weights stay in w
+        for (int ps = 0; ps < n_pass; ++ps) {
+            const int nx = c0 + (ps + 1) * kPass + tid * kRun;
+            if (ps + 1 < n_pass && (tid & 3) == 0 && nx < c1) {
+                // the next pass into L1 while this one is reduced (a 128-byte
+                // line holds the runs of four threads); only addresses inside
+                // the slice are touched
+                asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rt + nx));
+                if (residual) asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rd + nx));
+            }
+            kept = pass_scan<T>(d, residual, c0 + ps * kPass, c1, w, s_wsum, s_wlast);
+            if (tid == 0) s_pass[ps] = kept.total;
+            mass += kept.total;
+            last = max(last, kept.last);
+        }
+        const int slot = xr & 1;
+        ++xr;
+        if (tid == 0) s_x[slot] = make_float2(mass, __int_as_float(last));
+        cluster_arrive();
+        cluster_wait();
+        // every CTA folds the masses of ranks 0..n-1 in the same order
+        float2 x = make_float2(0.f, __int_as_float(-1));
+        if (lane < (int)n_ranks) x = ld_cluster_f2(&s_x[slot], lane);
+        const float incl = warp_incl_scan(x.x, lane);
+        const float Z = __shfl_sync(0xffffffffu, incl, 31);
+        if (!(Z > 0.f) && residual && round == 0) {
+            // no positive residual (p == q up to rounding): draw from p instead
+            residual = false;
+            continue;
+        }
+        const float t = uk * Z;
+        const float before = incl - x.x;
+        const unsigned own = __ballot_sync(0xffffffffu, lane < (int)n_ranks && x.x > 0.f && incl > t);
+        if (!own) {
+            // u_k * Z at or past the total through rounding: the last positive weight
+            const int lp = warp_max_int(__float_as_int(x.y));
+            token = lp >= 0 ? lp : 0;
+            if (rank == 0) writer = 0;
+            break;
+        }
+        const int owner = __ffs(own) - 1;
+        if ((int)rank != owner) break;
+        float tt = t - __shfl_sync(0xffffffffu, before, owner);   // position within this slice
+        // the pass that holds the cell, in the order the mass was summed
+        int pj = -1;
+        float cum = 0.f;
+        for (int ps = 0; ps < n_pass; ++ps) {
+            const float m = s_pass[ps];
+            if (m > 0.f && cum + m > tt) {
+                pj = ps;
+                break;
+            }
+            cum += m;
+        }
+        if (pj < 0) {   // rounding: the slice's last positive weight
+            token = last;
+            writer = 0;
+            break;
+        }
+        tt -= cum;
+        // the weights of the last pass are still in registers; others are recomputed
+        const PassScan sc = pj == n_pass - 1 ? kept : pass_scan<T>(d, residual, c0 + pj * kPass, c1, w, s_wsum, s_wlast);
+        // the first run with positive mass whose prefix passes tt (a run of
+        // zero weights can come first through rounding; it never owns the draw)
+        const unsigned cross = __ballot_sync(0xffffffffu, sc.own > 0.f && sc.incl > tt);
+        if (lane == 0) s_first[wid] = cross ? wid * 32 + __ffs(cross) - 1 : INT_MAX;
+        __syncthreads();
+        int first = INT_MAX;
+#pragma unroll
+        for (int j = 0; j < kDrawWarps; ++j) first = min(first, s_first[j]);
+        if (first == INT_MAX) {   // rounding: the pass's last positive weight
+            token = sc.last;
+            writer = 0;
+            break;
+        }
+        if (tid == first) {
+            const int start = c0 + pj * kPass + tid * kRun;
+            float c = sc.excl;
+            int pick = -1, lastp = -1;
+#pragma unroll
+            for (int e = 0; e < kRun; ++e) {
+                c += w[e];
+                if (w[e] > 0.f) {   // only a token with positive weight can be drawn
+                    lastp = start + e;
+                    if (pick < 0 && c > tt) pick = start + e;
+                }
+            }
+            token = pick >= 0 ? pick : lastp;   // the run has a positive weight
+        }
+        writer = first;
+        break;
+    }}
+
 // ------------------------------------------------------------ kernel 2
 template <typename T>
 __global__ void __launch_bounds__(kDrawThreads, 2) accept_draw_kernel(const AcceptParams p) {
@@ -605,103 +784,11 @@ __global__ void __launch_bounds__(kDrawThreads, 2) accept_draw_kernel(const Acce
             if (a < k) asm volatile("prefetch.global.L2 [%0];" ::"l"(bd + off));
         }
     }
-    bool residual = a < k;
-    float w[kRun];
     int token = 0;
     int writer = -1;   // the thread of this CTA that writes the emitted token
-    for (int round = 0; round < 2; ++round) {
-        float mass = 0.f;
-        int last = -1;
-        PassScan kept{0.f, 0.f, 0.f, 0.f, -1};   // the last pass, whose weights stay in w
-        for (int ps = 0; ps < n_pass; ++ps) {
-            const int nx = c0 + (ps + 1) * kPass + tid * kRun;
-            if (ps + 1 < n_pass && (tid & 3) == 0 && nx < c1) {
-                // the next pass into L1 while this one is reduced (a 128-byte
-                // line holds the runs of four threads); only addresses inside
-                // the slice are touched
-                asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rt + nx));
-                if (residual) asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rd + nx));
-            }
-            kept = pass_scan<T>(d, residual, c0 + ps * kPass, c1, w, s_wsum, s_wlast);
-            if (tid == 0) s_pass[ps] = kept.total;
-            mass += kept.total;
-            last = max(last, kept.last);
-        }
-        if (tid == 0) s_x[round] = make_float2(mass, __int_as_float(last));
-        cluster_arrive();
-        cluster_wait();
-        // every CTA folds the masses of ranks 0..n-1 in the same order
-        float2 x = make_float2(0.f, __int_as_float(-1));
-        if (lane < (int)n_ranks) x = ld_cluster_f2(&s_x[round], lane);
-        const float incl = warp_incl_scan(x.x, lane);
-        const float Z = __shfl_sync(0xffffffffu, incl, 31);
-        if (!(Z > 0.f) && residual && round == 0) {
-            // no positive residual (p == q up to rounding): draw from p instead
-            residual = false;
-            continue;
-        }
-        const float t = uk * Z;
-        const float before = incl - x.x;
-        const unsigned own = __ballot_sync(0xffffffffu, lane < (int)n_ranks && x.x > 0.f && incl > t);
-        if (!own) {
-            // u_k * Z at or past the total through rounding: the last positive weight
-            const int lp = warp_max_int(__float_as_int(x.y));
-            token = lp >= 0 ? lp : 0;
-            if (rank == 0) writer = 0;
-            break;
-        }
-        const int owner = __ffs(own) - 1;
-        if ((int)rank != owner) break;
-        float tt = t - __shfl_sync(0xffffffffu, before, owner);   // position within this slice
-        // the pass that holds the cell, in the order the mass was summed
-        int pj = -1;
-        float cum = 0.f;
-        for (int ps = 0; ps < n_pass; ++ps) {
-            const float m = s_pass[ps];
-            if (m > 0.f && cum + m > tt) {
-                pj = ps;
-                break;
-            }
-            cum += m;
-        }
-        if (pj < 0) {   // rounding: the slice's last positive weight
-            token = last;
-            writer = 0;
-            break;
-        }
-        tt -= cum;
-        // the weights of the last pass are still in registers; others are recomputed
-        const PassScan sc = pj == n_pass - 1 ? kept : pass_scan<T>(d, residual, c0 + pj * kPass, c1, w, s_wsum, s_wlast);
-        // the first run with positive mass whose prefix passes tt (a run of
-        // zero weights can come first through rounding; it never owns the draw)
-        const unsigned cross = __ballot_sync(0xffffffffu, sc.own > 0.f && sc.incl > tt);
-        if (lane == 0) s_first[wid] = cross ? wid * 32 + __ffs(cross) - 1 : INT_MAX;
-        __syncthreads();
-        int first = INT_MAX;
-#pragma unroll
-        for (int j = 0; j < kDrawWarps; ++j) first = min(first, s_first[j]);
-        if (first == INT_MAX) {   // rounding: the pass's last positive weight
-            token = sc.last;
-            writer = 0;
-            break;
-        }
-        if (tid == first) {
-            const int start = c0 + pj * kPass + tid * kRun;
-            float c = sc.excl;
-            int pick = -1, lastp = -1;
-#pragma unroll
-            for (int e = 0; e < kRun; ++e) {
-                c += w[e];
-                if (w[e] > 0.f) {   // only a token with positive weight can be drawn
-                    lastp = start + e;
-                    if (pick < 0 && c > tt) pick = start + e;
-                }
-            }
-            token = pick >= 0 ? pick : lastp;   // the run has a positive weight
-        }
-        writer = first;
-        break;
-    }
+    int xr = 0;
+    cluster_draw<T>(d, a < k, uk, c0, c1, n_pass, rank, n_ranks, s_pass, s_wsum, s_wlast, s_first, s_x, xr,
+                    token, writer);
     if (tid == writer) p.out_tokens[(size_t)b * (k + 1) + a] = token >= 0 ? token : 0;
     if (rank == 0 && tid <= k && tid != a) {
         const int32_t x = tid < a ? __ldg(p.tokens + (size_t)b * k + tid) : -1;
@@ -737,6 +824,224 @@ __global__ void __launch_bounds__(kThreads) accept_greedy_kernel(const AcceptPar
     if (lane == 0 && p.out_n) p.out_n[b] = a;
 }
 
+// ------------------------------------------------------------ token trees
+// Cluster-wide mass of the draw weights of row pair d (p scaled by S_t, or
+// max(p - kappa q, 0) scaled by S_t when `residual`): every CTA sums its
+// slice, the slice masses are swapped through distributed shared memory and
+// folded in rank order, so every CTA holds the same total.
+template <typename T>
+__device__ __forceinline__ float cluster_mass(const DrawRow<T>& d, bool residual, int c0, int c1, int n_pass,
+                                              uint32_t n_ranks, float (&s_wsum)[kDrawWarps],
+                                              int (&s_wlast)[kDrawWarps], float2* s_x, int& xr) {
+    constexpr int kRun = kRunVecs * 16 / (int)sizeof(T);
+    constexpr int kPass = kDrawThreads * kRun;
+    float w[kRun];
+    float mass = 0.f;
+    for (int ps = 0; ps < n_pass; ++ps) mass += pass_scan<T>(d, residual, c0 + ps * kPass, c1, w, s_wsum, s_wlast).total;
+    const int slot = xr & 1;
+    ++xr;
+    if (threadIdx.x == 0) s_x[slot] = make_float2(mass, 0.f);
+    cluster_arrive();
+    cluster_wait();
+    const int lane = threadIdx.x & 31;
+    float2 x = make_float2(0.f, 0.f);
+    if (lane < (int)n_ranks) x = ld_cluster_f2(&s_x[slot], lane);
+    return __shfl_sync(0xffffffffu, warp_incl_scan(x.x, lane), 31);
+}
+
+// One cluster per request walks its tree (multi-candidate speculative
+// sampling).  At node u the running distribution is r = max(p_u - kappa q_u,
+// 0) / Z (kappa = 0, Z = 1: r = p_u); child c with token x is accepted iff
+// u_{c-1} < r(x) / q_u(x) = max(p(x)/q(x) - kappa, 0) / Z.  A rejection
+// makes r the residual max(0, r - q_u) normalised, which is the same form
+// with kappa + Z in place of kappa; its mass is one cluster pass over the
+// row pair, needed only when another sibling is still to be tested (the
+// draw sums its own weights).  A residual without positive mass ends the
+// tests and the draw falls back to p_u.
+template <typename T>
+__global__ void __launch_bounds__(kDrawThreads, 2) tree_draw_kernel(const AcceptParams p) {
+    constexpr int kPer = 16 / (int)sizeof(T);
+    constexpr int kRun = kRunVecs * kPer;
+    constexpr int kPass = kDrawThreads * kRun;
+    __shared__ float2 s_stat[2 * kMaxTreeNodes];
+    __shared__ float2 s_z[kMaxTreeNodes];      // target / draft logit of node c's token in its parent's rows
+    __shared__ int s_par[kMaxTreeNodes];
+    __shared__ int s_tok[kMaxTreeNodes];
+    __shared__ float s_u[kMaxTreeNodes];
+    __shared__ unsigned long long s_kids[kMaxTreeNodes];
+    __shared__ int s_path[kMaxTreeNodes];
+    __shared__ float s_pass[kMaxPasses];
+    __shared__ float s_wsum[kDrawWarps];
+    __shared__ int s_wlast[kDrawWarps];
+    __shared__ int s_first[kDrawWarps];
+    __shared__ float2 s_x[2];
+
+    const int tid = threadIdx.x, lane = tid & 31;
+    const uint32_t rank = cluster_rank(), n_ranks = cluster_size();
+    const int b = p.b_base + blockIdx.y;
+    const int n = p.n_t, V = p.V;
+
+    // ---- the tree and every accept-test input, loaded before the statistics
+    for (int c = tid; c < n; c += kDrawThreads) {
+        int par = -1;
+        if (c > 0) {
+            const int q = __ldg(p.parents + (size_t)b * n + c);
+            par = (q >= 0 && q < c) ? q : -1;
+        }
+        const int x = __ldg(p.tokens + (size_t)b * n + c);
+        s_par[c] = par;
+        s_tok[c] = x;
+        s_u[c] = __ldg(p.uniforms + (size_t)b * n + c);
+        float2 z = make_float2(kNegInf, 0.f);    // an invalid token tests as ratio 0
+        if (par >= 0 && x >= 0 && x < V)
+            z = make_float2(to_f(row_ptr<T>(p, b, par)[x]), to_f(row_ptr<T>(p, b, n + par)[x]));
+        s_z[c] = z;
+    }
+    __syncthreads();
+    for (int u = tid; u < n; u += kDrawThreads) {
+        unsigned long long m = 0;
+        for (int c = u + 1; c < n; ++c)
+            if (s_par[c] == u) m |= 1ull << c;
+        s_kids[u] = m;
+    }
+    wait_prior_grid();
+    fold_rows<false, 8>(p, b, tid >> 5, kDrawWarps, p.R, lane, s_stat);
+    __syncthreads();
+
+    // ---- the walk: every thread takes the same decisions from shared data
+    const int c0 = min(V, (int)rank * p.slice), c1 = min(V, c0 + p.slice);
+    const int n_pass = (c1 - c0 + kPass - 1) / kPass;
+    int node = 0, depth = 0, xr = 0;
+    float kappa = 0.f;
+    DrawRow<T> d;
+    d.c_hi = p.c_hi;
+    for (;;) {
+        const float2 st = s_stat[node], sd = s_stat[n + node];
+        d.rt = row_ptr<T>(p, b, node);
+        d.rd = row_ptr<T>(p, b, n + node);
+        d.mt = st.x == kNegInf ? 0.f : st.x;
+        d.md = sd.x == kNegInf ? 0.f : sd.x;
+        d.at = aligned16(d.rt);
+        d.ad = aligned16(d.rd);
+        const float rho1 = sd.y > 0.f ? st.y / sd.y : 0.f;
+        unsigned long long kids = s_kids[node];
+        float kap = 0.f, Z = 1.f;
+        int next = -1;
+        while (kids) {
+            const int c = __ffsll((long long)kids) - 1;
+            kids &= kids - 1;
+            const float2 z = s_z[c];
+            float ratio = accept_ratio(z.x != kNegInf, z.x, z.y, st, sd, p.c_hi, p.c_lo);
+            if (kap > 0.f) ratio = fmaxf(ratio - kap, 0.f) / Z;
+            if (s_u[c - 1] < ratio) {
+                next = c;
+                break;
+            }
+            kap += Z;               // the residual of this rejection
+            if (!kids) break;       // no sibling left: the draw sums its own weights
+            d.rho = kap * rho1;
+            Z = cluster_mass<T>(d, true, c0, c1, n_pass, n_ranks, s_wsum, s_wlast, s_x, xr) / st.y;
+            if (!(Z > 0.f)) {       // no positive residual (p == kappa q up to rounding): draw from p
+                kap = 0.f;
+                break;
+            }
+        }
+        if (next < 0) {
+            kappa = kap;
+            break;
+        }
+        if (tid == 0) s_path[depth] = next;
+        ++depth;
+        node = next;
+    }
+
+    // ---- the draw at the final node
+    d.rho = kappa * (s_stat[n + node].y > 0.f ? s_stat[node].y / s_stat[n + node].y : 0.f);
+    if (!(kappa > 0.f)) d.rd = d.rt;
+    if (n_pass > 1) {
+        const char* bt = reinterpret_cast<const char*>(d.rt + c0);
+        const char* bd = reinterpret_cast<const char*>(d.rd + c0);
+        const int bytes = (c1 - c0) * (int)sizeof(T);
+        for (int off = tid * 128; off < bytes; off += kDrawThreads * 128) {
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(bt + off));
+            if (kappa > 0.f) asm volatile("prefetch.global.L2 [%0];" ::"l"(bd + off));
+        }
+    }
+    int token = 0, writer = -1;
+    cluster_draw<T>(d, kappa > 0.f, s_u[n - 1], c0, c1, n_pass, rank, n_ranks, s_pass, s_wsum, s_wlast, s_first,
+                    s_x, xr, token, writer);
+    __syncthreads();
+    int32_t* out = p.out_tokens + (size_t)b * n;
+    if (tid == writer) out[depth] = token >= 0 ? token : 0;
+    if (rank == 0) {
+        for (int i = tid; i < n; i += kDrawThreads) {
+            if (i < depth) {
+                out[i] = s_tok[s_path[i]];
+                p.out_path[(size_t)b * n + i] = s_path[i];
+            } else {
+                if (i > depth) out[i] = -1;
+                p.out_path[(size_t)b * n + i] = -1;
+            }
+        }
+        if (tid == 0) p.out_n[b] = depth;
+    }
+    // no CTA leaves while another may still read its exchange slots
+    cluster_arrive();
+    cluster_wait();
+}
+
+// Greedy tree walk, one warp per request: at node u the first child whose
+// token is the arg max of u's target row is accepted, else that arg max is
+// emitted.
+template <typename T>
+__global__ void __launch_bounds__(kThreads) tree_greedy_kernel(const AcceptParams p) {
+    __shared__ float2 s_stat[kWarps][kMaxTreeNodes];
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+    const int b = blockIdx.x * kWarps + wid;
+    if (b >= p.B) return;
+    const int n = p.n_t;
+    int par[2], tok[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int c = lane + 32 * h;
+        par[h] = -1;
+        tok[h] = -1;
+        if (c < n) {
+            tok[h] = __ldg(p.tokens + (size_t)b * n + c);
+            if (c > 0) {
+                const int q = __ldg(p.parents + (size_t)b * n + c);
+                par[h] = (q >= 0 && q < c) ? q : -1;
+            }
+        }
+    }
+    wait_prior_grid();
+    fold_rows<true, 4>(p, b, 0, 1, n, lane, s_stat[wid]);
+    __syncwarp();
+    int32_t* out = p.out_tokens + (size_t)b * n;
+    int32_t* path = p.out_path + (size_t)b * n;
+    int node = 0, depth = 0, g = 0;
+    for (;;) {
+        g = __float_as_int(s_stat[wid][node].y);
+        if (g == INT_MAX) g = 0;   // a row with no finite entry
+        const unsigned m0 = __ballot_sync(0xffffffffu, par[0] == node && tok[0] == g);
+        const unsigned m1 = __ballot_sync(0xffffffffu, par[1] == node && tok[1] == g);
+        if (!m0 && !m1) break;
+        const int next = m0 ? __ffs(m0) - 1 : 32 + __ffs(m1) - 1;
+        if (lane == 0) {
+            out[depth] = g;
+            path[depth] = next;
+        }
+        ++depth;
+        node = next;
+    }
+    for (int i = lane; i < n; i += 32) {
+        if (i == depth) out[i] = g;
+        else if (i > depth) out[i] = -1;
+        if (i >= depth) path[i] = -1;
+    }
+    if (lane == 0) p.out_n[b] = depth;
+}
+
 // ------------------------------------------------------------------- host
 // Resident CTAs of `kern` on the current device (cached per device and slot).
 template <typename K>
@@ -765,10 +1070,12 @@ int max_cluster_size() {
     if (dev < 0 || dev >= 64) return 8;
     if (g_max_cluster[dev]) return g_max_cluster[dev];
     int best = 8;
-    auto kern = accept_draw_kernel<__nv_bfloat16>;
-    auto kern32 = accept_draw_kernel<float>;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess &&
-        cudaFuncSetAttribute(kern32, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess) {
+    void (*kerns[4])(const AcceptParams) = {accept_draw_kernel<__nv_bfloat16>, accept_draw_kernel<float>,
+                                            tree_draw_kernel<__nv_bfloat16>, tree_draw_kernel<float>};
+    bool attrs_ok = true;
+    for (auto k : kerns)
+        attrs_ok = attrs_ok && cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) == cudaSuccess;
+    if (attrs_ok) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(kMaxCluster, 1, 1);
         cfg.blockDim = dim3(kDrawThreads, 1, 1);
@@ -779,10 +1086,12 @@ int max_cluster_size() {
         attr.val.clusterDim.z = 1;
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
-        int n = 0, n32 = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) == cudaSuccess && n > 0 &&
-            cudaOccupancyMaxActiveClusters(&n32, kern32, &cfg) == cudaSuccess && n32 > 0)
-            best = kMaxCluster;
+        bool all = true;
+        for (auto k : kerns) {
+            int n = 0;
+            all = all && cudaOccupancyMaxActiveClusters(&n, k, &cfg) == cudaSuccess && n > 0;
+        }
+        if (all) best = kMaxCluster;
     }
     cudaGetLastError();
     g_max_cluster[dev] = best;
@@ -802,10 +1111,12 @@ int stats_resident() {
     return resident_ctas(accept_stats_kernel<T, G>, slot, kThreads, 0);
 }
 
-AcceptPlan plan_accept(const cs_accept_dims& d, int n_draft, bool greedy, bool with_cluster) {
+// n_t target rows and d_rows draft rows per request (chain: k+1 and k;
+// tree: the node count twice).
+AcceptPlan plan_accept_rows(const cs_accept_dims& d, int n_t, int d_rows, bool greedy, bool with_cluster) {
     const bool f32 = d.logit_dtype == CS_F32;
     AcceptPlan P{};
-    P.R = greedy ? n_draft + 1 : 2 * n_draft + 1;
+    P.R = greedy ? n_t : n_t + d_rows;
     const int item = kItemBytes / (f32 ? 4 : 2);
     P.I = (d.vocab + item - 1) / item;
     P.N = (long long)d.batch * P.R * P.I;
@@ -846,8 +1157,12 @@ AcceptPlan plan_accept(const cs_accept_dims& d, int n_draft, bool greedy, bool w
     return P;
 }
 
+AcceptPlan plan_accept(const cs_accept_dims& d, int n_draft, bool greedy, bool with_cluster) {
+    return plan_accept_rows(d, n_draft + 1, n_draft, greedy, with_cluster);
+}
+
 template <typename T, bool G>
-cs_status launch_typed(AcceptParams p, const AcceptPlan& P, cudaStream_t stream) {
+cs_status launch_typed(AcceptParams p, const AcceptPlan& P, bool tree, cudaStream_t stream) {
     accept_stats_kernel<T, G><<<P.grid1, kThreads, 0, stream>>>(p);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "accept_stats_kernel launch");
@@ -864,11 +1179,11 @@ cs_status launch_typed(AcceptParams p, const AcceptPlan& P, cudaStream_t stream)
         cfg.stream = stream;
         cfg.attrs = attrs;
         cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, accept_greedy_kernel<T>, p);
-        if (e != cudaSuccess) return cuda_fail(e, "accept_greedy_kernel launch");
+        e = cudaLaunchKernelEx(&cfg, tree ? tree_greedy_kernel<T> : accept_greedy_kernel<T>, p);
+        if (e != cudaSuccess) return cuda_fail(e, "greedy acceptance kernel launch");
         return CS_OK;
     }
-    auto kern = accept_draw_kernel<T>;
+    auto kern = tree ? tree_draw_kernel<T> : accept_draw_kernel<T>;
     if (P.cluster > 8) {
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(non-portable cluster)");
@@ -886,7 +1201,7 @@ cs_status launch_typed(AcceptParams p, const AcceptPlan& P, cudaStream_t stream)
         cfg.attrs = attrs;
         cfg.numAttrs = 2;
         e = cudaLaunchKernelEx(&cfg, kern, p);
-        if (e != cudaSuccess) return cuda_fail(e, "accept_draw_kernel launch");
+        if (e != cudaSuccess) return cuda_fail(e, "acceptance draw kernel launch");
     }
     return CS_OK;
 }
@@ -920,6 +1235,8 @@ cs_status launch_spec_accept(const cs_accept_dims& d, const void* target, const 
     p.B = d.batch;
     p.V = d.vocab;
     p.k = n_draft;
+    p.n_t = n_draft + 1;
+    p.d_rows = n_draft;
     p.R = P.R;
     p.I = P.I;
     p.N = P.N;
@@ -932,9 +1249,52 @@ cs_status launch_spec_accept(const cs_accept_dims& d, const void* target, const 
     p.part = static_cast<float2*>(workspace);
     p.cnt = reinterpret_cast<int*>(static_cast<uint8_t*>(workspace) + P.off_cnt);
     if (d.logit_dtype == CS_F32)
-        return greedy ? launch_typed<float, true>(p, P, stream) : launch_typed<float, false>(p, P, stream);
-    return greedy ? launch_typed<__nv_bfloat16, true>(p, P, stream)
-                  : launch_typed<__nv_bfloat16, false>(p, P, stream);
+        return greedy ? launch_typed<float, true>(p, P, false, stream) : launch_typed<float, false>(p, P, false, stream);
+    return greedy ? launch_typed<__nv_bfloat16, true>(p, P, false, stream)
+                  : launch_typed<__nv_bfloat16, false>(p, P, false, stream);
+}
+
+size_t tree_accept_workspace_bytes(const cs_accept_dims& d, int n_nodes) {
+    const size_t a = plan_accept_rows(d, n_nodes, n_nodes, true, false).bytes;
+    const size_t b = plan_accept_rows(d, n_nodes, n_nodes, false, false).bytes;
+    return a > b ? a : b;
+}
+
+cs_status launch_tree_accept(const cs_accept_dims& d, const void* target, const void* draft,
+                             const int32_t* parents, const int32_t* tokens, const float* uniforms, int n_nodes,
+                             float temperature, int32_t* out_tokens, int32_t* out_path, int32_t* out_n,
+                             void* workspace, cudaStream_t stream) {
+    const bool greedy = temperature == 0.f;
+    const AcceptPlan P = plan_accept_rows(d, n_nodes, n_nodes, greedy, true);
+    AcceptParams p{};
+    p.target = target;
+    p.draft = draft;
+    p.tokens = tokens;
+    p.uniforms = uniforms;
+    p.out_tokens = out_tokens;
+    p.out_n = out_n;
+    p.parents = parents;
+    p.out_path = out_path;
+    p.B = d.batch;
+    p.V = d.vocab;
+    p.k = n_nodes - 1;
+    p.n_t = n_nodes;
+    p.d_rows = n_nodes;
+    p.R = P.R;
+    p.I = P.I;
+    p.N = P.N;
+    p.W = P.W;
+    p.J = P.J;
+    p.slice = P.slice;
+    const double c = temperature > 0.f ? 1.4426950408889634 / (double)temperature : 0.0;
+    p.c_hi = (float)c;
+    p.c_lo = (float)(c - (double)p.c_hi);
+    p.part = static_cast<float2*>(workspace);
+    p.cnt = reinterpret_cast<int*>(static_cast<uint8_t*>(workspace) + P.off_cnt);
+    if (d.logit_dtype == CS_F32)
+        return greedy ? launch_typed<float, true>(p, P, true, stream) : launch_typed<float, false>(p, P, true, stream);
+    return greedy ? launch_typed<__nv_bfloat16, true>(p, P, true, stream)
+                  : launch_typed<__nv_bfloat16, false>(p, P, true, stream);
 }
 
 }  // namespace cs

@@ -14,6 +14,13 @@
 // kernel merges the pieces of every cut span with log-sum-exp weights, all
 // spans in parallel.
 //
+// Token trees (the multi-candidate verification variant) use the same
+// kernel with a different mask: node i of a request's tree sees every prefix
+// key and the rows of its own ancestors, found from the parent array by
+// pointer doubling at the start of each span.  A tree whose (nodes x G)
+// query rows exceed what one CTA holds is cut into row blocks, each its own
+// span ("virtual head") over the same keys.
+//
 // Per CTA: one producer warp streams the K and V tiles of its range through
 // TMA (one 4-D tensor map over the page pool, 128-byte swizzle, one box per
 // page piece) into a 3-stage shared-memory ring guarded by mbarriers, without
@@ -53,10 +60,14 @@ struct AttnParams {
     __nv_bfloat16* out;          // [B, R, Hq, D]
     const int32_t* page_table;   // [B, max_pages]
     const int32_t* ctx_lens;     // [B]
+    const int32_t* parents;      // [B, R] tree parents (tree kernel only)
     float* part_o;               // [2 * grid, n_rows, D]
     float2* part_ml;             // [2 * grid, n_rows]  (m in log2 units, l)
     int* status;
     int Hq, Hkv, G, R, n_rows, ps, box_t, max_pages, row_warps;
+    int n_rb;                    // row blocks per KV head (n_rows rows each)
+    int n_vh;                    // Hkv * n_rb spans per request ("virtual heads")
+    int n_rows_all;              // R * G query rows per KV head
     int b_base, n_batch;         // requests [b_base, b_base + n_batch) in this launch
     float scale_log2;            // sm_scale * log2(e)
 };
@@ -78,7 +89,7 @@ struct Cursor {
 };
 
 __device__ __forceinline__ Cursor locate(long long f, const long long* prefix, const int* lens,
-                                         int n_batch, int Hkv) {
+                                         int n_batch, int n_vh) {
     int lo = 0, hi = n_batch - 1;   // largest b with prefix[b] <= f
     while (lo < hi) {
         const int mid = (lo + hi + 1) >> 1;
@@ -94,14 +105,51 @@ __device__ __forceinline__ Cursor locate(long long f, const long long* prefix, c
     return c;
 }
 
-__device__ __forceinline__ void advance(Cursor& c, const int* lens, int n_batch, int Hkv) {
+__device__ __forceinline__ void advance(Cursor& c, const int* lens, int n_batch, int n_vh) {
     if (++c.t < c.T) return;
     c.t = 0;
-    if (++c.h < Hkv) return;
+    if (++c.h < n_vh) return;
     c.h = 0;
     if (++c.b < n_batch) c.T = tiles_of(lens[c.b]);
 }
 
+// Ancestor-or-self bit masks of tree nodes `lane` and `lane + 32` (n <= 64
+// nodes; a parent outside [0, c) detaches node c).  Pointer doubling: after
+// round r a node's mask holds its ancestors closer than 2^(r+1) levels and
+// its jump points 2^(r+1) levels up, so six rounds cover any depth < 64.
+__device__ __forceinline__ void tree_ancestor_masks(const int32_t* par, int n, int lane, uint64_t& m0,
+                                                    uint64_t& m1) {
+    const int c0 = lane, c1 = lane + 32;
+    int j0 = -1, j1 = -1;
+    if (c0 > 0 && c0 < n) {
+        const int q = __ldg(par + c0);
+        j0 = (q >= 0 && q < c0) ? q : -1;
+    }
+    if (c1 < n) {
+        const int q = __ldg(par + c1);
+        j1 = (q >= 0 && q < c1) ? q : -1;
+    }
+    m0 = c0 < n ? (1ull << c0) : 0ull;
+    m1 = c1 < n ? (1ull << c1) : 0ull;
+#pragma unroll
+    for (int r = 0; r < 6; ++r) {
+        const int s0 = j0 & 31, s1 = j1 & 31;
+        const uint64_t a0 = __shfl_sync(0xffffffffu, m0, s0), a1 = __shfl_sync(0xffffffffu, m1, s0);
+        const int ja0 = __shfl_sync(0xffffffffu, j0, s0), ja1 = __shfl_sync(0xffffffffu, j1, s0);
+        const uint64_t b0 = __shfl_sync(0xffffffffu, m0, s1), b1 = __shfl_sync(0xffffffffu, m1, s1);
+        const int jb0 = __shfl_sync(0xffffffffu, j0, s1), jb1 = __shfl_sync(0xffffffffu, j1, s1);
+        if (j0 >= 0) {
+            m0 |= j0 >= 32 ? a1 : a0;
+            j0 = j0 >= 32 ? ja1 : ja0;
+        }
+        if (j1 >= 0) {
+            m1 |= j1 >= 32 ? b1 : b0;
+            j1 = j1 >= 32 ? jb1 : jb0;
+        }
+    }
+}
+
+template <bool kTree>
 __global__ void __launch_bounds__((kMaxRowWarps + 1) * 32, 1)
 verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                         const __grid_constant__ CUtensorMap tmap_v, const AttnParams p) {
@@ -140,7 +188,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             int L = __ldg(p.ctx_lens + p.b_base + bl);
             L = max(0, min(L, l_cap));
             s_len[bl] = L;
-            v = (long long)tiles_of(L) * p.Hkv;
+            v = (long long)tiles_of(L) * p.n_vh;
         }
         long long inc = v;
 #pragma unroll
@@ -184,7 +232,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
         const int pieces = kTileT / p.box_t;
         const uint32_t piece_bytes = (uint32_t)p.box_t * 128u;
-        Cursor cur = locate(f0, s_prefix, s_len, nb, p.Hkv);
+        Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
         auto piece_page = [&](const Cursor& cc) -> int {
             const int tok = cc.t * kTileT + lane * p.box_t;
             if (lane >= pieces || tok >= s_len[cc.b]) return -1;
@@ -197,8 +245,8 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             const int page = page_next;
             const int L = s_len[cur.b];
             const int ts = cur.t * kTileT;
-            const int h_cur = cur.h;
-            advance(cur, s_len, nb, p.Hkv);
+            const int h_cur = cur.h / p.n_rb;   // the KV head of this span
+            advance(cur, s_len, nb, p.n_vh);
             if (j + 1 < n_tiles) page_next = piece_page(cur);
             int ok = 1;
             if (lane == 0 && j >= kStages && !mbar_wait_bounded(&empty[st], (use - 1) & 1)) {
@@ -231,24 +279,33 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const int lm = lane >> 3, lr = lane & 7;   // ldmatrix: matrix index, row within it
     const float c = p.scale_log2;
 
-    Cursor cur = locate(f0, s_prefix, s_len, nb, p.Hkv);
+    Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
     int seg_t0 = cur.t;
     bool first_seg = true;
 
     uint32_t qa[8][4];
     float o[16][4];
     float m_raw[2], l[2];
-    int lim0 = 0, lim1 = 0;
+    int lim0 = 0, lim1 = 0;              // chain: exclusive key limit of each row
+    uint64_t anc0 = ~0ull, anc1 = ~0ull;   // tree: ancestor-or-self mask of each row's node
+    int tree_base = 0, span_L = 0;       // tree: key position of node 0, context length
+    int head = 0, grow0 = 0, grow1 = 0;  // KV head and global query rows of the span
 
     auto begin_span = [&](const Cursor& cc) {
         const int bg = p.b_base + cc.b;
+        head = cc.h / p.n_rb;
+        const int rbase = (cc.h - head * p.n_rb) * p.n_rows;
+        grow0 = row0 < p.n_rows ? rbase + row0 : p.n_rows_all;
+        grow1 = row1 < p.n_rows ? rbase + row1 : p.n_rows_all;
+        if (grow0 > p.n_rows_all) grow0 = p.n_rows_all;
+        if (grow1 > p.n_rows_all) grow1 = p.n_rows_all;
 #pragma unroll
         for (int k = 0; k < 2; ++k) {
-            const int r = k ? row1 : row0;
+            const int r = k ? grow1 : grow0;
             const __nv_bfloat16* qr = nullptr;
-            if (r < p.n_rows) {
+            if (r < p.n_rows_all) {
                 const int i = r / p.G, gi = r % p.G;
-                qr = p.q + (((size_t)bg * p.R + i) * p.Hq + (size_t)cc.h * p.G + gi) * kD;
+                qr = p.q + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD;
             }
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk) {
@@ -262,9 +319,21 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         m_raw[0] = m_raw[1] = kNegInf;
         l[0] = l[1] = 0.f;
         const int L = s_len[cc.b];
-        // exclusive key limit of each of this thread's two rows
-        lim0 = row0 < p.n_rows ? L - p.R + 1 + row0 / p.G : L;
-        lim1 = row1 < p.n_rows ? L - p.R + 1 + row1 / p.G : L;
+        if (kTree) {
+            uint64_t ma, mb;
+            tree_ancestor_masks(p.parents + (size_t)bg * p.R, p.R, lane, ma, mb);
+            const int i0 = grow0 / p.G, i1 = grow1 / p.G;
+            const uint64_t x0 = __shfl_sync(0xffffffffu, ma, i0 & 31), y0 = __shfl_sync(0xffffffffu, mb, i0 & 31);
+            const uint64_t x1 = __shfl_sync(0xffffffffu, ma, i1 & 31), y1 = __shfl_sync(0xffffffffu, mb, i1 & 31);
+            anc0 = grow0 < p.n_rows_all ? (i0 >= 32 ? y0 : x0) : ~0ull;
+            anc1 = grow1 < p.n_rows_all ? (i1 >= 32 ? y1 : x1) : ~0ull;
+            tree_base = L - p.R;
+            span_L = L;
+        } else {
+            // exclusive key limit of each of this thread's two rows
+            lim0 = grow0 < p.n_rows_all ? L - p.R + 1 + grow0 / p.G : L;
+            lim1 = grow1 < p.n_rows_all ? L - p.R + 1 + grow1 / p.G : L;
+        }
     };
     begin_span(cur);
 
@@ -310,7 +379,29 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             }
         }
         // ---- causal-verify mask (and the context end)
-        if (ts + kTileT > min(lim0, lim1)) {
+        if (kTree) {
+            // tree: a key in the tree region is visible iff its node is an
+            // ancestor (or the node itself); keys past L_b never are
+            if (ts + kTileT > tree_base) {
+                // visibility of the tile's 64 keys as one word per row: the
+                // prefix part, the row's ancestors shifted to the tile, and
+                // nothing at or past L_b
+                const int d = ts - tree_base;   // tree node of the tile's first key
+                const uint64_t pre = d >= 0 ? 0ull : (d <= -64 ? ~0ull : (1ull << -d) - 1ull);
+                const uint64_t live = span_L - ts >= 64 ? ~0ull : (1ull << max(span_L - ts, 0)) - 1ull;
+                const uint64_t t0 = d >= 64 ? 0ull : (d >= 0 ? anc0 >> d : (d <= -64 ? 0ull : anc0 << -d));
+                const uint64_t t1 = d >= 64 ? 0ull : (d >= 0 ? anc1 >> d : (d <= -64 ? 0ull : anc1 << -d));
+                const uint64_t v0 = ((pre | t0) & live) >> (tq * 2), v1 = ((pre | t1) & live) >> (tq * 2);
+#pragma unroll
+                for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        if (!((v0 >> (nt * 8 + e)) & 1ull)) sc[nt][e] = kNegInf;
+                        if (!((v1 >> (nt * 8 + e)) & 1ull)) sc[nt][2 + e] = kNegInf;
+                    }
+                }
+            }
+        } else if (ts + kTileT > min(lim0, lim1)) {
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
 #pragma unroll
@@ -377,7 +468,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         if (lane == 0) mbar_arrive(&empty[st]);
 
         if (j + 1 < n_tiles && cur.t + 1 < cur.T) {
-            advance(cur, s_len, nb, p.Hkv);
+            advance(cur, s_len, nb, p.n_vh);
             continue;
         }
 
@@ -394,12 +485,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         if (complete) {
 #pragma unroll
             for (int rh = 0; rh < 2; ++rh) {
-                const int row = rh ? row1 : row0;
-                if (row >= p.n_rows) continue;
+                const int grow = rh ? grow1 : grow0;
+                if (grow >= p.n_rows_all) continue;
                 const float inv = lt[rh] > 0.f ? 1.f / lt[rh] : 0.f;
-                const int i = row / p.G, gi = row % p.G;
+                const int i = grow / p.G, gi = grow % p.G;
                 __nv_bfloat16* dst =
-                    p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)cur.h * p.G + gi) * kD + tq * 2;
+                    p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + tq * 2;
 #pragma unroll
                 for (int dn = 0; dn < 16; ++dn)
                     *reinterpret_cast<uint32_t*>(dst + dn * 8) =
@@ -410,7 +501,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 #pragma unroll
             for (int rh = 0; rh < 2; ++rh) {
                 const int row = rh ? row1 : row0;
-                if (row >= p.n_rows) continue;
+                if (row >= p.n_rows || (rh ? grow1 : grow0) >= p.n_rows_all) continue;
                 float* dst = p.part_o + (slot * p.n_rows + row) * kD + tq * 2;
 #pragma unroll
                 for (int dn = 0; dn < 16; ++dn)
@@ -421,7 +512,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             }
         }
         if (j + 1 < n_tiles) {
-            advance(cur, s_len, nb, p.Hkv);
+            advance(cur, s_len, nb, p.n_vh);
             seg_t0 = cur.t;
             first_seg = false;
             begin_span(cur);
@@ -455,7 +546,7 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     for (int b = threadIdx.x; b < nb; b += kMergeThreads) {
         int L = __ldg(p.ctx_lens + p.b_base + b);
         L = max(0, min(L, l_cap));
-        const long long v = (long long)tiles_of(L) * p.Hkv;
+        const long long v = (long long)tiles_of(L) * p.n_vh;
         total += v;
         if (b < bl) before += v;
     }
@@ -500,7 +591,8 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     asm volatile("griddepcontrol.wait;" ::: "memory");
 
     const int bg = p.b_base + bl;
-    for (int row = warp; row < p.n_rows; row += kMergeThreads / 32) {
+    const int head = h / p.n_rb, rbase = (h - head * p.n_rb) * p.n_rows;
+    for (int row = warp; row < p.n_rows && rbase + row < p.n_rows_all; row += kMergeThreads / 32) {
         float M = kNegInf, lsum = 0.f;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int q0 = 0; q0 < n_p; q0 += kMergePieces) {
@@ -537,8 +629,8 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
             M = Mn;
         }
         const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
-        const int i = row / p.G, gi = row % p.G;
-        __nv_bfloat16* dst = p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)h * p.G + gi) * kD + lane * 4;
+        const int i = (rbase + row) / p.G, gi = (rbase + row) % p.G;
+        __nv_bfloat16* dst = p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + lane * 4;
         uint2 pk;
         pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
         pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
@@ -579,6 +671,7 @@ cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Resident CTAs per SM of the kernel at a given block size (cached per device).
+template <bool kTree>
 int resident_per_sm(int threads) {
     static int cache[64][kMaxRowWarps + 2] = {};
     int dev = 0;
@@ -590,9 +683,9 @@ int resident_per_sm(int threads) {
     if (key <= 0 || key > kMaxRowWarps + 1) return 1;
     if (!cache[dev][key]) {
         int n = 0;
-        if (cudaFuncSetAttribute(verify_attention_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(verify_attention_kernel<kTree>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  kSmemBytes) != cudaSuccess ||
-            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, verify_attention_kernel, threads,
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, verify_attention_kernel<kTree>, threads,
                                                           kSmemBytes) != cudaSuccess ||
             n <= 0) {
             cudaGetLastError();
@@ -605,14 +698,21 @@ int resident_per_sm(int threads) {
 
 }  // namespace
 
-AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count) {
+AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count) {
     AttnPlan pl{};
     pl.group = d.n_q_heads / d.n_kv_heads;
-    pl.rows = n_draft + 1;
-    pl.n_rows = pl.rows * pl.group;
+    pl.rows = rows;
+    pl.tree = tree;
+    pl.n_rows_all = pl.rows * pl.group;
+    // query rows of one span: all of them, or equal row blocks of a multiple
+    // of 16 rows when they do not fit one CTA
+    const int cap = kMaxRowWarps * 16;
+    pl.n_rb = (pl.n_rows_all + cap - 1) / cap;
+    pl.n_rows = pl.n_rb == 1 ? pl.n_rows_all : ((pl.n_rows_all + pl.n_rb - 1) / pl.n_rb + 15) / 16 * 16;
     pl.row_warps = (pl.n_rows + 15) / 16;
     // persistent grid: exactly the CTAs that are resident at once
-    pl.grid = (sm_count > 0 ? sm_count : 148) * resident_per_sm((pl.row_warps + 1) * 32);
+    const int threads = (pl.row_warps + 1) * 32;
+    pl.grid = (sm_count > 0 ? sm_count : 148) * (tree ? resident_per_sm<true>(threads) : resident_per_sm<false>(threads));
     if (pl.grid > kMaxGrid) pl.grid = kMaxGrid;
     size_t off = 256;   // status word lives at offset 0
     pl.off_part_ml = off;
@@ -623,10 +723,21 @@ AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count)
     return pl;
 }
 
+AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count) {
+    return plan_attention(d, n_draft + 1, false, sm_count);
+}
+
+AttnPlan plan_tree_attention(const cs_attn_dims& d, int n_nodes, int sm_count) {
+    return plan_attention(d, n_nodes, true, sm_count);
+}
+
 cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, const void* q,
                                   const void* k_pages, const void* v_pages,
-                                  const int32_t* page_table, const int32_t* ctx_lens, void* out,
-                                  void* workspace, cudaStream_t stream) {
+                                  const int32_t* page_table, const int32_t* ctx_lens,
+                                  const int32_t* parents, void* out, void* workspace,
+                                  cudaStream_t stream) {
+    if (pl.tree != (parents != nullptr))
+        return fail(CS_ERR_INVALID_ARG, "tree plan and parent array do not match");
     const int box_t = d.page_size < kTileT ? d.page_size : kTileT;
     CUtensorMap tk, tv;
     cs_status st = encode_pool_map(&tk, k_pages, d, box_t);
@@ -640,6 +751,7 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     p.out = static_cast<__nv_bfloat16*>(out);
     p.page_table = page_table;
     p.ctx_lens = ctx_lens;
+    p.parents = parents;
     p.status = reinterpret_cast<int*>(ws);
     p.part_ml = reinterpret_cast<float2*>(ws + pl.off_part_ml);
     p.part_o = reinterpret_cast<float*>(ws + pl.off_part_o);
@@ -652,27 +764,30 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     p.box_t = box_t;
     p.max_pages = d.max_pages_per_seq;
     p.row_warps = pl.row_warps;
+    p.n_rb = pl.n_rb;
+    p.n_vh = d.n_kv_heads * pl.n_rb;
+    p.n_rows_all = pl.n_rows_all;
     const float scale = d.sm_scale > 0.f ? d.sm_scale : 1.0f / sqrtf((float)d.head_dim);
     p.scale_log2 = scale * 1.4426950408889634f;
 
+    auto kern = pl.tree ? verify_attention_kernel<true> : verify_attention_kernel<false>;
     cudaError_t e = cudaSuccess;
     {
-        static bool attr_done[64] = {};
+        static bool attr_done[2][64] = {};
         int dev = 0;
         e = cudaGetDevice(&dev);
         if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-        if (dev < 0 || dev >= 64 || !attr_done[dev]) {
-            e = cudaFuncSetAttribute(verify_attention_kernel,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (dev < 0 || dev >= 64 || !attr_done[pl.tree][dev]) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
             if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_attention_kernel)");
-            if (dev >= 0 && dev < 64) attr_done[dev] = true;
+            if (dev >= 0 && dev < 64) attr_done[pl.tree][dev] = true;
         }
     }
     const dim3 block((pl.row_warps + 1) * 32);
     for (int b0 = 0; b0 < d.batch; b0 += kMaxBatchPerLaunch) {
         p.b_base = b0;
         p.n_batch = d.batch - b0 < kMaxBatchPerLaunch ? d.batch - b0 : kMaxBatchPerLaunch;
-        verify_attention_kernel<<<pl.grid, block, kSmemBytes, stream>>>(tk, tv, p);
+        kern<<<pl.grid, block, kSmemBytes, stream>>>(tk, tv, p);
         e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_fail(e, "verify_attention_kernel launch");
         // programmatic dependent launch: the merge kernel may start early and
@@ -681,7 +796,7 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
         attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr.val.programmaticStreamSerializationAllowed = 1;
         cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(d.n_kv_heads, p.n_batch, 1);
+        cfg.gridDim = dim3(p.n_vh, p.n_batch, 1);
         cfg.blockDim = dim3(kMergeThreads, 1, 1);
         cfg.stream = stream;
         cfg.attrs = &attr;

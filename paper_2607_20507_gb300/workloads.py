@@ -309,3 +309,109 @@ def route_inputs(w: RouteWorkload, device="cpu", seed: int | None = None) -> dic
     far = torch.randn(B, d, generator=g) / math.sqrt(d)
     emb = torch.where(hit[:, None], near, far) * (0.3 + 3.0 * torch.rand(B, 1, generator=g))
     return dict(emb=emb.to(torch.bfloat16).to(device), centroids=cent.to(torch.bfloat16).to(device))
+
+
+# --------------------------------------------------------------------------
+# token trees (multi-candidate verification): a static draft tree per
+# workload, the same shape for every request, nodes in breadth-first order
+# --------------------------------------------------------------------------
+
+@dataclasses.dataclass(frozen=True)
+class TreeWorkload:
+    """A draft tree of `branching[d]` children per node at depth d, verified in
+    one target pass; the attention geometry and logits of a serving workload."""
+
+    wid: int
+    name: str
+    batch: int
+    branching: tuple
+    vocab: int
+    logit_dtype: str
+    draft_sigma: float
+    temperatures: tuple
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    ctx: tuple
+    page_size: int
+    cell: int = 0
+
+    @property
+    def n_nodes(self) -> int:
+        return len(tree_parents(self.branching))
+
+    def chain_workload(self) -> Workload:
+        """A chain-workload view with n_draft = nodes - 1 (for the shared generators)."""
+        return Workload(self.wid, self.name, self.batch, self.n_nodes - 1, self.vocab, self.logit_dtype,
+                        self.draft_sigma, self.temperatures, self.n_q_heads, self.n_kv_heads, self.head_dim,
+                        self.ctx, self.page_size, cell=self.cell)
+
+
+def tree_parents(branching) -> list:
+    """Parent array of the tree with branching[d] children per node at depth d
+    (breadth-first order; node 0, the root, has parent -1)."""
+    parents = [-1]
+    level = [0]
+    for fan in branching:
+        nxt = []
+        for u in level:
+            for _ in range(int(fan)):
+                parents.append(u)
+                nxt.append(len(parents) - 1)
+        level = nxt
+    return parents
+
+
+TREE_WORKLOADS = {
+    # the attention geometry and logits of the B = 8 serving workload, with a
+    # 34-node tree (3, 2, 2, 1) in place of the 5-token chain
+    2: TreeWorkload(12, "tree-b8-n34-v128256-bf16-ctx1k-4k", batch=8, branching=(3, 2, 2, 1), vocab=128256,
+                    logit_dtype="bf16", draft_sigma=0.5, temperatures=(0.0, 0.7), n_q_heads=32, n_kv_heads=8,
+                    head_dim=128, ctx=("uniform", 1024, 4096), page_size=16),
+}
+
+
+def tree_attention_inputs(w: TreeWorkload, device="cpu") -> dict:
+    """q [B, n, Hq, D], paged K/V pools, page table, context lengths (counting the
+    n tree positions) and parents [B, n] int32 for a tree workload."""
+    inp = attention_inputs(w.chain_workload(), device)
+    par = torch.tensor(tree_parents(w.branching), dtype=torch.int32)
+    inp["parents"] = par.repeat(w.batch, 1).to(device)
+    inp.pop("n_draft")
+    return inp
+
+
+def tree_accept_inputs(w: TreeWorkload, temperature: float, device="cpu") -> dict:
+    """Target and draft logits [B, n, V] (target ~ N(0, 3^2), draft = target +
+    N(0, sigma^2), rounded to the logit dtype), node tokens [B, n] and uniforms
+    [B, n].  The children of a node are independent draws from the node's
+    draft distribution softmax(draft / T) (Gumbel-max); at T == 0 they are the
+    node's top draft tokens, best first."""
+    par = tree_parents(w.branching)
+    n, B, V = len(par), w.batch, w.vocab
+    dt = _logit_torch_dtype(w)
+    g_t = _gen(device, seed_of(w.chain_workload(), TAG_TARGET))
+    g_n = _gen(device, seed_of(w.chain_workload(), TAG_NOISE))
+    g_x = _gen(device, seed_of(w.chain_workload(), TAG_TOKENS))
+    target = (torch.randn((B, n, V), generator=g_t, device=device, dtype=torch.float32) * 3.0).to(dt)
+    zd = target.float() + w.draft_sigma * torch.randn((B, n, V), generator=g_n, device=device,
+                                                      dtype=torch.float32)
+    draft = zd.to(dt)
+    tokens = torch.zeros((B, n), dtype=torch.int32, device=device)
+    children = {}
+    for c in range(1, n):
+        children.setdefault(par[c], []).append(c)
+    for u, kids in children.items():
+        z = draft[:, u].float()
+        if temperature > 0:
+            uu = torch.rand((B, len(kids), V), generator=g_x, device=device, dtype=torch.float32)
+            uu.clamp_(min=1e-12, max=1.0 - 1e-7)
+            pick = torch.argmax(z[:, None, :] / temperature - uu.log_().neg_().log_(), dim=-1)
+        else:
+            pick = torch.topk(z, len(kids), dim=-1).indices
+        tokens[:, kids] = pick.to(torch.int32)
+    uniforms = torch.rand((B, n), generator=_gen(device, seed_of(w.chain_workload(), TAG_UNIFORM)),
+                          device=device, dtype=torch.float32)
+    return dict(target=target, draft=draft, parents=torch.tensor(par, dtype=torch.int32,
+                                                                 device=device).repeat(B, 1),
+                node_tokens=tokens, uniforms=uniforms)

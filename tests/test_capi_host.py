@@ -224,6 +224,71 @@ def test_route_argument_checks(lib):
     assert lib.cs_route_norms(0, 64, None, None, None) == binding.CS_OK
 
 
+def test_tree_argument_checks(lib):
+    d = good_attn_dims()
+
+    def tattn(dims=d, n=8, par=FAKE, ws=FAKE, ws_bytes=1 << 40, **kw):
+        return lib.cs_tree_verify_attention(ctypes.byref(dims), kw.get("q", FAKE), kw.get("kp", FAKE),
+                                            kw.get("vp", FAKE), kw.get("pt", FAKE), kw.get("cl", FAKE), par, n,
+                                            kw.get("out", FAKE), ws, ws_bytes, None)
+    for n in (0, -1, 65):
+        assert tattn(n=n) == binding.CS_ERR_INVALID_ARG
+        assert lib.cs_tree_verify_attention_workspace_bytes(ctypes.byref(d), n) == 0
+    for arg in ("q", "kp", "vp", "pt", "cl", "out"):
+        assert tattn(**{arg: None}) == binding.CS_ERR_INVALID_ARG
+    assert tattn(par=None) == binding.CS_ERR_INVALID_ARG
+    assert tattn(par=FAKE + 2) == binding.CS_ERR_INVALID_ARG
+    assert tattn(kp=FAKE + 8) == binding.CS_ERR_INVALID_ARG
+    bad = good_attn_dims()
+    bad.head_dim = 64
+    assert tattn(dims=bad) == binding.CS_ERR_UNSUPPORTED
+    # trees beyond 144 query rows per KV head are accepted (row blocks): G = 16, 64 nodes
+    wide = binding.AttnDims(2, 128, 8, 128, 16, 8, 64, 0.0)
+    need = lib.cs_tree_verify_attention_workspace_bytes(ctypes.byref(wide), 64)
+    assert need >= 256
+    assert tattn(dims=wide, n=64, ws=None) == binding.CS_ERR_WORKSPACE
+    assert tattn(dims=wide, n=64, ws_bytes=need - 1) == binding.CS_ERR_WORKSPACE
+    empty = good_attn_dims()
+    empty.batch = 0
+    assert tattn(dims=empty, par=None, ws=None, q=None, kp=None, vp=None, pt=None, cl=None, out=None) == binding.CS_OK
+
+    a = binding.AcceptDims(4, 32000, binding.CS_BF16)
+
+    def tacc(dims=a, n=8, T=1.0, ws=FAKE, ws_bytes=1 << 40, **kw):
+        return lib.cs_tree_accept(ctypes.byref(dims), kw.get("t", FAKE), kw.get("dd", FAKE), kw.get("par", FAKE),
+                                  kw.get("x", FAKE), kw.get("u", FAKE), n, T, kw.get("out", FAKE),
+                                  kw.get("path", FAKE), kw.get("na", FAKE), ws, ws_bytes, None)
+    for n in (0, 65):
+        assert tacc(n=n) == binding.CS_ERR_INVALID_ARG
+        assert lib.cs_tree_accept_workspace_bytes(ctypes.byref(a), n) == 0
+    for T in (-1.0, float("nan"), float("inf")):
+        assert tacc(T=T) == binding.CS_ERR_INVALID_ARG
+    for arg in ("t", "par", "x", "u", "out", "path", "na"):
+        assert tacc(**{arg: None}) == binding.CS_ERR_INVALID_ARG
+    assert tacc(dd=None) == binding.CS_ERR_INVALID_ARG            # sampling needs the draft rows
+    assert tacc(t=FAKE + 1) == binding.CS_ERR_INVALID_ARG
+    assert tacc(path=FAKE + 2) == binding.CS_ERR_INVALID_ARG
+    assert tacc(dims=binding.AcceptDims(2, (1 << 22) + 1, binding.CS_BF16)) == binding.CS_ERR_UNSUPPORTED
+    need = lib.cs_tree_accept_workspace_bytes(ctypes.byref(a), 8)
+    assert need >= 4 * 16 * 4                                     # at least a count per streamed row
+    assert tacc(ws=None) == binding.CS_ERR_WORKSPACE
+    assert tacc(ws_bytes=need - 1) == binding.CS_ERR_WORKSPACE
+    assert tacc(ws=FAKE + 64) == binding.CS_ERR_INVALID_ARG
+    assert tacc(dims=binding.AcceptDims(0, 100, binding.CS_F32), t=None, dd=None, par=None, x=None, u=None,
+                out=None, path=None, na=None, ws=None) == binding.CS_OK
+
+    def commit(dims=d, n=8, **kw):
+        return lib.cs_kv_commit_tree(ctypes.byref(dims), kw.get("kp", FAKE), kw.get("vp", FAKE), kw.get("pt", FAKE),
+                                     kw.get("cl", FAKE), kw.get("path", FAKE), kw.get("na", FAKE), n, None)
+    for arg in ("kp", "vp", "pt", "cl", "path", "na"):
+        assert commit(**{arg: None}) == binding.CS_ERR_INVALID_ARG
+    assert commit(n=0) == binding.CS_ERR_INVALID_ARG
+    assert commit(n=65) == binding.CS_ERR_INVALID_ARG
+    assert commit(vp=FAKE + 4) == binding.CS_ERR_INVALID_ARG
+    assert commit(dims=bad) == binding.CS_ERR_UNSUPPORTED
+    assert commit(dims=empty, kp=None, vp=None, pt=None, cl=None, path=None, na=None) == binding.CS_OK
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     with pytest.raises(RuntimeError, match="not found"):
         binding.load_library(str(tmp_path / "missing.so"))
