@@ -377,6 +377,32 @@ def run_gb300(args) -> dict | None:
             "us": 1e6 * t_rt, "tflops": flops / t_rt / 1e12, "flops": flops, "bytes": r_bytes,
             "hit_rate": float((r_out[0] >= 0).float().mean().item())}
         del rx, r_inv, r_out
+    # token-tree verification at the same attention geometry and vocabulary:
+    # tree attention over the paged cache and the acceptance walk
+    tw = W.TREE_WORKLOADS[2]
+    ta = W.tree_attention_inputs(tw, dev)
+    t_out = torch.empty_like(ta["q"])
+    t_tat = timed_graph(lambda: binding.cs_tree_verify_attention(ta["q"], ta["k_pages"], ta["v_pages"],
+                                                                 ta["page_table"], ta["ctx_lens"], ta["parents"],
+                                                                 out=t_out))
+    tlens = ta["ctx_lens"].cpu().numpy()
+    tat_bytes = attention_bytes(tlens, tw.chain_workload())
+    T_tree = max(tw.temperatures)
+    tc = W.tree_accept_inputs(tw, T_tree, dev)
+    t_bufs = [torch.empty((tw.batch, tw.n_nodes), dtype=torch.int32, device=dev) for _ in range(2)]
+    t_na = torch.empty((tw.batch,), dtype=torch.int32, device=dev)
+    t_tac = timed_graph(lambda: binding.cs_tree_accept(tc["target"], tc["draft"], tc["parents"], tc["node_tokens"],
+                                                       tc["uniforms"], T_tree, *t_bufs, t_na))
+    par = W.tree_parents(tw.branching)
+    internal = len(set(u for u in par[1:]))
+    s_log = 4 if tw.logit_dtype == "f32" else 2
+    tac_bytes = tw.batch * (tw.n_nodes + internal) * tw.vocab * s_log
+    next_rows[f"tree_{tw.name}"] = {
+        "nodes": tw.n_nodes, "branching": list(tw.branching), "temperature": T_tree,
+        "attention_us": 1e6 * t_tat, "attention_bytes": tat_bytes, "attention_gbs": tat_bytes / t_tat / 1e9,
+        "accept_us": 1e6 * t_tac, "accept_bytes": tac_bytes, "accept_gbs": tac_bytes / t_tac / 1e9,
+        "mean_accepted": float(t_na.float().mean().item())}
+    del ta, tc, t_out, t_bufs
 
     # end to end through the public API: inputs start in pinned host memory
     host = {name: t.cpu().pin_memory() for name, t in

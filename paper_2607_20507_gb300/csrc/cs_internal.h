@@ -25,7 +25,8 @@ struct AttnPlan {
     int n_rows_all;   // rows * G query rows per KV head
     int n_rb;         // row blocks per KV head (each one span of the schedule)
     int n_rows;       // query rows per row block (n_rows_all when n_rb == 1)
-    int row_warps;    // ceil(n_rows / 16) consumer warps
+    int row_warps;    // ceil(n_rows / 16) warps of query rows
+    int split;        // consumer groups sharing each tile's keys (1 or 2)
     int grid;         // persistent CTAs (resident capacity of the device)
     size_t off_part_o, off_part_ml, bytes;   // workspace layout (status word at 0)
 };

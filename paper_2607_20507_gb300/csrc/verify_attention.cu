@@ -21,10 +21,20 @@
 // query rows exceed what one CTA holds is cut into row blocks, each its own
 // span ("virtual head") over the same keys.
 //
+// With few query rows (at most 32 per KV head) every 64-key tile is split
+// between two consumer warp groups, each running its own online softmax over
+// 32 of the keys; the two states of a row are folded in shared memory when a
+// span piece ends.  Twice the warps then hide the latency of the mma.sync
+// chains, which otherwise pace the tile rate.
+//
 // Per CTA: one producer warp streams the K and V tiles of its range through
-// TMA (one 4-D tensor map over the page pool, 128-byte swizzle, one box per
-// page piece) into a 3-stage shared-memory ring guarded by mbarriers, without
-// draining between spans.  Consumer warps own 16 of the (k+1)*G query rows of
+// TMA into a 3-stage shared-memory ring guarded by mbarriers, without
+// draining between spans.  One 5-D tensor map covers each page pool as
+// (64 dims, keys, 2 dim halves, heads, pages): a box is both 128-byte halves
+// of up to 64 keys of one page and head, landing as [half][key][64 dims]
+// with the 128-byte swizzle, so a 16-token page is one 4 KB copy.  The page
+// ids of the next 32 / pieces tiles come from one warp-wide load issued a
+// batch ahead, and the page table is prefetched into L2 at launch.  Consumer warps own 16 of the (k+1)*G query rows of
 // the current span each (draft row i = r / G, query head h*G + r % G), so
 // every K/V byte staged in shared memory serves all rows; they run S = Q K^T
 // and O += P V on bf16 tensor cores (mma.sync m16n8k16, fp32 accumulate) with
@@ -42,11 +52,11 @@ namespace {
 
 constexpr int kD = 128;                       // head dim implemented
 constexpr int kTileT = 64;                    // keys per pipeline tile
-constexpr int kHalfBytes = kTileT * 128;      // 64 keys x 64 dims x 2 B (one swizzle half)
-constexpr int kTensorTileBytes = 2 * kHalfBytes;
+constexpr int kTensorTileBytes = kTileT * 256; // 64 keys x 128 dims x 2 B
 constexpr int kStageBytes = 2 * kTensorTileBytes;   // K + V
 constexpr int kStages = 3;
 constexpr int kMaxRowWarps = 9;               // 144 query rows
+constexpr int kMaxSplitRowWarps = 2;          // key-split consumers: up to 32 query rows
 constexpr int kMaxBatchPerLaunch = 1024;      // requests whose schedule one launch holds
 constexpr int kMaxGrid = 512;                 // persistent CTAs at most (slot list size)
 constexpr int kMinTilesPerCta = 8;            // 256 KB of K/V per CTA before a span is cut
@@ -149,8 +159,11 @@ __device__ __forceinline__ void tree_ancestor_masks(const int32_t* par, int n, i
     }
 }
 
-template <bool kTree>
-__global__ void __launch_bounds__((kMaxRowWarps + 1) * 32, 1)
+// kSplit: consumer warp groups that share each tile (1, or 2 when the query
+// rows fit two row warps: each group takes 32 of the tile's 64 keys)
+template <bool kTree, int kBoxT, int kSplit>
+__global__ void __launch_bounds__(kSplit == 1 ? (kMaxRowWarps + 1) * 32 : (2 * kMaxSplitRowWarps + 1) * 32,
+                                  kSplit == 1 ? 1 : 2)
 verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                         const __grid_constant__ CUtensorMap tmap_v, const AttnParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -158,6 +171,8 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
     uint64_t* empty = full + kStages;
+    uint64_t* fold_a = empty + kStages;   // key-split: every consumer is done with the stage
+    uint64_t* fold_b = fold_a + 1;        // key-split: the second group's state is in the stage
     long long* s_prefix = reinterpret_cast<long long*>(smem + kStages * kStageBytes + kBarrierBytes);
     int* s_len = reinterpret_cast<int*>(s_prefix + kMaxBatchPerLaunch + 1);
     __shared__ long long s_wtot[kMaxRowWarps + 1];
@@ -170,13 +185,24 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     // its schedule) while this kernel runs
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
+    // the page table of this launch into L2, spread over the CTAs, while the
+    // schedule is computed (the producer's first lookups then hit L2)
+    if (warp == kSplit * nw) {
+        const char* tab = reinterpret_cast<const char*>(p.page_table + (size_t)p.b_base * p.max_pages);
+        const long long lines = ((long long)nb * p.max_pages * 4 + 127) / 128;
+        for (long long i = (long long)blockIdx.x * 32 + lane; i < lines; i += (long long)gridDim.x * 32)
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(tab + i * 128));
+    }
+
     // ---- schedule: exclusive prefix of tiles per request (x heads), clamped L
     if (threadIdx.x == 0) {
         s_carry = 0;
         for (int i = 0; i < kStages; ++i) {
             mbar_init(&full[i], 1);
-            mbar_init(&empty[i], nw);
+            mbar_init(&empty[i], kSplit * nw);
         }
+        mbar_init(fold_a, kSplit * nw);
+        mbar_init(fold_b, nw);
         fence_barrier_init();
     }
     __syncthreads();
@@ -220,7 +246,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const int n_tiles = (int)(f1 - f0);
     const uint32_t smem_base = smem_u32(smem);
 
-    if (warp == nw) {
+    if (warp == kSplit * nw) {
         // ------------------------------------------------------ producer
         // The whole warp produces: lane pc owns page piece pc of a tile (its
         // page id is loaded one tile ahead, so the table lookups of all pieces
@@ -230,24 +256,34 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             tma_prefetch_desc(&tmap_k);
             tma_prefetch_desc(&tmap_v);
         }
-        const int pieces = kTileT / p.box_t;
-        const uint32_t piece_bytes = (uint32_t)p.box_t * 128u;
-        Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
-        auto piece_page = [&](const Cursor& cc) -> int {
-            const int tok = cc.t * kTileT + lane * p.box_t;
-            if (lane >= pieces || tok >= s_len[cc.b]) return -1;
+        constexpr int pieces = kTileT / kBoxT;
+        constexpr uint32_t piece_bytes = (uint32_t)kBoxT * 256u;   // both dim halves of kBoxT keys
+        constexpr int per_batch = 32 / pieces;   // tiles whose page ids one warp-wide load covers
+        // lane l: the page of piece l % pieces of tile j0 + l / pieces
+        auto batch_pages = [&](int j0) -> int {
+            const int jj = j0 + lane / pieces;
+            if (jj >= n_tiles) return -1;
+            const Cursor cc = locate(f0 + jj, s_prefix, s_len, nb, p.n_vh);
+            const int tok = cc.t * kTileT + (lane % pieces) * kBoxT;
+            if (tok >= s_len[cc.b]) return -1;
             return __ldg(p.page_table + (size_t)(p.b_base + cc.b) * p.max_pages + tok / p.ps);
         };
-        int page_next = piece_page(cur);
+        Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
+        int pg_cur = batch_pages(0);
+        int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
         for (int j = 0; j < n_tiles; ++j) {
             const int st = j % kStages;
             const uint32_t use = (uint32_t)(j / kStages);
-            const int page = page_next;
+            const int jb = j % per_batch;
+            if (j > 0 && jb == 0) {
+                pg_cur = pg_next;
+                pg_next = j + per_batch < n_tiles ? batch_pages(j + per_batch) : -1;
+            }
+            const int page = __shfl_sync(0xffffffffu, pg_cur, jb * pieces + lane % pieces);
             const int L = s_len[cur.b];
             const int ts = cur.t * kTileT;
             const int h_cur = cur.h / p.n_rb;   // the KV head of this span
             advance(cur, s_len, nb, p.n_vh);
-            if (j + 1 < n_tiles) page_next = piece_page(cur);
             int ok = 1;
             if (lane == 0 && j >= kStages && !mbar_wait_bounded(&empty[st], (use - 1) & 1)) {
                 flag_timeout(p.status);
@@ -256,32 +292,36 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             if (!__shfl_sync(0xffffffffu, ok, 0)) break;
             int valid = 0;
             for (int pc = 0; pc < pieces; ++pc)
-                if (ts + pc * p.box_t < L) ++valid;
-            if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)valid * piece_bytes * 4u);
+                if (ts + pc * kBoxT < L) ++valid;
+            if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)valid * piece_bytes * 2u);
             __syncwarp();
             if (lane < valid) {
                 const uint32_t kdst = smem_base + st * kStageBytes + (uint32_t)lane * piece_bytes;
                 const uint32_t vdst = kdst + kTensorTileBytes;
-                const int slot = (ts + lane * p.box_t) % p.ps;
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    tma_load_4d(kdst + hh * kHalfBytes, &tmap_k, &full[st], hh * 64, slot, h_cur, page);
-                    tma_load_4d(vdst + hh * kHalfBytes, &tmap_v, &full[st], hh * 64, slot, h_cur, page);
-                }
+                const int slot = (ts + lane * kBoxT) % p.ps;
+                tma_load_5d(kdst, &tmap_k, &full[st], 0, slot, 0, h_cur, page);
+                tma_load_5d(vdst, &tmap_v, &full[st], 0, slot, 0, h_cur, page);
             }
         }
         return;
     }
 
     // ---------------------------------------------------------- consumers
+    // 128-byte row of (key, dim half) in a K or V tile: pieces of box_t keys,
+    // each [half][key][64 dims]
+    auto key_row = [](int key, int half) { return key + (key & ~(kBoxT - 1)) + half * kBoxT; };
+    constexpr int kNT = 8 / kSplit;        // 8-key n-tiles of a warp's share of a tile
+    const int kh = kSplit == 1 ? 0 : warp / nw;   // key share: keys [kh*64/kSplit, (kh+1)*64/kSplit) of a tile
+    const int rw = warp - kh * nw;         // row warp: query rows [16 rw, 16 rw + 16)
     const int g = lane >> 2, tq = lane & 3;
-    const int row0 = warp * 16 + g, row1 = row0 + 8;
+    const int row0 = rw * 16 + g, row1 = row0 + 8;
     const int lm = lane >> 3, lr = lane & 7;   // ldmatrix: matrix index, row within it
     const float c = p.scale_log2;
 
     Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
     int seg_t0 = cur.t;
     bool first_seg = true;
+    int folds = 0;
 
     uint32_t qa[8][4];
     float o[16][4];
@@ -355,25 +395,25 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             uint8_t* vrow = smem + st * kStageBytes + kTensorTileBytes;
             for (int idx = lane; idx < (kTileT - first) * 16; idx += 32) {
                 const int r = first + (idx >> 4), ch = idx & 15;
-                *reinterpret_cast<uint4*>(vrow + (ch >> 3) * kHalfBytes + r * 128 + (ch & 7) * 16) =
+                *reinterpret_cast<uint4*>(vrow + key_row(r, ch >> 3) * 128 + (ch & 7) * 16) =
                     make_uint4(0, 0, 0, 0);
             }
             __syncwarp();
         }
 
-        // ---- S = Q K^T over 64 keys: 8 n-tiles of 8 keys
-        float sc[8][4];
+        // ---- S = Q K^T over this warp's keys: kNT n-tiles of 8 keys
+        float sc[kNT][4];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
+        for (int i = 0; i < kNT; ++i) sc[i][0] = sc[i][1] = sc[i][2] = sc[i][3] = 0.f;
+        const int key0 = kh * (kTileT / kSplit);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t half = kb + (kk >> 2) * kHalfBytes;
 #pragma unroll
-            for (int np = 0; np < 4; ++np) {
-                const int key = (2 * np + (lm >> 1)) * 8 + lr;
+            for (int np = 0; np < kNT / 2; ++np) {
+                const int key = key0 + (2 * np + (lm >> 1)) * 8 + lr;
                 const int ch = (kk & 3) * 2 + (lm & 1);
                 uint32_t b0, b1, b2, b3;
-                ldsm_x4(half + key * 128 + ((ch ^ (key & 7)) << 4), b0, b1, b2, b3);
+                ldsm_x4(kb + key_row(key, kk >> 2) * 128 + ((ch ^ (key & 7)) << 4), b0, b1, b2, b3);
                 mma_bf16_16816(sc[2 * np], qa[kk], b0, b1);
                 mma_bf16_16816(sc[2 * np + 1], qa[kk], b2, b3);
             }
@@ -391,9 +431,9 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                 const uint64_t live = span_L - ts >= 64 ? ~0ull : (1ull << max(span_L - ts, 0)) - 1ull;
                 const uint64_t t0 = d >= 64 ? 0ull : (d >= 0 ? anc0 >> d : (d <= -64 ? 0ull : anc0 << -d));
                 const uint64_t t1 = d >= 64 ? 0ull : (d >= 0 ? anc1 >> d : (d <= -64 ? 0ull : anc1 << -d));
-                const uint64_t v0 = ((pre | t0) & live) >> (tq * 2), v1 = ((pre | t1) & live) >> (tq * 2);
+                const uint64_t v0 = ((pre | t0) & live) >> (key0 + tq * 2), v1 = ((pre | t1) & live) >> (key0 + tq * 2);
 #pragma unroll
-                for (int nt = 0; nt < 8; ++nt) {
+                for (int nt = 0; nt < kNT; ++nt) {
 #pragma unroll
                     for (int e = 0; e < 2; ++e) {
                         if (!((v0 >> (nt * 8 + e)) & 1ull)) sc[nt][e] = kNegInf;
@@ -403,10 +443,10 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             }
         } else if (ts + kTileT > min(lim0, lim1)) {
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
+            for (int nt = 0; nt < kNT; ++nt) {
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
-                    const int key = ts + nt * 8 + tq * 2 + e;
+                    const int key = ts + key0 + nt * 8 + tq * 2 + e;
                     if (key >= lim0) sc[nt][e] = kNegInf;
                     if (key >= lim1) sc[nt][2 + e] = kNegInf;
                 }
@@ -417,7 +457,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         for (int rh = 0; rh < 2; ++rh) {
             float mx = kNegInf;
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) mx = fmaxf(mx, fmaxf(sc[nt][2 * rh], sc[nt][2 * rh + 1]));
+            for (int nt = 0; nt < kNT; ++nt) mx = fmaxf(mx, fmaxf(sc[nt][2 * rh], sc[nt][2 * rh + 1]));
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
             const float m_new = fmaxf(m_raw[rh], mx);
@@ -427,7 +467,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             const float neg = -m_use * c;
             float rs = 0.f;
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
+            for (int nt = 0; nt < kNT; ++nt) {
                 const float p0 = ex2(fmaf(sc[nt][2 * rh], c, neg));
                 const float p1 = ex2(fmaf(sc[nt][2 * rh + 1], c, neg));
                 sc[nt][2 * rh] = p0;
@@ -441,39 +481,96 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                 o[dn][2 * rh + 1] *= alpha;
             }
         }
-        // ---- O += P V over the 64 keys: 4 k-steps of 16 keys
+        // ---- O += P V over this warp's keys: k-steps of 16 keys
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
+        for (int kk = 0; kk < kNT / 2; ++kk) {
             uint32_t a[4];
             a[0] = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
             a[1] = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
             a[2] = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
             a[3] = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
-            const int key = kk * 16 + (lm & 1) * 8 + lr;
+            const int key = key0 + kk * 16 + (lm & 1) * 8 + lr;
 #pragma unroll
             for (int dp = 0; dp < 8; ++dp) {
                 const int dblk = 2 * dp + (lm >> 1);
                 const int ch = dblk & 7;
                 uint32_t b0, b1, b2, b3;
-                ldsm_x4_trans(vb + (dblk >> 3) * kHalfBytes + key * 128 + ((ch ^ (key & 7)) << 4), b0,
+                ldsm_x4_trans(vb + key_row(key, dblk >> 3) * 128 + ((ch ^ (key & 7)) << 4), b0,
                               b1, b2, b3);
                 mma_bf16_16816(o[2 * dp], a, b0, b1);
                 mma_bf16_16816(o[2 * dp + 1], a, b2, b3);
             }
         }
-        // generic-proxy writes (the zeroed rows) must be ordered before the
-        // next TMA write into this stage
-        if (ts + kTileT > L) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        const bool piece_end = !(j + 1 < n_tiles && cur.t + 1 < cur.T);
+        if (kSplit > 1 && piece_end) {
+            // fold the two key shares of every row: once every consumer is
+            // done with this stage (fold_a), the second group leaves its
+            // (O, m, l) in it (fold_b) and the first group folds them into
+            // its own.  Both waits are bounded.
+            const uint32_t ph = (uint32_t)(folds++ & 1);
+            float* scr = reinterpret_cast<float*>(smem + st * kStageBytes) + rw * (64 * 32 + 4 * 32);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(fold_a);
+            if (kh == 1) {
+                if (!mbar_wait_bounded(fold_a, ph)) {
+                    flag_timeout(p.status);
+                    break;
+                }
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    reinterpret_cast<float4*>(scr)[i * 32 + lane] = make_float4(o[i][0], o[i][1], o[i][2], o[i][3]);
+                reinterpret_cast<float4*>(scr + 64 * 32)[lane] = make_float4(m_raw[0], m_raw[1], l[0], l[1]);
+                __syncwarp();
+                if (lane == 0) mbar_arrive(fold_b);
+            } else {
+                if (!mbar_wait_bounded(fold_b, ph)) {
+                    flag_timeout(p.status);
+                    break;
+                }
+                const float4 ml = reinterpret_cast<const float4*>(scr + 64 * 32)[lane];
+                const float mo[2] = {ml.x, ml.y}, lo[2] = {ml.z, ml.w};
+                float a_s[2], a_o[2];
+#pragma unroll
+                for (int rh = 0; rh < 2; ++rh) {
+                    const float mn = fmaxf(m_raw[rh], mo[rh]);
+                    const float mu = mn == kNegInf ? 0.f : mn;
+                    a_s[rh] = ex2((m_raw[rh] - mu) * c);
+                    a_o[rh] = ex2((mo[rh] - mu) * c);
+                    l[rh] = l[rh] * a_s[rh] + lo[rh] * a_o[rh];
+                    m_raw[rh] = mn;
+                }
+#pragma unroll
+                for (int i = 0; i < 16; ++i) {
+                    const float4 v = reinterpret_cast<const float4*>(scr)[i * 32 + lane];
+                    o[i][0] = o[i][0] * a_s[0] + v.x * a_o[0];
+                    o[i][1] = o[i][1] * a_s[0] + v.y * a_o[0];
+                    o[i][2] = o[i][2] * a_s[1] + v.z * a_o[1];
+                    o[i][3] = o[i][3] * a_s[1] + v.w * a_o[1];
+                }
+            }
+        }
+        // generic-proxy writes (zeroed rows, the fold's scratch) must be
+        // ordered before the next TMA write into this stage
+        if (ts + kTileT > L || (kSplit > 1 && piece_end)) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[st]);
 
-        if (j + 1 < n_tiles && cur.t + 1 < cur.T) {
+        if (!piece_end) {
             advance(cur, s_len, nb, p.n_vh);
             continue;
         }
 
         // ---------------------------------------------- end of a piece of span
         const int bg = p.b_base + cur.b;
+        if (kSplit > 1 && kh == 1) {   // folded into the first group's state
+            if (j + 1 < n_tiles) {
+                advance(cur, s_len, nb, p.n_vh);
+                seg_t0 = cur.t;
+                first_seg = false;
+                begin_span(cur);
+            }
+            continue;
+        }
         const bool complete = seg_t0 == 0 && cur.t + 1 == cur.T;
         float lt[2];
 #pragma unroll
@@ -525,10 +622,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 // from the context lengths, so it knows which CTAs cut its span (b, h) and in
 // which slots their pieces are; a span with a single piece was written by the
 // main kernel and is skipped.  The pieces are folded with log-sum-exp weights:
-// one warp per query row, lanes across the 128 dims (one coalesced 512-byte
+// one warp per query row (a CTA holds 8 rows of one span, so all rows of a
+// span merge at once), lanes across the 128 dims (one coalesced 512-byte
 // read per piece), every piece's loads issued before any is used.
 // ---------------------------------------------------------------------------
 constexpr int kMergeThreads = 256;
+constexpr int kMergeRows = kMergeThreads / 32;   // query rows per merge CTA
 constexpr int kMergePieces = 8;   // pieces in flight per row
 
 __global__ void __launch_bounds__(kMergeThreads)
@@ -592,7 +691,8 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
 
     const int bg = p.b_base + bl;
     const int head = h / p.n_rb, rbase = (h - head * p.n_rb) * p.n_rows;
-    for (int row = warp; row < p.n_rows && rbase + row < p.n_rows_all; row += kMergeThreads / 32) {
+    const int row = blockIdx.z * kMergeRows + warp;
+    if (row < p.n_rows && rbase + row < p.n_rows_all) {
         float M = kNegInf, lsum = 0.f;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
         for (int q0 = 0; q0 < n_p; q0 += kMergePieces) {
@@ -654,13 +754,15 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims& d, int box_t) {
     auto enc = tensor_map_encoder();
     if (!enc) return fail(CS_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
-    const cuuint64_t dims[4] = {(cuuint64_t)d.head_dim, (cuuint64_t)d.page_size,
-                                (cuuint64_t)d.n_kv_heads, (cuuint64_t)d.num_pages};
+    // (64 dims, keys, 2 dim halves, heads, pages): one box holds both halves
+    // of box_t keys, half-major, so it lands as [half][key][64 dims]
+    const cuuint64_t dims[5] = {64, (cuuint64_t)d.page_size, 2, (cuuint64_t)d.n_kv_heads,
+                                (cuuint64_t)d.num_pages};
     const cuuint64_t row = (cuuint64_t)d.head_dim * 2;
-    const cuuint64_t strides[3] = {row, row * d.page_size, row * d.page_size * d.n_kv_heads};
-    const cuuint32_t box[4] = {64, (cuuint32_t)box_t, 1, 1};
-    const cuuint32_t estr[4] = {1, 1, 1, 1};
-    const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(pool), dims,
+    const cuuint64_t strides[4] = {row, 128, row * d.page_size, row * d.page_size * d.n_kv_heads};
+    const cuuint32_t box[5] = {64, (cuuint32_t)box_t, 2, 1, 1};
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(pool), dims,
                            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -671,8 +773,9 @@ cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Resident CTAs per SM of the kernel at a given block size (cached per device).
-template <bool kTree>
+template <bool kTree, int kSplit>
 int resident_per_sm(int threads) {
+    // every box size instantiates the same code shape; the 16-key one stands for all
     static int cache[64][kMaxRowWarps + 2] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
@@ -683,9 +786,9 @@ int resident_per_sm(int threads) {
     if (key <= 0 || key > kMaxRowWarps + 1) return 1;
     if (!cache[dev][key]) {
         int n = 0;
-        if (cudaFuncSetAttribute(verify_attention_kernel<kTree>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kSmemBytes) != cudaSuccess ||
-            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, verify_attention_kernel<kTree>, threads,
+        if (cudaFuncSetAttribute(verify_attention_kernel<kTree, 16, kSplit>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, verify_attention_kernel<kTree, 16, kSplit>, threads,
                                                           kSmemBytes) != cudaSuccess ||
             n <= 0) {
             cudaGetLastError();
@@ -710,9 +813,13 @@ AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count
     pl.n_rb = (pl.n_rows_all + cap - 1) / cap;
     pl.n_rows = pl.n_rb == 1 ? pl.n_rows_all : ((pl.n_rows_all + pl.n_rb - 1) / pl.n_rb + 15) / 16 * 16;
     pl.row_warps = (pl.n_rows + 15) / 16;
+    // few rows: two consumer groups share each tile's keys
+    pl.split = pl.row_warps <= kMaxSplitRowWarps ? 2 : 1;
     // persistent grid: exactly the CTAs that are resident at once
-    const int threads = (pl.row_warps + 1) * 32;
-    pl.grid = (sm_count > 0 ? sm_count : 148) * (tree ? resident_per_sm<true>(threads) : resident_per_sm<false>(threads));
+    const int threads = (pl.split * pl.row_warps + 1) * 32;
+    const int res = pl.split == 2 ? (tree ? resident_per_sm<true, 2>(threads) : resident_per_sm<false, 2>(threads))
+                                  : (tree ? resident_per_sm<true, 1>(threads) : resident_per_sm<false, 1>(threads));
+    pl.grid = (sm_count > 0 ? sm_count : 148) * res;
     if (pl.grid > kMaxGrid) pl.grid = kMaxGrid;
     size_t off = 256;   // status word lives at offset 0
     pl.off_part_ml = off;
@@ -770,20 +877,33 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     const float scale = d.sm_scale > 0.f ? d.sm_scale : 1.0f / sqrtf((float)d.head_dim);
     p.scale_log2 = scale * 1.4426950408889634f;
 
-    auto kern = pl.tree ? verify_attention_kernel<true> : verify_attention_kernel<false>;
+    // kernels by (key split, tree, box size 8/16/32/64 keys)
+    using Kern = void (*)(const CUtensorMap, const CUtensorMap, const AttnParams);
+    static const Kern kerns[2][2][4] = {
+        {{verify_attention_kernel<false, 8, 1>, verify_attention_kernel<false, 16, 1>,
+          verify_attention_kernel<false, 32, 1>, verify_attention_kernel<false, 64, 1>},
+         {verify_attention_kernel<true, 8, 1>, verify_attention_kernel<true, 16, 1>,
+          verify_attention_kernel<true, 32, 1>, verify_attention_kernel<true, 64, 1>}},
+        {{verify_attention_kernel<false, 8, 2>, verify_attention_kernel<false, 16, 2>,
+          verify_attention_kernel<false, 32, 2>, verify_attention_kernel<false, 64, 2>},
+         {verify_attention_kernel<true, 8, 2>, verify_attention_kernel<true, 16, 2>,
+          verify_attention_kernel<true, 32, 2>, verify_attention_kernel<true, 64, 2>}}};
+    const int bi = box_t == 8 ? 0 : box_t == 16 ? 1 : box_t == 32 ? 2 : 3;
+    const int si = pl.split == 2 ? 1 : 0;
+    const Kern kern = kerns[si][pl.tree][bi];
     cudaError_t e = cudaSuccess;
     {
-        static bool attr_done[2][64] = {};
+        static bool attr_done[2][2][4][64] = {};
         int dev = 0;
         e = cudaGetDevice(&dev);
         if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-        if (dev < 0 || dev >= 64 || !attr_done[pl.tree][dev]) {
+        if (dev < 0 || dev >= 64 || !attr_done[si][pl.tree][bi][dev]) {
             e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
             if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_attention_kernel)");
-            if (dev >= 0 && dev < 64) attr_done[pl.tree][dev] = true;
+            if (dev >= 0 && dev < 64) attr_done[si][pl.tree][bi][dev] = true;
         }
     }
-    const dim3 block((pl.row_warps + 1) * 32);
+    const dim3 block((pl.split * pl.row_warps + 1) * 32);
     for (int b0 = 0; b0 < d.batch; b0 += kMaxBatchPerLaunch) {
         p.b_base = b0;
         p.n_batch = d.batch - b0 < kMaxBatchPerLaunch ? d.batch - b0 : kMaxBatchPerLaunch;
@@ -796,7 +916,7 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
         attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr.val.programmaticStreamSerializationAllowed = 1;
         cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(p.n_vh, p.n_batch, 1);
+        cfg.gridDim = dim3(p.n_vh, p.n_batch, (pl.n_rows + kMergeRows - 1) / kMergeRows);
         cfg.blockDim = dim3(kMergeThreads, 1, 1);
         cfg.stream = stream;
         cfg.attrs = &attr;
