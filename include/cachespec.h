@@ -132,7 +132,10 @@ const char* cs_last_error(void);
  * [0, max_pages_per_seq*ps]; a row with no admissible key
  * (L_b-(k+1)+i < 0) outputs zeros; a page id outside [0, P) reads as zeros.
  * Pool slots past L_b may hold any bits (including NaN); they never reach
- * the output.
+ * the output.  Arithmetic: S = q.K in bf16 with fp32 accumulation, the
+ * softmax in fp32, and the P.V product in fp16 with fp32 accumulation (P
+ * rounded to fp16; V converted from bf16, exact for |v| < 65520 -- larger
+ * V entries overflow there).
  *
  * Returns CS_ERR_INVALID_ARG (null pointer, misalignment, bad dimension, NaN
  * scale, n_draft out of range), CS_ERR_UNSUPPORTED (D != 128, page size,

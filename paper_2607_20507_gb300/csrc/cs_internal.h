@@ -27,6 +27,7 @@ struct AttnPlan {
     int n_rows;       // query rows per row block (n_rows_all when n_rb == 1)
     int row_warps;    // ceil(n_rows / 16) warps of query rows
     int split;        // consumer groups sharing each tile's keys (1 or 2)
+    bool tc;          // the tcgen05 kernel (33..128 rows, one row block)
     int grid;         // persistent CTAs (resident capacity of the device)
     size_t off_part_o, off_part_ml, bytes;   // workspace layout (status word at 0)
 };

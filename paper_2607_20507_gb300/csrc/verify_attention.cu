@@ -37,8 +37,12 @@
 // batch ahead, and the page table is prefetched into L2 at launch.  Consumer warps own 16 of the (k+1)*G query rows of
 // the current span each (draft row i = r / G, query head h*G + r % G), so
 // every K/V byte staged in shared memory serves all rows; they run S = Q K^T
-// and O += P V on bf16 tensor cores (mma.sync m16n8k16, fp32 accumulate) with
-// an fp32 online softmax in the log2 domain.
+// on bf16 tensor cores and O += P V on fp16 ones (mma.sync m16n8k16, fp32
+// accumulate; P rounded to fp16, V fragments converted from bf16, which is
+// exact for values inside fp16's range) with an fp32 online softmax in the
+// log2 domain.  fp16 P is eight times finer than bf16: with bf16 P the
+// rounding of the weights alone can exceed 2e-3 + 1e-2|o| on rows whose
+// terms cancel.
 #include <math.h>
 #include <stdio.h>
 
@@ -78,6 +82,7 @@ struct AttnParams {
     int n_rb;                    // row blocks per KV head (n_rows rows each)
     int n_vh;                    // Hkv * n_rb spans per request ("virtual heads")
     int n_rows_all;              // R * G query rows per KV head
+    int tc_stages, tc_q_half;    // tcgen05 kernel: K/V ring depth, bytes between query dim halves
     int b_base, n_batch;         // requests [b_base, b_base + n_batch) in this launch
     float scale_log2;            // sm_scale * log2(e)
 };
@@ -485,10 +490,10 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 #pragma unroll
         for (int kk = 0; kk < kNT / 2; ++kk) {
             uint32_t a[4];
-            a[0] = pack_bf16x2(sc[2 * kk][0], sc[2 * kk][1]);
-            a[1] = pack_bf16x2(sc[2 * kk][2], sc[2 * kk][3]);
-            a[2] = pack_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-            a[3] = pack_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+            a[0] = pack_f16x2(sc[2 * kk][0], sc[2 * kk][1]);
+            a[1] = pack_f16x2(sc[2 * kk][2], sc[2 * kk][3]);
+            a[2] = pack_f16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
+            a[3] = pack_f16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
             const int key = key0 + kk * 16 + (lm & 1) * 8 + lr;
 #pragma unroll
             for (int dp = 0; dp < 8; ++dp) {
@@ -497,8 +502,8 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                 uint32_t b0, b1, b2, b3;
                 ldsm_x4_trans(vb + key_row(key, dblk >> 3) * 128 + ((ch ^ (key & 7)) << 4), b0,
                               b1, b2, b3);
-                mma_bf16_16816(o[2 * dp], a, b0, b1);
-                mma_bf16_16816(o[2 * dp + 1], a, b2, b3);
+                mma_f16_16816(o[2 * dp], a, bf16x2_to_f16x2(b0), bf16x2_to_f16x2(b1));
+                mma_f16_16816(o[2 * dp + 1], a, bf16x2_to_f16x2(b2), bf16x2_to_f16x2(b3));
             }
         }
         const bool piece_end = !(j + 1 < n_tiles && cur.t + 1 < cur.T);
@@ -738,6 +743,8 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     }
 }
 
+#include "verify_attention_tc.cuh"
+
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
@@ -751,7 +758,9 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
     return fn;
 }
 
-cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims& d, int box_t) {
+// halves: dim halves per box (2: [half][keys][64 dims] per page piece; 1: one
+// half per box, for tiles laid out [half][64 keys][64 dims])
+cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims& d, int box_t, int halves = 2) {
     auto enc = tensor_map_encoder();
     if (!enc) return fail(CS_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
     // (64 dims, keys, 2 dim halves, heads, pages): one box holds both halves
@@ -760,7 +769,7 @@ cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims
                                 (cuuint64_t)d.num_pages};
     const cuuint64_t row = (cuuint64_t)d.head_dim * 2;
     const cuuint64_t strides[4] = {row, 128, row * d.page_size, row * d.page_size * d.n_kv_heads};
-    const cuuint32_t box[5] = {64, (cuuint32_t)box_t, 2, 1, 1};
+    const cuuint32_t box[5] = {64, (cuuint32_t)box_t, (cuuint32_t)halves, 1, 1};
     const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
     const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(pool), dims,
                            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
@@ -770,7 +779,62 @@ cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims
     return CS_OK;
 }
 
+// The query rows of one KV head of one request as one box per dim half: q
+// [B, R, Hq, D] seen as (D, Hq, R, B), box (64, G, R, 1), landing as
+// [draft row][group head][64 dims] = query row i*G + g.
+cs_status encode_q_map(CUtensorMap* map, const void* q, const cs_attn_dims& d, int rows) {
+    auto enc = tensor_map_encoder();
+    if (!enc) return fail(CS_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+    const int G = d.n_q_heads / d.n_kv_heads;
+    const cuuint64_t dims[4] = {(cuuint64_t)d.head_dim, (cuuint64_t)d.n_q_heads, (cuuint64_t)rows, (cuuint64_t)d.batch};
+    const cuuint64_t row = (cuuint64_t)d.head_dim * 2;
+    const cuuint64_t strides[3] = {row, row * d.n_q_heads, row * d.n_q_heads * rows};
+    const cuuint32_t box[4] = {64, (cuuint32_t)G, (cuuint32_t)rows, 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(q), dims, strides, box, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(CS_ERR_CUDA, "cuTensorMapEncodeTiled (q) failed (CUresult %d)", (int)r);
+    return CS_OK;
+}
+
+// CTAs per SM of the tcgen05 kernel (1 when its shared memory fits; cached).
+int tc_resident_per_sm() {
+    static int cache[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+        cudaGetLastError();
+        return 0;
+    }
+    if (!cache[dev]) {
+        int n = 0;
+        if (cudaFuncSetAttribute(verify_attention_tc_kernel<false, 16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 tc_smem_bytes(kTcRows)) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, verify_attention_tc_kernel<false, 16>, kTcThreads,
+                                                          tc_smem_bytes(kTcRows)) != cudaSuccess)
+            n = 0;
+        cudaGetLastError();
+        cache[dev] = n + 1;
+    }
+    return cache[dev] - 1;
+}
+
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// The split merge as a programmatic dependent of the main kernel: it may
+// start early and waits (griddepcontrol.wait) before it reads the partials.
+cudaError_t launch_merge(const AttnParams& p, const AttnPlan& pl, cudaStream_t stream) {
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(p.n_vh, p.n_batch, (pl.n_rows + kMergeRows - 1) / kMergeRows);
+    cfg.blockDim = dim3(kMergeThreads, 1, 1);
+    cfg.stream = stream;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, verify_attention_merge_kernel, p, (int)pl.grid);
+}
 
 // Resident CTAs per SM of the kernel at a given block size (cached per device).
 template <bool kTree, int kSplit>
@@ -815,12 +879,22 @@ AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count
     pl.row_warps = (pl.n_rows + 15) / 16;
     // few rows: two consumer groups share each tile's keys
     pl.split = pl.row_warps <= kMaxSplitRowWarps ? 2 : 1;
-    // persistent grid: exactly the CTAs that are resident at once
-    const int threads = (pl.split * pl.row_warps + 1) * 32;
-    const int res = pl.split == 2 ? (tree ? resident_per_sm<true, 2>(threads) : resident_per_sm<false, 2>(threads))
-                                  : (tree ? resident_per_sm<true, 1>(threads) : resident_per_sm<false, 1>(threads));
-    pl.grid = (sm_count > 0 ? sm_count : 148) * res;
-    if (pl.grid > kMaxGrid) pl.grid = kMaxGrid;
+    // 49..128 rows (one row block) on pages of 16+ tokens: the tcgen05 kernel
+    // (with fewer rows its M = 128 padding costs more than the mma.sync form)
+    pl.tc = pl.n_rb == 1 && pl.n_rows_all > kTcMinRows && pl.n_rows_all <= kTcRows &&
+            d.page_size >= 16 && rows <= 256 && pl.group <= 256 && tc_resident_per_sm() >= 1;
+    if (pl.tc) {
+        pl.split = 1;
+        pl.grid = (sm_count > 0 ? sm_count : 148) * tc_resident_per_sm();
+        if (pl.grid > kMaxGrid) pl.grid = kMaxGrid;
+    } else {
+        // persistent grid: exactly the CTAs that are resident at once
+        const int threads = (pl.split * pl.row_warps + 1) * 32;
+        const int res = pl.split == 2 ? (tree ? resident_per_sm<true, 2>(threads) : resident_per_sm<false, 2>(threads))
+                                      : (tree ? resident_per_sm<true, 1>(threads) : resident_per_sm<false, 1>(threads));
+        pl.grid = (sm_count > 0 ? sm_count : 148) * res;
+        if (pl.grid > kMaxGrid) pl.grid = kMaxGrid;
+    }
     size_t off = 256;   // status word lives at offset 0
     pl.off_part_ml = off;
     off = align_up(off + sizeof(float) * 2 * (size_t)2 * pl.grid * pl.n_rows, 256);
@@ -877,6 +951,51 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     const float scale = d.sm_scale > 0.f ? d.sm_scale : 1.0f / sqrtf((float)d.head_dim);
     p.scale_log2 = scale * 1.4426950408889634f;
 
+    if (pl.tc && (reinterpret_cast<uintptr_t>(q) & 15) != 0) {
+        // the query rows come in by TMA, which needs a 16-byte aligned base:
+        // run the mma.sync form on the same workspace (its grid capped at
+        // the plan's, so the partial slots fit)
+        AttnPlan alt = plan_attention(d, pl.rows, pl.tree, 0);
+        alt.tc = false;
+        if (alt.grid > pl.grid) alt.grid = pl.grid;
+        alt.off_part_ml = pl.off_part_ml;
+        alt.off_part_o = pl.off_part_o;
+        alt.bytes = pl.bytes;
+        return launch_verify_attention(d, alt, q, k_pages, v_pages, page_table, ctx_lens, parents, out, workspace,
+                                       stream);
+    }
+    if (pl.tc) {
+        CUtensorMap tq;
+        st = encode_q_map(&tq, q, d, pl.rows);
+        if (st != CS_OK) return st;
+        st = encode_pool_map(&tk, k_pages, d, box_t, 1);
+        if (st != CS_OK) return st;
+        st = encode_pool_map(&tv, v_pages, d, box_t, 1);
+        if (st != CS_OK) return st;
+        using TcKern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const AttnParams);
+        static const TcKern tc_kerns[2][3] = {
+            {verify_attention_tc_kernel<false, 16>, verify_attention_tc_kernel<false, 32>,
+             verify_attention_tc_kernel<false, 64>},
+            {verify_attention_tc_kernel<true, 16>, verify_attention_tc_kernel<true, 32>,
+             verify_attention_tc_kernel<true, 64>}};
+        const int ti = box_t == 16 ? 0 : box_t == 32 ? 1 : 2;
+        const TcKern tk_fn = tc_kerns[pl.tree][ti];
+        p.tc_stages = tc_stages(pl.n_rows_all);
+        p.tc_q_half = tc_q_half_bytes(pl.n_rows_all);
+        const int smem_bytes = tc_smem_bytes(pl.n_rows_all);
+        cudaError_t e = cudaFuncSetAttribute(tk_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_attention_tc_kernel)");
+        for (int b0 = 0; b0 < d.batch; b0 += kMaxBatchPerLaunch) {
+            p.b_base = b0;
+            p.n_batch = d.batch - b0 < kMaxBatchPerLaunch ? d.batch - b0 : kMaxBatchPerLaunch;
+            tk_fn<<<pl.grid, kTcThreads, smem_bytes, stream>>>(tk, tv, tq, p);
+            e = cudaGetLastError();
+            if (e != cudaSuccess) return cuda_fail(e, "verify_attention_tc_kernel launch");
+            e = launch_merge(p, pl, stream);
+            if (e != cudaSuccess) return cuda_fail(e, "verify_attention_merge_kernel launch");
+        }
+        return CS_OK;
+    }
     // kernels by (key split, tree, box size 8/16/32/64 keys)
     using Kern = void (*)(const CUtensorMap, const CUtensorMap, const AttnParams);
     static const Kern kerns[2][2][4] = {
@@ -910,18 +1029,7 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
         kern<<<pl.grid, block, kSmemBytes, stream>>>(tk, tv, p);
         e = cudaGetLastError();
         if (e != cudaSuccess) return cuda_fail(e, "verify_attention_kernel launch");
-        // programmatic dependent launch: the merge kernel may start early and
-        // waits (griddepcontrol.wait) before it reads the partials
-        cudaLaunchAttribute attr;
-        attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr.val.programmaticStreamSerializationAllowed = 1;
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(p.n_vh, p.n_batch, (pl.n_rows + kMergeRows - 1) / kMergeRows);
-        cfg.blockDim = dim3(kMergeThreads, 1, 1);
-        cfg.stream = stream;
-        cfg.attrs = &attr;
-        cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, verify_attention_merge_kernel, (const AttnParams)p, (int)pl.grid);
+        e = launch_merge(p, pl, stream);
         if (e != cudaSuccess) return cuda_fail(e, "verify_attention_merge_kernel launch");
     }
     return CS_OK;

@@ -1,0 +1,596 @@
+// verify_attention_tc.cuh -- the tcgen05 form of the verify-attention kernel
+// (included by verify_attention.cu inside its anonymous namespace, so that it
+// shares the schedule, the parameter block, the tensor maps and the merge).
+//
+// Used for 49..128 query rows per KV head, where the mma.sync consumers of
+// the other form run out of tensor throughput (with fewer rows the M = 128
+// padding of every MMA costs more than it saves).  Same persistent schedule
+// (equal contiguous tile ranges, spans, two partial slots per CTA, merge
+// kernel), one CTA per SM, warp roles:
+//   warp 0  TMA producer: the span's query rows (one 4-D box per dim half,
+//           double-buffered across spans, each half as many 128-byte rows as
+//           the span has: the MMA's 128-row window runs on into whatever
+//           follows, which only feeds padded rows) and the K/V tiles of the
+//           range through a ring of as many 32 KB stages as shared memory
+//           then holds (4-6), one box per page piece and dim half, so a tile
+//           lands as [dim half][64 keys][128 B], 128-byte swizzle;
+//   warp 1  MMA issuer (one thread): S_t = Q K_t^T into tensor memory
+//           (M = 128 padded rows, N = 64 keys, K-major operands, 8 steps of
+//           16 dims), then O += P_{t-1} V_{t-1} (N = 128 dims, 4 steps of 16
+//           keys) with P read from tensor memory and V an MN-major operand
+//           whose two dim halves lie one leading offset apart -- one tile
+//           behind, so that the tensor core computes S_t while the softmax
+//           works on S_{t-1};
+//   warp 2  tensor-memory allocation (512 columns: four S/P buffers of 64,
+//           O in 128), so that QK can run up to three tiles ahead of PV;
+//   warps 4-7  softmax and epilogue, one query row per thread (warp 4+s
+//           owns tensor-memory lanes 32s..32s+31): mask, running max, exp2,
+//           row sum, P written back over S as fp16 (and the V tile turned
+//           from bf16 into fp16 in place, so that PV multiplies fp16 by fp16:
+//           bf16 P alone can exceed the output tolerance on rows whose terms
+//           cancel); O is rescaled in tensor
+//           memory only when the running max grows by more than 2^8 (the
+//           stale max keeps every P below 256); at a span piece's end the
+//           row is normalised and written (bf16) or left as a partial.
+// Every mbarrier wait is bounded; a wait that gives up sets the status word
+// and a shared flag that ends every warp's loop.
+
+constexpr int kTcMaxStages = 6;
+constexpr int kTcThreads = 256;
+constexpr int kTcRows = 128;                       // MMA M: query rows, padded
+constexpr int kTcMinRows = 48;                     // fewer query rows take the mma.sync form
+constexpr int kTcSBuf = 4;                         // S/P buffers in tensor memory
+constexpr int kTcOCol = kTcSBuf * 64;              // first column of O
+constexpr int kTcTmemCols = 512;                   // S/P [0, 256) in four buffers, O [256, 384)
+constexpr int kTcBarBytes = 512;
+constexpr int kTcFixedSmem = kTcBarBytes + (kMaxBatchPerLaunch + 1) * 8 + kMaxBatchPerLaunch * 4 + 1024;
+constexpr int kTcSmemLimit = 232448 - 256;         // opt-in shared memory per block, less the static part
+
+// Bytes between the two dim halves of a span's query rows (1024-aligned).
+__host__ __device__ constexpr int tc_q_half_bytes(int rows) { return (rows * 128 + 1023) / 1024 * 1024; }
+// K/V stages that fit beside two query buffers of `rows` rows.
+__host__ __device__ constexpr int tc_stages(int rows) {
+    return (kTcSmemLimit - kTcFixedSmem - 4 * tc_q_half_bytes(rows)) / kStageBytes < kTcMaxStages
+               ? (kTcSmemLimit - kTcFixedSmem - 4 * tc_q_half_bytes(rows)) / kStageBytes
+               : kTcMaxStages;
+}
+__host__ __device__ constexpr int tc_smem_bytes(int rows) {
+    return 4 * tc_q_half_bytes(rows) + tc_stages(rows) * kStageBytes + kTcFixedSmem;
+}
+static_assert(tc_stages(kTcRows) >= 4, "ring too shallow for 128 query rows");
+constexpr float kTcRescale = 8.f;                  // log2 growth of the max that forces a rescale of O
+
+__device__ __forceinline__ uint64_t tc_sw128_desc(uint32_t addr) {
+    // K-major, 128-byte swizzle: 8-row groups 1024 bytes apart (leading offset unused)
+    return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) |
+           (2ull << 61);
+}
+
+// MN-major, 128-byte swizzle, for the V tile [dim half][64 keys][128 B]:
+// 8-key groups 1024 bytes apart (stride), the two 64-dim halves one half
+// tile apart (leading offset)
+__device__ __forceinline__ uint64_t tc_mn_desc(uint32_t addr) {
+    return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)((kTileT * 128) >> 4) << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) | (2ull << 61);
+}
+
+// kind::f16 instruction descriptor: fp32 D, M = 128, N = n, A and B both
+// bf16 (QK) or both fp16 (PV); b_mn: B is MN-major (its N index contiguous)
+__host__ __device__ constexpr uint32_t tc_idesc(int n, bool b_mn, bool f16) {
+    return (1u << 4) | (f16 ? 0u : (1u << 7) | (1u << 10)) | (b_mn ? (1u << 16) : 0u) | ((uint32_t)(n >> 3) << 17) |
+           ((uint32_t)(kTcRows >> 4) << 24);
+}
+
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ void tc_mma_ss(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, q;\n\t}\n" ::"r"(d),
+        "l"(a), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_mma_ts(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, q;\n\t}\n" ::"r"(d),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_ld32(uint32_t addr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(addr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void tc_st32(uint32_t addr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(addr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]),
+        "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]),
+        "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Bounded wait that also gives up at once when another warp already has.
+__device__ __forceinline__ bool tc_wait(uint64_t* bar, uint32_t parity, volatile int* dead, int* status) {
+    if (*dead) return false;
+    if (mbar_wait_bounded(bar, parity)) return true;
+    *dead = 1;
+    atomicOr(status, CS_DEVICE_WAIT_TIMEOUT);
+    return false;
+}
+
+constexpr int kTcHalfBytes = kTileT * 128;       // one dim half of a 64-key K or V tile
+
+template <bool kTree, int kBoxT>
+__global__ void __launch_bounds__(kTcThreads, 1)
+verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __grid_constant__ CUtensorMap tmap_v,
+                           const __grid_constant__ CUtensorMap tmap_q, const AttnParams p) {
+    constexpr int kPieces = kTileT / kBoxT;
+    constexpr uint32_t kPieceBytes = (uint32_t)kBoxT * 256u;   // K and V bytes of one page piece each
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int kTcStages = p.tc_stages;                      // K/V ring depth
+    const int qh = p.tc_q_half;                             // bytes between the dim halves of a span's rows
+    uint8_t* sq = smem;                                     // [2 spans][2 halves][rows][128 B]
+    uint8_t* skv = smem + 4 * qh;                           // [stage][K | V][half][64 keys][128 B]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(skv + kTcStages * kStageBytes);
+    uint64_t* full = bars;                                  // [stages] K/V landed
+    uint64_t* empty = bars + kTcMaxStages;                  // [stages] K/V consumed (PV done)
+    uint64_t* q_full = bars + 2 * kTcMaxStages;             // [2] Q of a span landed
+    uint64_t* q_free = q_full + 2;                          // [2] last QK of a span done
+    uint64_t* s_full = q_free + 2;                          // [kTcSBuf] S_t in tensor memory
+    uint64_t* s_free = s_full + kTcSBuf;                    // [kTcSBuf] P_t consumed (PV_t done)
+    uint64_t* p_full = s_free + kTcSBuf;                    // [kTcSBuf] P_t written (count 4 warps)
+    uint64_t* o_ready = p_full + kTcSBuf;                   // [kTcSBuf] PV_t done, by S buffer
+    uint64_t* o_free = o_ready + kTcSBuf;                   // O read out by the epilogue (count 4 warps)
+    long long* s_prefix = reinterpret_cast<long long*>(reinterpret_cast<uint8_t*>(bars) + kTcBarBytes);
+    int* s_len = reinterpret_cast<int*>(s_prefix + kMaxBatchPerLaunch + 1);
+    __shared__ long long s_wtot[kTcThreads / 32];
+    __shared__ long long s_carry;
+    __shared__ uint32_t s_tmem;
+    __shared__ volatile int s_dead;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nb = p.n_batch;
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    if (warp == 0) {
+        // the page table of this launch into L2 while the schedule is computed
+        const char* tab = reinterpret_cast<const char*>(p.page_table + (size_t)p.b_base * p.max_pages);
+        const long long lines = ((long long)nb * p.max_pages * 4 + 127) / 128;
+        for (long long i = (long long)blockIdx.x * 32 + lane; i < lines; i += (long long)gridDim.x * 32)
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(tab + i * 128));
+    }
+    if (warp == 2) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s_tmem)),
+                     "n"(kTcTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    if (threadIdx.x == 0) {
+        s_carry = 0;
+        s_dead = 0;
+        for (int i = 0; i < kTcStages; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&q_full[i], 1);
+            mbar_init(&q_free[i], 1);
+        }
+        for (int i = 0; i < kTcSBuf; ++i) {
+            mbar_init(&s_full[i], 1);
+            mbar_init(&s_free[i], 1);
+            mbar_init(&p_full[i], 4);
+            mbar_init(&o_ready[i], 1);
+        }
+        mbar_init(o_free, 4);
+        fence_barrier_init();
+    }
+    // ---- schedule: exclusive prefix of tiles per request (x spans), clamped L
+    __syncthreads();
+    const int l_cap = p.max_pages * p.ps;
+    for (int base = 0; base < nb; base += kTcThreads) {
+        const int bl = base + threadIdx.x;
+        long long v = 0;
+        if (bl < nb) {
+            int L = __ldg(p.ctx_lens + p.b_base + bl);
+            L = max(0, min(L, l_cap));
+            s_len[bl] = L;
+            v = (long long)tiles_of(L) * p.n_vh;
+        }
+        long long inc = v;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const long long y = __shfl_up_sync(0xffffffffu, inc, off);
+            if (lane >= off) inc += y;
+        }
+        if (lane == 31) s_wtot[warp] = inc;
+        __syncthreads();
+        long long before = s_carry;
+        for (int w = 0; w < warp; ++w) before += s_wtot[w];
+        if (bl < nb) s_prefix[bl] = before + inc - v;
+        __syncthreads();
+        if (threadIdx.x == kTcThreads - 1) s_carry = before + inc;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) s_prefix[nb] = s_carry;
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+
+    const long long W = s_prefix[nb];
+    const long long g_need = (W + kMinTilesPerCta - 1) / kMinTilesPerCta;
+    const int Gc = (int)(g_need < (long long)gridDim.x ? (g_need > 0 ? g_need : 1) : gridDim.x);
+    const int cta = blockIdx.x;
+    long long f0 = (long long)cta * W / Gc, f1 = (long long)(cta + 1) * W / Gc;
+    if (cta >= Gc) f0 = f1 = 0;
+    const int n_tiles = (int)(f1 - f0);
+    const uint32_t qrow_bytes = (uint32_t)(p.R * p.G) * 128u;   // one dim half of a span's rows
+
+    if (warp == 0 && n_tiles > 0) {
+        // ---------------------------------------------------------- producer
+        constexpr int per_batch = 32 / kPieces;
+        auto batch_pages = [&](int j0) -> int {
+            const int jj = j0 + lane / kPieces;
+            if (jj >= n_tiles) return -1;
+            const Cursor cc = locate(f0 + jj, s_prefix, s_len, nb, p.n_vh);
+            const int tok = cc.t * kTileT + (lane % kPieces) * kBoxT;
+            if (tok >= s_len[cc.b]) return -1;
+            return __ldg(p.page_table + (size_t)(p.b_base + cc.b) * p.max_pages + tok / p.ps);
+        };
+        if (lane == 0) {
+            tma_prefetch_desc(&tmap_k);
+            tma_prefetch_desc(&tmap_v);
+            tma_prefetch_desc(&tmap_q);
+        }
+        Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
+        int pg_cur = batch_pages(0);
+        int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
+        int span = -1;
+        for (int j = 0; j < n_tiles; ++j) {
+            const int st = j % kTcStages;
+            const uint32_t use = (uint32_t)(j / kTcStages);
+            const int jb = j % per_batch;
+            if (j > 0 && jb == 0) {
+                pg_cur = pg_next;
+                pg_next = j + per_batch < n_tiles ? batch_pages(j + per_batch) : -1;
+            }
+            const int page = __shfl_sync(0xffffffffu, pg_cur, jb * kPieces + lane % kPieces);
+            const int L = s_len[cur.b];
+            const int ts = cur.t * kTileT;
+            const int h_cur = cur.h / p.n_rb;
+            int ok = 1;
+            if (lane == 0) {
+                if (j == 0 || cur.t == 0) {
+                    // a new span: its query rows into buffer span % 2, once
+                    // the span two back is done with it
+                    ++span;
+                    const int qb = span & 1;
+                    if (span >= 2 && !tc_wait(&q_free[qb], (uint32_t)((span - 2) >> 1) & 1, &s_dead, p.status)) ok = 0;
+                    if (ok) {
+                        mbar_arrive_expect_tx(&q_full[qb], 2 * qrow_bytes);
+                        const uint32_t qdst = smem_u32(sq + qb * 2 * qh);
+#pragma unroll
+                        for (int hh = 0; hh < 2; ++hh)
+                            tma_load_4d(qdst + hh * qh, &tmap_q, &q_full[qb], hh * 64, h_cur * p.G, 0,
+                                        p.b_base + cur.b);
+                    }
+                }
+                if (ok && j >= kTcStages && !tc_wait(&empty[st], (use - 1) & 1, &s_dead, p.status)) ok = 0;
+            }
+            advance(cur, s_len, nb, p.n_vh);
+            if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+            int valid = 0;
+            for (int pc = 0; pc < kPieces; ++pc)
+                if (ts + pc * kBoxT < L) ++valid;
+            if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)valid * kPieceBytes * 2u);
+            __syncwarp();
+            if (lane < valid) {
+                const uint32_t kdst = smem_u32(skv + st * kStageBytes) + (uint32_t)lane * (kBoxT * 128);
+                const int slot = (ts + lane * kBoxT) % p.ps;
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    tma_load_5d(kdst + hh * kTcHalfBytes, &tmap_k, &full[st], 0, slot, hh, h_cur, page);
+                    tma_load_5d(kdst + kTensorTileBytes + hh * kTcHalfBytes, &tmap_v, &full[st], 0, slot, hh, h_cur,
+                                page);
+                }
+            }
+        }
+        // no copy in flight at exit: the last fill of every stage has landed
+        if (lane == 0)
+            for (int j = n_tiles > kTcStages ? n_tiles - kTcStages : 0; j < n_tiles; ++j)
+                if (!mbar_wait_bounded(&full[j % kTcStages], (uint32_t)(j / kTcStages) & 1))
+                    atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+    } else if (warp == 1 && n_tiles > 0) {
+        // ---------------------------------------------------------- MMA
+        // One thread, polling: QK of tile qt as soon as its K/V, its S buffer
+        // and (first tile of a piece) its query rows are ready, up to
+        // kTcSBuf - 1 tiles ahead of PV; PV of tile vt as soon as its P is
+        // written and (first tile of a piece) the previous piece's epilogue
+        // has read O.  Each readiness probe names a phase its barrier can be
+        // at most one phase short of, so a parity probe is exact.
+        if (lane == 0) {
+            const uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, true);
+            Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
+            int qt = 0, vt = 0, span = -1;
+            uint32_t fl_first = 0;          // bit sb: the tile in S buffer sb opened its piece
+            int fl_piece[kTcSBuf] = {};     // piece of the tile in each S buffer
+            uint64_t t_progress = global_timer_ns();
+            uint32_t polls = 0;
+            while (vt < n_tiles) {
+                if (s_dead) break;
+                bool progress = false;
+                if (qt < n_tiles && qt - vt < kTcSBuf) {
+                    const bool first = qt == 0 || cur.t == 0;
+                    const int sp = first ? span + 1 : span;
+                    const int st = qt % kTcStages, sb = qt % kTcSBuf;
+                    if ((!first || mbar_test_wait(&q_full[sp & 1], (uint32_t)(sp >> 1) & 1)) &&
+                        mbar_test_wait(&full[st], (uint32_t)(qt / kTcStages) & 1) &&
+                        (qt < kTcSBuf || mbar_test_wait(&s_free[sb], (uint32_t)((qt - kTcSBuf) / kTcSBuf) & 1))) {
+                        span = sp;
+                        tc_fence_after();
+                        // S_qt = Q K_qt^T, 8 steps of 16 dims
+                        const uint32_t qbase = smem_u32(sq + (span & 1) * 2 * qh);
+                        const uint32_t kbase = smem_u32(skv + st * kStageBytes);
+#pragma unroll
+                        for (int ks = 0; ks < kD / 16; ++ks) {
+                            const int hh = ks >> 2, kc = (ks & 3) * 32;
+                            tc_mma_ss(tmem + sb * 64, tc_sw128_desc(qbase + hh * qh + kc),
+                                      tc_sw128_desc(kbase + hh * kTcHalfBytes + kc), id_s, ks > 0 ? 1u : 0u);
+                        }
+                        tc_commit(&s_full[sb]);
+                        if (qt + 1 == n_tiles || cur.t + 1 == cur.T) tc_commit(&q_free[span & 1]);
+                        fl_first = first ? (fl_first | (1u << sb)) : (fl_first & ~(1u << sb));
+                        fl_piece[sb] = span;
+                        advance(cur, s_len, nb, p.n_vh);
+                        ++qt;
+                        progress = true;
+                    }
+                }
+                if (vt < qt) {
+                    const int st = vt % kTcStages, sb = vt % kTcSBuf;
+                    const bool first = (fl_first >> sb) & 1u;
+                    const int piece = fl_piece[sb];
+                    if (mbar_test_wait(&p_full[sb], (uint32_t)(vt / kTcSBuf) & 1) &&
+                        (!first || piece == 0 || mbar_test_wait(o_free, (uint32_t)(piece - 1) & 1))) {
+                        tc_fence_after();
+                        // O += P_vt V_vt, 4 steps of 16 keys, both dim halves per step
+                        const uint32_t vbase = smem_u32(skv + st * kStageBytes + kTensorTileBytes);
+#pragma unroll
+                        for (int kk = 0; kk < kTileT / 16; ++kk)
+                            tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + kk * 8, tc_mn_desc(vbase + kk * 16 * 128),
+                                      id_o, (first && kk == 0) ? 0u : 1u);
+                        tc_commit(&o_ready[sb]);
+                        tc_commit(&empty[st]);
+                        tc_commit(&s_free[sb]);
+                        ++vt;
+                        progress = true;
+                    }
+                }
+                if (progress) {
+                    polls = 0;
+                } else if ((++polls & 255u) == 0) {
+                    const uint64_t now = global_timer_ns();
+                    if (polls == 256) t_progress = now;
+                    else if (now - t_progress > 1000000000ull) {   // about one second without progress
+                        s_dead = 1;
+                        atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+                        break;
+                    }
+                }
+            }
+            // every MMA of this CTA completes before tensor memory is freed:
+            // the last PV of each S buffer is the latest phase of its barrier
+            for (int t = vt >= kTcSBuf ? vt - kTcSBuf : 0; t < vt; ++t)
+                if (!mbar_wait_bounded(&o_ready[t % kTcSBuf], (uint32_t)(t / kTcSBuf) & 1)) break;
+        }
+    } else if (warp >= 4 && n_tiles > 0) {
+        // ---------------------------------------------------- softmax, epilogue
+        const int sub = warp & 3;
+        const int row = sub * 32 + lane;                       // query row of the span = tensor-memory lane
+        const uint32_t t_row = tmem + ((uint32_t)(sub * 32) << 16);
+        const float c = p.scale_log2;
+        Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
+        int seg_t0 = cur.t;
+        bool first_seg = true;
+        float m_run = kNegInf, l_run = 0.f;
+        int lim = 0, tree_base = 0, span_L = 0;
+        uint64_t anc = ~0ull;
+        auto begin_span = [&](const Cursor& cc) {
+            const int L = s_len[cc.b];
+            m_run = kNegInf;
+            l_run = 0.f;
+            if (kTree) {
+                uint64_t ma, mb;
+                tree_ancestor_masks(p.parents + (size_t)(p.b_base + cc.b) * p.R, p.R, lane, ma, mb);
+                const int i = row / p.G;
+                const uint64_t x = __shfl_sync(0xffffffffu, ma, i & 31), y = __shfl_sync(0xffffffffu, mb, i & 31);
+                anc = row < p.n_rows_all ? (i >= 32 ? y : x) : ~0ull;
+                tree_base = L - p.R;
+                span_L = L;
+            } else {
+                lim = row < p.n_rows_all ? L - p.R + 1 + row / p.G : L;
+            }
+        };
+        begin_span(cur);
+        for (int t = 0; t < n_tiles; ++t) {
+            const int sb = t % kTcSBuf, st = t % kTcStages;
+            const int L = s_len[cur.b];
+            const int ts = cur.t * kTileT;
+            const bool piece_end = t + 1 == n_tiles || cur.t + 1 == cur.T;
+            if (!tc_wait(&s_full[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) break;
+            tc_fence_after();
+            float s[64];
+            tc_ld32(t_row + sb * 64, *reinterpret_cast<float(*)[32]>(&s[0]));
+            tc_ld32(t_row + sb * 64 + 32, *reinterpret_cast<float(*)[32]>(&s[32]));
+            // ---- mask (tree ancestors or the causal chain, and the context end);
+            // padded rows see nothing
+            float mt = kNegInf;
+            if (row >= p.n_rows_all) {
+#pragma unroll
+                for (int e = 0; e < 64; ++e) s[e] = kNegInf;
+            } else if (kTree) {
+                const int d = ts - tree_base;
+                const uint64_t pre = d >= 0 ? 0ull : (d <= -64 ? ~0ull : (1ull << -d) - 1ull);
+                const uint64_t live = span_L - ts >= 64 ? ~0ull : (1ull << max(span_L - ts, 0)) - 1ull;
+                const uint64_t tr = d >= 64 ? 0ull : (d >= 0 ? anc >> d : (d <= -64 ? 0ull : anc << -d));
+                const uint64_t vis = (pre | tr) & live;
+#pragma unroll
+                for (int e = 0; e < 64; ++e) {
+                    if (!((vis >> e) & 1ull)) s[e] = kNegInf;
+                    mt = fmaxf(mt, s[e]);
+                }
+            } else {
+                const int lim_t = lim - ts;   // keys e < lim_t are visible
+#pragma unroll
+                for (int e = 0; e < 64; ++e) {
+                    if (e >= lim_t) s[e] = kNegInf;
+                    mt = fmaxf(mt, s[e]);
+                }
+            }
+            // ---- running max, lazily: O is rescaled only for a growth > 2^8
+            float alpha = 1.f;
+            if (mt != kNegInf && (m_run == kNegInf || (mt - m_run) * c > kTcRescale)) {
+                alpha = m_run == kNegInf ? 0.f : ex2((m_run - mt) * c);
+                m_run = mt;
+            }
+            const float neg = m_run == kNegInf ? 0.f : -m_run * c;
+            float rs = 0.f;
+            uint32_t pk[32];
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                const float p0 = ex2(fmaf(s[2 * e], c, neg)), p1 = ex2(fmaf(s[2 * e + 1], c, neg));
+                rs += p0 + p1;
+                pk[e] = pack_f16x2(p0, p1);
+            }
+            l_run = l_run * alpha + rs;
+            // ---- a rescale of O waits for PV_{t-1}; the first tile of a piece
+            // needs none (its PV overwrites O).  o_ready[b] completes once per
+            // tile of S buffer b: PV_{t-5} is complete (QK_t waited for
+            // PV_{t-4}) and PV_{t+3} is not issued, so the parity of PV_{t-1}'s
+            // phase is unambiguous.
+            const unsigned need = __ballot_sync(0xffffffffu, alpha != 1.f && cur.t != seg_t0);
+            if (need) {
+                const int tp = t - 1;
+                if (!tc_wait(&o_ready[tp % kTcSBuf], (uint32_t)(tp / kTcSBuf) & 1, &s_dead, p.status)) break;
+                tc_fence_after();
+#pragma unroll 1
+                for (int c0 = 0; c0 < 128; c0 += 32) {
+                    float o[32];
+                    tc_ld32(t_row + kTcOCol + c0, o);
+                    uint32_t r[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(o[i] * alpha);
+                    tc_st32(t_row + kTcOCol + c0, r);
+                }
+            }
+            tc_st32(t_row + sb * 64, pk);
+            tc_wait_st();
+            // the V tile into fp16, in place: each thread owns 8 of its 1024
+            // 16-byte chunks (the swizzle only permutes chunks within a
+            // 128-byte row, so a chunk's key is its row); rows past L_b may
+            // hold any bits and are zeroed instead
+            {
+                uint4* vt = reinterpret_cast<uint4*>(skv + st * kStageBytes + kTensorTileBytes);
+                const int keys = min(kTileT, L - ts);
+#pragma unroll
+                for (int i = 0; i < kTensorTileBytes / 16 / 128; ++i) {
+                    const int ci = i * 128 + sub * 32 + lane;
+                    uint4 v = make_uint4(0, 0, 0, 0);
+                    if (((ci >> 3) & (kTileT - 1)) < keys) {
+                        v = vt[ci];
+                        v.x = bf16x2_to_f16x2(v.x);
+                        v.y = bf16x2_to_f16x2(v.y);
+                        v.z = bf16x2_to_f16x2(v.z);
+                        v.w = bf16x2_to_f16x2(v.w);
+                    }
+                    vt[ci] = v;
+                }
+            }
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&p_full[sb]);
+
+            if (!piece_end) {
+                advance(cur, s_len, nb, p.n_vh);
+                continue;
+            }
+            // ---- end of a span piece: O after its last PV (every earlier MMA
+            // completes before that commit), then written
+            if (!tc_wait(&o_ready[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) break;
+            tc_fence_after();
+            const int bg = p.b_base + cur.b;
+            const int head = cur.h / p.n_rb;
+            const bool complete = seg_t0 == 0 && cur.t + 1 == cur.T;
+            const size_t slot = 2 * (size_t)cta + (first_seg ? 0 : 1);
+            const bool live_row = row < p.n_rows_all;
+            const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+#pragma unroll 1
+            for (int c0 = 0; c0 < 128; c0 += 32) {
+                float o[32];
+                tc_ld32(t_row + kTcOCol + c0, o);
+                if (!live_row) continue;
+                if (complete) {
+                    const int i = row / p.G, gi = row % p.G;
+                    __nv_bfloat16* dst = p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + c0;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint4 v;
+                        v.x = pack_bf16x2(o[8 * q + 0] * inv, o[8 * q + 1] * inv);
+                        v.y = pack_bf16x2(o[8 * q + 2] * inv, o[8 * q + 3] * inv);
+                        v.z = pack_bf16x2(o[8 * q + 4] * inv, o[8 * q + 5] * inv);
+                        v.w = pack_bf16x2(o[8 * q + 6] * inv, o[8 * q + 7] * inv);
+                        *reinterpret_cast<uint4*>(dst + 8 * q) = v;
+                    }
+                } else {
+                    float* dst = p.part_o + (slot * p.n_rows + row) * kD + c0;
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        *reinterpret_cast<float4*>(dst + 4 * q) =
+                            make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                }
+            }
+            if (live_row && !complete)
+                p.part_ml[slot * p.n_rows + row] = make_float2(m_run == kNegInf ? kNegInf : m_run * c, l_run);
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(o_free);
+            if (t + 1 < n_tiles) {
+                advance(cur, s_len, nb, p.n_vh);
+                seg_t0 = cur.t;
+                first_seg = false;
+                begin_span(cur);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 2)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(kTcTmemCols) : "memory");
+}

@@ -204,3 +204,36 @@ def test_empty_batch():
     e = {k: (v[:0] if k in ("q", "page_table", "ctx_lens") else v) for k, v in inp.items()}
     out = gpu(e)
     assert out.shape[0] == 0
+
+
+# ---- the tcgen05 form (49..128 query rows per KV head, pages of 16+ tokens)
+@pytest.mark.parametrize("k,Hq,Hkv,ps", [(8, 64, 8, 16), (8, 64, 8, 32), (8, 64, 8, 64), (8, 64, 8, 128),
+                                         (8, 64, 8, 256), (6, 28, 4, 16), (15, 64, 8, 32), (16, 32, 8, 16)])
+def test_tcgen05_row_counts_and_page_sizes(k, Hq, Hkv, ps):
+    """Boundary row counts (49, 128), every page size the form takes."""
+    inp = W.attention_inputs(small(B=3, k=k, Hq=Hq, Hkv=Hkv, ps=ps, lo=k + 1, hi=900, cell=7000 + k * 10 + ps), DEV)
+    assert_parity(gpu(inp), ref(inp), f"tc k={k} G={Hq // Hkv} ps={ps}")
+
+
+def test_tcgen05_span_pieces_and_repeat_calls():
+    """Many short spans (every CTA crosses spans and cut pieces) and the same
+    workspace used for consecutive calls."""
+    inp = W.attention_inputs(small(B=40, k=8, Hq=64, Hkv=8, ps=16, lo=9, hi=400, cell=7100), DEV)
+    expect = ref(inp)
+    for _ in range(3):
+        assert_parity(gpu(inp), expect, "tc many spans")
+
+
+def test_tcgen05_unaligned_query_falls_back():
+    """A query base that is 4- but not 16-byte aligned cannot feed TMA: the call
+    runs the other form on the same workspace and still matches."""
+    inp = W.attention_inputs(small(B=2, k=8, Hq=64, Hkv=8, ps=16, lo=100, hi=600, cell=7200), DEV)
+    q = inp["q"]
+    buf = torch.empty(q.numel() + 2, dtype=torch.bfloat16, device=DEV)
+    q2 = buf[2:].view(q.shape)
+    q2.copy_(q)
+    assert q2.data_ptr() % 16 != 0 and q2.data_ptr() % 4 == 0
+    out = binding.cs_verify_attention(q2, inp["k_pages"], inp["v_pages"], inp["page_table"], inp["ctx_lens"],
+                                      inp["n_draft"])
+    torch.cuda.synchronize()
+    assert_parity(out, ref(inp), "tc fallback")

@@ -67,6 +67,8 @@ def assert_close(got, ref):
     (2, 32, 64, 8, 32, ("uniform", 100, 900), 2),      # 256 rows: two row blocks
     (1, 64, 28, 4, 16, ("const", 2000), 3),            # 448 rows: four row blocks, 64 nodes
     (4, 12, 16, 4, 8, ("uniform", 5, 60), 4),          # contexts shorter than a tile, some L < n
+    (3, 16, 32, 8, 16, ("uniform", 20, 700), 5),       # 64 rows: the tcgen05 form
+    (2, 30, 16, 4, 32, ("uniform", 40, 900), 6),       # 120 rows: the tcgen05 form, 32-token pages
 ])
 def test_tree_attention_matches_oracle(B, n, Hq, Hkv, ps, ctx, seed):
     inp = tree_attn_case(B, n, Hq, Hkv, ps, ctx, seed)
