@@ -38,9 +38,10 @@
 // the current span each (draft row i = r / G, query head h*G + r % G), so
 // every K/V byte staged in shared memory serves all rows; they run S = Q K^T
 // on bf16 tensor cores and O += P V on fp16 ones (mma.sync m16n8k16, fp32
-// accumulate; P rounded to fp16, V fragments converted from bf16, which is
-// exact for values inside fp16's range) with an fp32 online softmax in the
-// log2 domain.  fp16 P is eight times finer than bf16: with bf16 P the
+// accumulate; P rounded to fp16, V converted from bf16 -- in shared memory by
+// the producer warp, or in registers by key-split consumers -- which is exact
+// for values inside fp16's range) with an fp32 online softmax in the log2
+// domain.  fp16 P is eight times finer than bf16: with bf16 P the
 // rounding of the weights alone can exceed 2e-3 + 1e-2|o| on rows whose
 // terms cancel.
 #include <math.h>
@@ -178,6 +179,9 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     uint64_t* empty = full + kStages;
     uint64_t* fold_a = empty + kStages;   // key-split: every consumer is done with the stage
     uint64_t* fold_b = fold_a + 1;        // key-split: the second group's state is in the stage
+    uint64_t* ready = fold_b + 1;         // [kStages] the producer converted the stage's V (no key split)
+    constexpr bool kConvert = kSplit == 1;
+    __shared__ int s_keys[kStages];       // keys of the tile in each stage (rows past are zeroed)
     long long* s_prefix = reinterpret_cast<long long*>(smem + kStages * kStageBytes + kBarrierBytes);
     int* s_len = reinterpret_cast<int*>(s_prefix + kMaxBatchPerLaunch + 1);
     __shared__ long long s_wtot[kMaxRowWarps + 1];
@@ -205,6 +209,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         for (int i = 0; i < kStages; ++i) {
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], kSplit * nw);
+            mbar_init(&ready[i], 1);
         }
         mbar_init(fold_a, kSplit * nw);
         mbar_init(fold_b, nw);
@@ -253,10 +258,13 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 
     if (warp == kSplit * nw) {
         // ------------------------------------------------------ producer
-        // The whole warp produces: lane pc owns page piece pc of a tile (its
-        // page id is loaded one tile ahead, so the table lookups of all pieces
-        // overlap each other and the previous tile), lane 0 arms the stage's
-        // barrier, and every lane issues the TMA copies of its own piece.
+        // The whole warp produces: the next tile is issued once its stage is
+        // free (lane pc owns page piece pc; the page ids of 32/pieces tiles
+        // come from one warp-wide load issued a batch ahead).  Without the
+        // key split (three or more row warps, whose tensor throughput paces
+        // them) the producer also turns each landed V tile into fp16 in
+        // place before `ready` releases it; with it, the consumers convert
+        // their V fragments in registers, which adds less to their latency.
         if (lane == 0) {
             tma_prefetch_desc(&tmap_k);
             tma_prefetch_desc(&tmap_v);
@@ -276,36 +284,85 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
         int pg_cur = batch_pages(0);
         int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
-        for (int j = 0; j < n_tiles; ++j) {
-            const int st = j % kStages;
-            const uint32_t use = (uint32_t)(j / kStages);
-            const int jb = j % per_batch;
-            if (j > 0 && jb == 0) {
-                pg_cur = pg_next;
-                pg_next = j + per_batch < n_tiles ? batch_pages(j + per_batch) : -1;
+        int jt = 0, jc = 0;   // next tile to issue, next tile to convert
+        uint32_t polls = 0;
+        uint64_t t_idle = 0;
+        while (kConvert ? jc < n_tiles : jt < n_tiles) {
+            bool progress = false;
+            if (jt < n_tiles) {
+                const int st = jt % kStages;
+                int go = 1;
+                if (lane == 0 && jt >= kStages) go = mbar_test_wait(&empty[st], (uint32_t)(jt / kStages - 1) & 1);
+                if (__shfl_sync(0xffffffffu, go, 0)) {
+                    const int jb = jt % per_batch;
+                    if (jt > 0 && jb == 0) {
+                        pg_cur = pg_next;
+                        pg_next = jt + per_batch < n_tiles ? batch_pages(jt + per_batch) : -1;
+                    }
+                    const int page = __shfl_sync(0xffffffffu, pg_cur, jb * pieces + lane % pieces);
+                    const int L = s_len[cur.b];
+                    const int ts = cur.t * kTileT;
+                    const int h_cur = cur.h / p.n_rb;   // the KV head of this span
+                    advance(cur, s_len, nb, p.n_vh);
+                    int valid = 0;
+                    for (int pc = 0; pc < pieces; ++pc)
+                        if (ts + pc * kBoxT < L) ++valid;
+                    if (lane == 0) {
+                        s_keys[st] = max(0, min(kTileT, L - ts));
+                        mbar_arrive_expect_tx(&full[st], (uint32_t)valid * piece_bytes * 2u);
+                    }
+                    __syncwarp();
+                    if (lane < valid) {
+                        const uint32_t kdst = smem_base + st * kStageBytes + (uint32_t)lane * piece_bytes;
+                        const uint32_t vdst = kdst + kTensorTileBytes;
+                        const int slot = (ts + lane * kBoxT) % p.ps;
+                        tma_load_5d(kdst, &tmap_k, &full[st], 0, slot, 0, h_cur, page);
+                        tma_load_5d(vdst, &tmap_v, &full[st], 0, slot, 0, h_cur, page);
+                    }
+                    ++jt;
+                    progress = true;
+                }
             }
-            const int page = __shfl_sync(0xffffffffu, pg_cur, jb * pieces + lane % pieces);
-            const int L = s_len[cur.b];
-            const int ts = cur.t * kTileT;
-            const int h_cur = cur.h / p.n_rb;   // the KV head of this span
-            advance(cur, s_len, nb, p.n_vh);
-            int ok = 1;
-            if (lane == 0 && j >= kStages && !mbar_wait_bounded(&empty[st], (use - 1) & 1)) {
-                flag_timeout(p.status);
-                ok = 0;
+            if (kConvert && jc < jt) {
+                const int st = jc % kStages;
+                int landed = 0;
+                if (lane == 0) landed = mbar_test_wait(&full[st], (uint32_t)(jc / kStages) & 1);
+                if (__shfl_sync(0xffffffffu, landed, 0)) {
+                    // V tile rows are [piece][dim half][key]: row r holds key
+                    // (r / (2 kBoxT)) kBoxT + r % kBoxT; rows past L_b are zeroed
+                    const int keys = s_keys[st];
+                    uint4* vt = reinterpret_cast<uint4*>(smem + st * kStageBytes + kTensorTileBytes);
+#pragma unroll 4
+                    for (int i = lane; i < kTensorTileBytes / 16; i += 32) {
+                        const int r = i >> 3;
+                        const int key = (r / (2 * kBoxT)) * kBoxT + r % kBoxT;
+                        uint4 v = make_uint4(0, 0, 0, 0);
+                        if (key < keys) {
+                            v = vt[i];
+                            v.x = bf16x2_to_f16x2(v.x);
+                            v.y = bf16x2_to_f16x2(v.y);
+                            v.z = bf16x2_to_f16x2(v.z);
+                            v.w = bf16x2_to_f16x2(v.w);
+                        }
+                        vt[i] = v;
+                    }
+                    // these generic writes precede the next TMA write into the stage
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&ready[st]);
+                    ++jc;
+                    progress = true;
+                }
             }
-            if (!__shfl_sync(0xffffffffu, ok, 0)) break;
-            int valid = 0;
-            for (int pc = 0; pc < pieces; ++pc)
-                if (ts + pc * kBoxT < L) ++valid;
-            if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)valid * piece_bytes * 2u);
-            __syncwarp();
-            if (lane < valid) {
-                const uint32_t kdst = smem_base + st * kStageBytes + (uint32_t)lane * piece_bytes;
-                const uint32_t vdst = kdst + kTensorTileBytes;
-                const int slot = (ts + lane * kBoxT) % p.ps;
-                tma_load_5d(kdst, &tmap_k, &full[st], 0, slot, 0, h_cur, page);
-                tma_load_5d(vdst, &tmap_v, &full[st], 0, slot, 0, h_cur, page);
+            if (progress) {
+                polls = 0;
+            } else if ((++polls & 255u) == 0) {
+                const uint64_t now = global_timer_ns();
+                if (polls == 256) t_idle = now;
+                else if (now - t_idle > 1000000000ull) {   // about one second without progress
+                    if (lane == 0) flag_timeout(p.status);
+                    break;
+                }
             }
         }
         return;
@@ -385,15 +442,13 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     for (int j = 0; j < n_tiles; ++j) {
         const int st = j % kStages;
         const uint32_t use = (uint32_t)(j / kStages);
-        if (!mbar_wait_bounded(&full[st], use & 1)) {
+        if (!mbar_wait_bounded(kConvert ? &ready[st] : &full[st], use & 1)) {
             flag_timeout(p.status);
             break;
         }
         const int L = s_len[cur.b];
         const int ts = cur.t * kTileT;
-        const uint32_t kb = smem_base + st * kStageBytes;
-        const uint32_t vb = kb + kTensorTileBytes;
-        if (ts + kTileT > L) {
+        if (!kConvert && ts + kTileT > L) {
             // keys past L_b (pages not loaded, or slots past the context) may
             // hold any bits: zero their V rows so that P = 0 cannot meet NaN
             const int first = max(0, L - ts);
@@ -405,7 +460,8 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             }
             __syncwarp();
         }
-
+        const uint32_t kb = smem_base + st * kStageBytes;
+        const uint32_t vb = kb + kTensorTileBytes;
         // ---- S = Q K^T over this warp's keys: kNT n-tiles of 8 keys
         float sc[kNT][4];
 #pragma unroll
@@ -502,8 +558,14 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                 uint32_t b0, b1, b2, b3;
                 ldsm_x4_trans(vb + key_row(key, dblk >> 3) * 128 + ((ch ^ (key & 7)) << 4), b0,
                               b1, b2, b3);
-                mma_f16_16816(o[2 * dp], a, bf16x2_to_f16x2(b0), bf16x2_to_f16x2(b1));
-                mma_f16_16816(o[2 * dp + 1], a, bf16x2_to_f16x2(b2), bf16x2_to_f16x2(b3));
+                if (!kConvert) {   // V fragments from bf16 to fp16
+                    b0 = bf16x2_to_f16x2(b0);
+                    b1 = bf16x2_to_f16x2(b1);
+                    b2 = bf16x2_to_f16x2(b2);
+                    b3 = bf16x2_to_f16x2(b3);
+                }
+                mma_f16_16816(o[2 * dp], a, b0, b1);
+                mma_f16_16816(o[2 * dp + 1], a, b2, b3);
             }
         }
         const bool piece_end = !(j + 1 < n_tiles && cur.t + 1 < cur.T);
@@ -556,7 +618,8 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
         // generic-proxy writes (zeroed rows, the fold's scratch) must be
         // ordered before the next TMA write into this stage
-        if (ts + kTileT > L || (kSplit > 1 && piece_end)) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        if ((!kConvert && ts + kTileT > L) || (kSplit > 1 && piece_end))
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[st]);
 

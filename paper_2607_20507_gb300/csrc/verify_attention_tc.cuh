@@ -23,12 +23,13 @@
 //           works on S_{t-1};
 //   warp 2  tensor-memory allocation (512 columns: four S/P buffers of 64,
 //           O in 128), so that QK can run up to three tiles ahead of PV;
+//   warps 2-3  the V tile of every stage from bf16 into fp16, in place;
 //   warps 4-7  softmax and epilogue, one query row per thread (warp 4+s
 //           owns tensor-memory lanes 32s..32s+31): mask, running max, exp2,
-//           row sum, P written back over S as fp16 (and the V tile turned
-//           from bf16 into fp16 in place, so that PV multiplies fp16 by fp16:
-//           bf16 P alone can exceed the output tolerance on rows whose terms
-//           cancel); O is rescaled in tensor
+//           row sum, P written back over S as fp16 (warps 2-3 turn each V
+//           tile into fp16, so PV multiplies fp16 by fp16: bf16 P alone can
+//           exceed the output tolerance on rows whose terms cancel); O is
+//           rescaled in tensor
 //           memory only when the running max grows by more than 2^8 (the
 //           stale max keeps every P below 256); at a span piece's end the
 //           row is normalised and written (bf16) or left as a partial.
@@ -158,7 +159,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     uint64_t* bars = reinterpret_cast<uint64_t*>(skv + kTcStages * kStageBytes);
     uint64_t* full = bars;                                  // [stages] K/V landed
     uint64_t* empty = bars + kTcMaxStages;                  // [stages] K/V consumed (PV done)
-    uint64_t* q_full = bars + 2 * kTcMaxStages;             // [2] Q of a span landed
+    uint64_t* ready = bars + 2 * kTcMaxStages;              // [stages] the stage's V is in fp16
+    uint64_t* q_full = bars + 3 * kTcMaxStages;             // [2] Q of a span landed
     uint64_t* q_free = q_full + 2;                          // [2] last QK of a span done
     uint64_t* s_full = q_free + 2;                          // [kTcSBuf] S_t in tensor memory
     uint64_t* s_free = s_full + kTcSBuf;                    // [kTcSBuf] P_t consumed (PV_t done)
@@ -171,6 +173,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     __shared__ long long s_carry;
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_dead;
+    __shared__ int s_keys[kTcMaxStages];   // keys of the tile in each stage (V rows past are zeroed)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = p.n_batch;
@@ -195,6 +198,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         for (int i = 0; i < kTcStages; ++i) {
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], 1);
+            mbar_init(&ready[i], 2);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(&q_full[i], 1);
@@ -271,60 +275,115 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         int pg_cur = batch_pages(0);
         int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
         int span = -1;
-        for (int j = 0; j < n_tiles; ++j) {
-            const int st = j % kTcStages;
-            const uint32_t use = (uint32_t)(j / kTcStages);
-            const int jb = j % per_batch;
-            if (j > 0 && jb == 0) {
-                pg_cur = pg_next;
-                pg_next = j + per_batch < n_tiles ? batch_pages(j + per_batch) : -1;
-            }
-            const int page = __shfl_sync(0xffffffffu, pg_cur, jb * kPieces + lane % kPieces);
-            const int L = s_len[cur.b];
-            const int ts = cur.t * kTileT;
-            const int h_cur = cur.h / p.n_rb;
-            int ok = 1;
-            if (lane == 0) {
-                if (j == 0 || cur.t == 0) {
-                    // a new span: its query rows into buffer span % 2, once
-                    // the span two back is done with it
-                    ++span;
-                    const int qb = span & 1;
-                    if (span >= 2 && !tc_wait(&q_free[qb], (uint32_t)((span - 2) >> 1) & 1, &s_dead, p.status)) ok = 0;
-                    if (ok) {
-                        mbar_arrive_expect_tx(&q_full[qb], 2 * qrow_bytes);
-                        const uint32_t qdst = smem_u32(sq + qb * 2 * qh);
+        // issue tile jt (and, opening a piece, its query rows) once its stage
+        // and the query buffer are free
+        int jt = 0;
+        uint32_t polls = 0;
+        uint64_t t_idle = 0;
+        while (jt < n_tiles) {
+            if (s_dead) break;
+            bool progress = false;
+            {
+                const int st = jt % kTcStages;
+                const bool first = jt == 0 || cur.t == 0;
+                const int sp = first ? span + 1 : span;
+                int go = 1;
+                if (lane == 0) {
+                    if (jt >= kTcStages) go = mbar_test_wait(&empty[st], (uint32_t)(jt / kTcStages - 1) & 1);
+                    if (go && first && sp >= 2) go = mbar_test_wait(&q_free[sp & 1], (uint32_t)((sp - 2) >> 1) & 1);
+                }
+                if (__shfl_sync(0xffffffffu, go, 0)) {
+                    const int jb = jt % per_batch;
+                    if (jt > 0 && jb == 0) {
+                        pg_cur = pg_next;
+                        pg_next = jt + per_batch < n_tiles ? batch_pages(jt + per_batch) : -1;
+                    }
+                    const int page = __shfl_sync(0xffffffffu, pg_cur, jb * kPieces + lane % kPieces);
+                    const int L = s_len[cur.b];
+                    const int ts = cur.t * kTileT;
+                    const int h_cur = cur.h / p.n_rb;
+                    if (first && lane == 0) {
+                        // a new span piece: its query rows into buffer sp % 2
+                        mbar_arrive_expect_tx(&q_full[sp & 1], 2 * qrow_bytes);
+                        const uint32_t qdst = smem_u32(sq + (sp & 1) * 2 * qh);
 #pragma unroll
                         for (int hh = 0; hh < 2; ++hh)
-                            tma_load_4d(qdst + hh * qh, &tmap_q, &q_full[qb], hh * 64, h_cur * p.G, 0,
+                            tma_load_4d(qdst + hh * qh, &tmap_q, &q_full[sp & 1], hh * 64, h_cur * p.G, 0,
                                         p.b_base + cur.b);
                     }
-                }
-                if (ok && j >= kTcStages && !tc_wait(&empty[st], (use - 1) & 1, &s_dead, p.status)) ok = 0;
-            }
-            advance(cur, s_len, nb, p.n_vh);
-            if (!__shfl_sync(0xffffffffu, ok, 0)) break;
-            int valid = 0;
-            for (int pc = 0; pc < kPieces; ++pc)
-                if (ts + pc * kBoxT < L) ++valid;
-            if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)valid * kPieceBytes * 2u);
-            __syncwarp();
-            if (lane < valid) {
-                const uint32_t kdst = smem_u32(skv + st * kStageBytes) + (uint32_t)lane * (kBoxT * 128);
-                const int slot = (ts + lane * kBoxT) % p.ps;
+                    span = sp;
+                    advance(cur, s_len, nb, p.n_vh);
+                    int valid = 0;
+                    for (int pc = 0; pc < kPieces; ++pc)
+                        if (ts + pc * kBoxT < L) ++valid;
+                    if (lane == 0) {
+                        s_keys[st] = max(0, min(kTileT, L - ts));
+                        mbar_arrive_expect_tx(&full[st], (uint32_t)valid * kPieceBytes * 2u);
+                    }
+                    __syncwarp();
+                    if (lane < valid) {
+                        const uint32_t kdst = smem_u32(skv + st * kStageBytes) + (uint32_t)lane * (kBoxT * 128);
+                        const int slot = (ts + lane * kBoxT) % p.ps;
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    tma_load_5d(kdst + hh * kTcHalfBytes, &tmap_k, &full[st], 0, slot, hh, h_cur, page);
-                    tma_load_5d(kdst + kTensorTileBytes + hh * kTcHalfBytes, &tmap_v, &full[st], 0, slot, hh, h_cur,
-                                page);
+                        for (int hh = 0; hh < 2; ++hh) {
+                            tma_load_5d(kdst + hh * kTcHalfBytes, &tmap_k, &full[st], 0, slot, hh, h_cur, page);
+                            tma_load_5d(kdst + kTensorTileBytes + hh * kTcHalfBytes, &tmap_v, &full[st], 0, slot, hh,
+                                        h_cur, page);
+                        }
+                    }
+                    ++jt;
+                    progress = true;
+                }
+            }
+            if (progress) {
+                polls = 0;
+            } else if ((++polls & 255u) == 0) {
+                const uint64_t now = global_timer_ns();
+                if (polls == 256) t_idle = now;
+                else if (now - t_idle > 1000000000ull) {   // about one second without progress
+                    if (lane == 0) {
+                        s_dead = 1;
+                        atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+                    }
+                    break;
                 }
             }
         }
-        // no copy in flight at exit: the last fill of every stage has landed
+        // no copy in flight at exit: every issued tile has landed
         if (lane == 0)
-            for (int j = n_tiles > kTcStages ? n_tiles - kTcStages : 0; j < n_tiles; ++j)
+            for (int j = jt > kTcStages ? jt - kTcStages : 0; j < jt; ++j)
                 if (!mbar_wait_bounded(&full[j % kTcStages], (uint32_t)(j / kTcStages) & 1))
                     atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+    } else if ((warp == 2 || warp == 3) && n_tiles > 0) {
+        // ------------------------------------------------------- V to fp16
+        // Each landed V tile is turned from bf16 into fp16 in place by these
+        // two warps (16-byte chunk i of the tile, laid out [dim half][64
+        // keys][128 B], holds key (i / 8) % 64; rows past L_b are zeroed),
+        // then released to PV through `ready`.
+        const int ct = (warp - 2) * 32 + lane;
+        for (int jc = 0; jc < n_tiles; ++jc) {
+            const int st = jc % kTcStages;
+            if (!tc_wait(&full[st], (uint32_t)(jc / kTcStages) & 1, &s_dead, p.status)) break;
+            const int keys = s_keys[st];
+            uint4* vt = reinterpret_cast<uint4*>(skv + st * kStageBytes + kTensorTileBytes);
+#pragma unroll 4
+            for (int i = ct; i < kTensorTileBytes / 16; i += 64) {
+                uint4 v = make_uint4(0, 0, 0, 0);
+                if (((i >> 3) & (kTileT - 1)) < keys) {
+                    v = vt[i];
+                    v.x = bf16x2_to_f16x2(v.x);
+                    v.y = bf16x2_to_f16x2(v.y);
+                    v.z = bf16x2_to_f16x2(v.z);
+                    v.w = bf16x2_to_f16x2(v.w);
+                }
+                vt[i] = v;
+            }
+            // generic writes the tensor core reads next (and the next TMA
+            // write into the stage follows them)
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&ready[st]);
+        }
     } else if (warp == 1 && n_tiles > 0) {
         // ---------------------------------------------------------- MMA
         // One thread, polling: QK of tile qt as soon as its K/V, its S buffer
@@ -376,6 +435,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                     const bool first = (fl_first >> sb) & 1u;
                     const int piece = fl_piece[sb];
                     if (mbar_test_wait(&p_full[sb], (uint32_t)(vt / kTcSBuf) & 1) &&
+                        mbar_test_wait(&ready[st], (uint32_t)(vt / kTcStages) & 1) &&
                         (!first || piece == 0 || mbar_test_wait(o_free, (uint32_t)(piece - 1) & 1))) {
                         tc_fence_after();
                         // O += P_vt V_vt, 4 steps of 16 keys, both dim halves per step
@@ -438,8 +498,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         };
         begin_span(cur);
         for (int t = 0; t < n_tiles; ++t) {
-            const int sb = t % kTcSBuf, st = t % kTcStages;
-            const int L = s_len[cur.b];
+            const int sb = t % kTcSBuf;
             const int ts = cur.t * kTileT;
             const bool piece_end = t + 1 == n_tiles || cur.t + 1 == cur.T;
             if (!tc_wait(&s_full[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) break;
@@ -510,28 +569,6 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             }
             tc_st32(t_row + sb * 64, pk);
             tc_wait_st();
-            // the V tile into fp16, in place: each thread owns 8 of its 1024
-            // 16-byte chunks (the swizzle only permutes chunks within a
-            // 128-byte row, so a chunk's key is its row); rows past L_b may
-            // hold any bits and are zeroed instead
-            {
-                uint4* vt = reinterpret_cast<uint4*>(skv + st * kStageBytes + kTensorTileBytes);
-                const int keys = min(kTileT, L - ts);
-#pragma unroll
-                for (int i = 0; i < kTensorTileBytes / 16 / 128; ++i) {
-                    const int ci = i * 128 + sub * 32 + lane;
-                    uint4 v = make_uint4(0, 0, 0, 0);
-                    if (((ci >> 3) & (kTileT - 1)) < keys) {
-                        v = vt[ci];
-                        v.x = bf16x2_to_f16x2(v.x);
-                        v.y = bf16x2_to_f16x2(v.y);
-                        v.z = bf16x2_to_f16x2(v.z);
-                        v.w = bf16x2_to_f16x2(v.w);
-                    }
-                    vt[ci] = v;
-                }
-            }
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&p_full[sb]);
