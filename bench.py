@@ -42,6 +42,7 @@ NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 512 << 20
 KERNEL_SOURCES = ("paper_2607_20507_gb300/csrc/verify_attention.cu",
+                  "paper_2607_20507_gb300/csrc/verify_attention_tc.cuh",
                   "paper_2607_20507_gb300/csrc/spec_accept.cu",
                   "paper_2607_20507_gb300/csrc/cs_device.cuh")
 
