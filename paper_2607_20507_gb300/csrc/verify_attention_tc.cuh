@@ -13,16 +13,21 @@
 //           follows, which only feeds padded rows) and the K/V tiles of the
 //           range through a ring of as many 32 KB stages as shared memory
 //           then holds (4-6), one box per page piece and dim half, so a tile
-//           lands as [dim half][64 keys][128 B], 128-byte swizzle;
-//   warp 1  MMA issuer (one thread): S_t = Q K_t^T into tensor memory
-//           (M = 128 padded rows, N = 64 keys, K-major operands, 8 steps of
-//           16 dims), then O += P_{t-1} V_{t-1} (N = 128 dims, 4 steps of 16
-//           keys) with P read from tensor memory and V an MN-major operand
-//           whose two dim halves lie one leading offset apart -- one tile
-//           behind, so that the tensor core computes S_t while the softmax
-//           works on S_{t-1};
+//           lands as [dim half][64 keys][128 B], 128-byte swizzle; beside
+//           each stage it leaves whether the tile opens or closes a piece;
+//   warp 1  MMA issuer (the whole warp waits, one elected lane issues;
+//           fixed order): at a piece's start the query rows from shared into
+//           tensor memory (tcgen05.cp, one buffer per span parity), then per
+//           tile S_t = Q K_t^T into tensor memory (M = 128 padded rows,
+//           N = 64 keys, Q from tensor memory, K a K-major shared-memory
+//           operand, 8 steps of 16 dims) and O += P_t V_t
+//           (N = 128 dims, 4 steps of 16 keys) with P read from tensor
+//           memory and V an MN-major operand whose two dim halves lie one
+//           leading offset apart; QK runs two tiles ahead of PV, so that the
+//           tensor core computes S_{t+1} and S_{t+2} while the softmax works
+//           on S_t;
 //   warp 2  tensor-memory allocation (512 columns: four S/P buffers of 64,
-//           O in 128), so that QK can run up to three tiles ahead of PV;
+//           O in 128, two query buffers of 64);
 //   warps 2-3  the V tile of every stage from bf16 into fp16, in place;
 //   warps 4-7  softmax and epilogue, one query row per thread (warp 4+s
 //           owns tensor-memory lanes 32s..32s+31): mask, running max, exp2,
@@ -42,7 +47,8 @@ constexpr int kTcRows = 128;                       // MMA M: query rows, padded
 constexpr int kTcMinRows = 48;                     // fewer query rows take the mma.sync form
 constexpr int kTcSBuf = 4;                         // S/P buffers in tensor memory
 constexpr int kTcOCol = kTcSBuf * 64;              // first column of O
-constexpr int kTcTmemCols = 512;                   // S/P [0, 256) in four buffers, O [256, 384)
+constexpr int kTcQCol = kTcOCol + 128;             // first column of the two query buffers (64 each)
+constexpr int kTcTmemCols = 512;                   // S/P [0, 256) in four buffers, O [256, 384), Q [384, 512)
 constexpr int kTcBarBytes = 512;
 constexpr int kTcFixedSmem = kTcBarBytes + (kMaxBatchPerLaunch + 1) * 8 + kMaxBatchPerLaunch * 4 + 1024;
 constexpr int kTcSmemLimit = 232448 - 256;         // opt-in shared memory per block, less the static part
@@ -80,6 +86,23 @@ __device__ __forceinline__ uint64_t tc_mn_desc(uint32_t addr) {
 __host__ __device__ constexpr uint32_t tc_idesc(int n, bool b_mn, bool f16) {
     return (1u << 4) | (f16 ? 0u : (1u << 7) | (1u << 10)) | (b_mn ? (1u << 16) : 0u) | ((uint32_t)(n >> 3) << 17) |
            ((uint32_t)(kTcRows >> 4) << 24);
+}
+
+// One lane of the (converged) warp, the same one every time: the lowest.
+__device__ __forceinline__ bool elect_one() {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred P;\n\telect.sync _|P, 0xffffffff;\n\tselp.u32 %0, 1, 0, P;\n\t}\n"
+        : "=r"(r));
+    return r != 0;
+}
+
+// 128 rows x 32 bytes of a K-major shared-memory operand (the same
+// descriptor the MMA would read it through) into 128 lanes x 8 columns of
+// tensor memory, laid out as an A operand from tensor memory.  Executes in
+// issue order with the MMAs of the same thread that follow it.
+__device__ __forceinline__ void tc_cp_128x256b(uint32_t taddr, uint64_t sdesc) {
+    asm volatile("tcgen05.cp.cta_group::1.128x256b [%0], %1;" ::"r"(taddr), "l"(sdesc) : "memory");
 }
 
 __device__ __forceinline__ void tc_commit(uint64_t* bar) {
@@ -135,6 +158,7 @@ __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::
 
 // Bounded wait that also gives up at once when another warp already has.
 __device__ __forceinline__ bool tc_wait(uint64_t* bar, uint32_t parity, volatile int* dead, int* status) {
+    if (mbar_test_wait(bar, parity)) return true;
     if (*dead) return false;
     if (mbar_wait_bounded(bar, parity)) return true;
     *dead = 1;
@@ -163,9 +187,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     uint64_t* q_full = bars + 3 * kTcMaxStages;             // [2] Q of a span landed
     uint64_t* q_free = q_full + 2;                          // [2] last QK of a span done
     uint64_t* s_full = q_free + 2;                          // [kTcSBuf] S_t in tensor memory
-    uint64_t* s_free = s_full + kTcSBuf;                    // [kTcSBuf] P_t consumed (PV_t done)
-    uint64_t* p_full = s_free + kTcSBuf;                    // [kTcSBuf] P_t written (count 4 warps)
-    uint64_t* o_ready = p_full + kTcSBuf;                   // [kTcSBuf] PV_t done, by S buffer
+    uint64_t* p_full = s_full + kTcSBuf;                    // [kTcSBuf] P_t written (count 4 warps)
+    uint64_t* o_ready = p_full + kTcSBuf;                   // [kTcSBuf] PV_t done (S buffer free again)
     uint64_t* o_free = o_ready + kTcSBuf;                   // O read out by the epilogue (count 4 warps)
     long long* s_prefix = reinterpret_cast<long long*>(reinterpret_cast<uint8_t*>(bars) + kTcBarBytes);
     int* s_len = reinterpret_cast<int*>(s_prefix + kMaxBatchPerLaunch + 1);
@@ -174,6 +197,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_dead;
     __shared__ int s_keys[kTcMaxStages];   // keys of the tile in each stage (V rows past are zeroed)
+    __shared__ int s_info[kTcMaxStages];   // bit 0: the stage's tile opens a span piece, bit 1: ends one
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = p.n_batch;
@@ -206,7 +230,6 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         }
         for (int i = 0; i < kTcSBuf; ++i) {
             mbar_init(&s_full[i], 1);
-            mbar_init(&s_free[i], 1);
             mbar_init(&p_full[i], 4);
             mbar_init(&o_ready[i], 1);
         }
@@ -275,77 +298,53 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         int pg_cur = batch_pages(0);
         int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
         int span = -1;
-        // issue tile jt (and, opening a piece, its query rows) once its stage
-        // and the query buffer are free
+        // tile jt goes out once its stage is free and, opening a piece, once
+        // the query buffer it reuses is free
         int jt = 0;
-        uint32_t polls = 0;
-        uint64_t t_idle = 0;
-        while (jt < n_tiles) {
-            if (s_dead) break;
-            bool progress = false;
-            {
-                const int st = jt % kTcStages;
-                const bool first = jt == 0 || cur.t == 0;
-                const int sp = first ? span + 1 : span;
-                int go = 1;
-                if (lane == 0) {
-                    if (jt >= kTcStages) go = mbar_test_wait(&empty[st], (uint32_t)(jt / kTcStages - 1) & 1);
-                    if (go && first && sp >= 2) go = mbar_test_wait(&q_free[sp & 1], (uint32_t)((sp - 2) >> 1) & 1);
-                }
-                if (__shfl_sync(0xffffffffu, go, 0)) {
-                    const int jb = jt % per_batch;
-                    if (jt > 0 && jb == 0) {
-                        pg_cur = pg_next;
-                        pg_next = jt + per_batch < n_tiles ? batch_pages(jt + per_batch) : -1;
-                    }
-                    const int page = __shfl_sync(0xffffffffu, pg_cur, jb * kPieces + lane % kPieces);
-                    const int L = s_len[cur.b];
-                    const int ts = cur.t * kTileT;
-                    const int h_cur = cur.h / p.n_rb;
-                    if (first && lane == 0) {
-                        // a new span piece: its query rows into buffer sp % 2
-                        mbar_arrive_expect_tx(&q_full[sp & 1], 2 * qrow_bytes);
-                        const uint32_t qdst = smem_u32(sq + (sp & 1) * 2 * qh);
-#pragma unroll
-                        for (int hh = 0; hh < 2; ++hh)
-                            tma_load_4d(qdst + hh * qh, &tmap_q, &q_full[sp & 1], hh * 64, h_cur * p.G, 0,
-                                        p.b_base + cur.b);
-                    }
-                    span = sp;
-                    advance(cur, s_len, nb, p.n_vh);
-                    int valid = 0;
-                    for (int pc = 0; pc < kPieces; ++pc)
-                        if (ts + pc * kBoxT < L) ++valid;
-                    if (lane == 0) {
-                        s_keys[st] = max(0, min(kTileT, L - ts));
-                        mbar_arrive_expect_tx(&full[st], (uint32_t)valid * kPieceBytes * 2u);
-                    }
-                    __syncwarp();
-                    if (lane < valid) {
-                        const uint32_t kdst = smem_u32(skv + st * kStageBytes) + (uint32_t)lane * (kBoxT * 128);
-                        const int slot = (ts + lane * kBoxT) % p.ps;
-#pragma unroll
-                        for (int hh = 0; hh < 2; ++hh) {
-                            tma_load_5d(kdst + hh * kTcHalfBytes, &tmap_k, &full[st], 0, slot, hh, h_cur, page);
-                            tma_load_5d(kdst + kTensorTileBytes + hh * kTcHalfBytes, &tmap_v, &full[st], 0, slot, hh,
-                                        h_cur, page);
-                        }
-                    }
-                    ++jt;
-                    progress = true;
-                }
+        for (; jt < n_tiles; ++jt) {
+            const int st = jt % kTcStages;
+            const bool first = jt == 0 || cur.t == 0;
+            const bool last = jt + 1 == n_tiles || cur.t + 1 == cur.T;
+            if (first) ++span;
+            bool go = jt < kTcStages || tc_wait(&empty[st], (uint32_t)(jt / kTcStages - 1) & 1, &s_dead, p.status);
+            if (go && first && span >= 2)
+                go = tc_wait(&q_free[span & 1], (uint32_t)((span - 2) >> 1) & 1, &s_dead, p.status);
+            if (!__all_sync(0xffffffffu, go)) break;
+            const int jb = jt % per_batch;
+            if (jt > 0 && jb == 0) {
+                pg_cur = pg_next;
+                pg_next = jt + per_batch < n_tiles ? batch_pages(jt + per_batch) : -1;
             }
-            if (progress) {
-                polls = 0;
-            } else if ((++polls & 255u) == 0) {
-                const uint64_t now = global_timer_ns();
-                if (polls == 256) t_idle = now;
-                else if (now - t_idle > 1000000000ull) {   // about one second without progress
-                    if (lane == 0) {
-                        s_dead = 1;
-                        atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-                    }
-                    break;
+            const int page = __shfl_sync(0xffffffffu, pg_cur, jb * kPieces + lane % kPieces);
+            const int L = s_len[cur.b];
+            const int ts = cur.t * kTileT;
+            const int h_cur = cur.h / p.n_rb;
+            if (first && lane == 0) {
+                // a new span piece: its query rows into buffer span % 2
+                mbar_arrive_expect_tx(&q_full[span & 1], 2 * qrow_bytes);
+                const uint32_t qdst = smem_u32(sq + (span & 1) * 2 * qh);
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh)
+                    tma_load_4d(qdst + hh * qh, &tmap_q, &q_full[span & 1], hh * 64, h_cur * p.G, 0, p.b_base + cur.b);
+            }
+            advance(cur, s_len, nb, p.n_vh);
+            int valid = 0;
+            for (int pc = 0; pc < kPieces; ++pc)
+                if (ts + pc * kBoxT < L) ++valid;
+            if (lane == 0) {
+                s_keys[st] = max(0, min(kTileT, L - ts));
+                s_info[st] = (first ? 1 : 0) | (last ? 2 : 0);
+                mbar_arrive_expect_tx(&full[st], (uint32_t)valid * kPieceBytes * 2u);
+            }
+            __syncwarp();
+            if (lane < valid) {
+                const uint32_t kdst = smem_u32(skv + st * kStageBytes) + (uint32_t)lane * (kBoxT * 128);
+                const int slot = (ts + lane * kBoxT) % p.ps;
+#pragma unroll
+                for (int hh = 0; hh < 2; ++hh) {
+                    tma_load_5d(kdst + hh * kTcHalfBytes, &tmap_k, &full[st], 0, slot, hh, h_cur, page);
+                    tma_load_5d(kdst + kTensorTileBytes + hh * kTcHalfBytes, &tmap_v, &full[st], 0, slot, hh, h_cur,
+                                page);
                 }
             }
         }
@@ -359,7 +358,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // Each landed V tile is turned from bf16 into fp16 in place by these
         // two warps (16-byte chunk i of the tile, laid out [dim half][64
         // keys][128 B], holds key (i / 8) % 64; rows past L_b are zeroed),
-        // then released to PV through `ready`.
+        // then released through `ready`, which the softmax checks before it
+        // hands P_t to the MMA warp.
         const int ct = (warp - 2) * 32 + lane;
         for (int jc = 0; jc < n_tiles; ++jc) {
             const int st = jc % kTcStages;
@@ -386,87 +386,103 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         }
     } else if (warp == 1 && n_tiles > 0) {
         // ---------------------------------------------------------- MMA
-        // One thread, polling: QK of tile qt as soon as its K/V, its S buffer
-        // and (first tile of a piece) its query rows are ready, up to
-        // kTcSBuf - 1 tiles ahead of PV; PV of tile vt as soon as its P is
-        // written and (first tile of a piece) the previous piece's epilogue
-        // has read O.  Each readiness probe names a phase its barrier can be
-        // at most one phase short of, so a parity probe is exact.
-        if (lane == 0) {
-            const uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, true);
-            Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
-            int qt = 0, vt = 0, span = -1;
-            uint32_t fl_first = 0;          // bit sb: the tile in S buffer sb opened its piece
-            int fl_piece[kTcSBuf] = {};     // piece of the tile in each S buffer
-            uint64_t t_progress = global_timer_ns();
-            uint32_t polls = 0;
-            while (vt < n_tiles) {
-                if (s_dead) break;
-                bool progress = false;
-                if (qt < n_tiles && qt - vt < kTcSBuf) {
-                    const bool first = qt == 0 || cur.t == 0;
-                    const int sp = first ? span + 1 : span;
-                    const int st = qt % kTcStages, sb = qt % kTcSBuf;
-                    if ((!first || mbar_test_wait(&q_full[sp & 1], (uint32_t)(sp >> 1) & 1)) &&
-                        mbar_test_wait(&full[st], (uint32_t)(qt / kTcStages) & 1) &&
-                        (qt < kTcSBuf || mbar_test_wait(&s_free[sb], (uint32_t)((qt - kTcSBuf) / kTcSBuf) & 1))) {
-                        span = sp;
-                        tc_fence_after();
-                        // S_qt = Q K_qt^T, 8 steps of 16 dims
-                        const uint32_t qbase = smem_u32(sq + (span & 1) * 2 * qh);
-                        const uint32_t kbase = smem_u32(skv + st * kStageBytes);
+        // A fixed order: QK_0, QK_1, then PV_t followed by
+        // QK_{t+2} -- S_{t+1} is in tensor memory while the softmax works on
+        // S_t, and S_{t+2} is computed while it works on S_{t+1}.  Each wait
+        // names a phase its barrier can be at most one phase short of (the
+        // next phase needs an MMA this warp has not issued yet), so a parity
+        // wait is exact.  Descriptors advance by constant offsets (addresses
+        // stay below 256 KB, so the 14-bit start field cannot carry).  The
+        // whole warp runs the loop and waits; lane 0 issues the MMAs and the
+        // commits (a lone lane beside 31 parked at the block barrier pays
+        // hundreds of cycles per barrier probe and per tcgen05 instruction).
+        {
+            constexpr uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, true);
+            const uint64_t dq0 = tc_sw128_desc(smem_u32(sq));
+            const uint64_t qbuf16 = (uint64_t)(2 * qh) >> 4, qhalf16 = (uint64_t)qh >> 4;
+            const uint64_t dkv0 = tc_sw128_desc(smem_u32(skv)), dv0 = tc_mn_desc(smem_u32(skv + kTensorTileBytes));
+            uint32_t first_bits = 0;        // bit sb: the tile in S buffer sb opened its piece
+            int span = -1, pv_piece = 0;
+            uint64_t* last_bar = nullptr;   // the latest commit: completes after every MMA issued
+            uint32_t last_par = 0;
+            // every lane waits; the result is made warp-uniform, so that no lane
+            // leaves the loop while another still issues
+            auto wait_all = [&](uint64_t* bar, uint32_t par, volatile int* dead, int* status) -> bool {
+                return __all_sync(0xffffffffu, tc_wait(bar, par, dead, status));
+            };
+            auto issue_qk = [&](int t) -> bool {
+                const int st = t % kTcStages, sb = t % kTcSBuf;
+                if (!wait_all(&full[st], (uint32_t)(t / kTcStages) & 1, &s_dead, p.status)) return false;
+                const int info = s_info[st];
+                if (info & 1) {
+                    // a new piece: its query rows landed, and the QKs of the
+                    // piece two back are done reading the query buffer
+                    ++span;
+                    if (!wait_all(&q_full[span & 1], (uint32_t)(span >> 1) & 1, &s_dead, p.status)) return false;
+                    if (span >= 2 && !wait_all(&q_free[span & 1], (uint32_t)((span - 2) >> 1) & 1, &s_dead, p.status))
+                        return false;
+                }
+                // S buffer sb held S_{t-4}: PV_{t-4} is done with it
+                if (t >= kTcSBuf && !wait_all(&o_ready[sb], (uint32_t)((t - kTcSBuf) / kTcSBuf) & 1, &s_dead, p.status))
+                    return false;
+                tc_fence_after();
+                const uint32_t tq = tmem + kTcQCol + (span & 1) * 64;
+                const uint64_t dk = dkv0 + (uint64_t)((st * kStageBytes) >> 4);
+                if (elect_one()) {
+                    if (info & 1) {
+                        // the query rows into tensor memory once per piece, 16
+                        // dims (8 columns) per copy; every QK of the piece then
+                        // reads only K from shared memory
+                        const uint64_t dq = dq0 + (span & 1) * qbuf16;
 #pragma unroll
-                        for (int ks = 0; ks < kD / 16; ++ks) {
-                            const int hh = ks >> 2, kc = (ks & 3) * 32;
-                            tc_mma_ss(tmem + sb * 64, tc_sw128_desc(qbase + hh * qh + kc),
-                                      tc_sw128_desc(kbase + hh * kTcHalfBytes + kc), id_s, ks > 0 ? 1u : 0u);
-                        }
-                        tc_commit(&s_full[sb]);
-                        if (qt + 1 == n_tiles || cur.t + 1 == cur.T) tc_commit(&q_free[span & 1]);
-                        fl_first = first ? (fl_first | (1u << sb)) : (fl_first & ~(1u << sb));
-                        fl_piece[sb] = span;
-                        advance(cur, s_len, nb, p.n_vh);
-                        ++qt;
-                        progress = true;
+                        for (int ks = 0; ks < kD / 16; ++ks)
+                            tc_cp_128x256b(tq + ks * 8, dq + (ks >> 2) * qhalf16 + (uint64_t)((ks & 3) * 2));
                     }
-                }
-                if (vt < qt) {
-                    const int st = vt % kTcStages, sb = vt % kTcSBuf;
-                    const bool first = (fl_first >> sb) & 1u;
-                    const int piece = fl_piece[sb];
-                    if (mbar_test_wait(&p_full[sb], (uint32_t)(vt / kTcSBuf) & 1) &&
-                        mbar_test_wait(&ready[st], (uint32_t)(vt / kTcStages) & 1) &&
-                        (!first || piece == 0 || mbar_test_wait(o_free, (uint32_t)(piece - 1) & 1))) {
-                        tc_fence_after();
-                        // O += P_vt V_vt, 4 steps of 16 keys, both dim halves per step
-                        const uint32_t vbase = smem_u32(skv + st * kStageBytes + kTensorTileBytes);
 #pragma unroll
-                        for (int kk = 0; kk < kTileT / 16; ++kk)
-                            tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + kk * 8, tc_mn_desc(vbase + kk * 16 * 128),
-                                      id_o, (first && kk == 0) ? 0u : 1u);
-                        tc_commit(&o_ready[sb]);
-                        tc_commit(&empty[st]);
-                        tc_commit(&s_free[sb]);
-                        ++vt;
-                        progress = true;
+                    for (int ks = 0; ks < kD / 16; ++ks) {
+                        const uint64_t ko = (uint64_t)((((ks >> 2) * kTcHalfBytes) >> 4) + (ks & 3) * 2);
+                        tc_mma_ts(tmem + sb * 64, tq + ks * 8, dk + ko, id_s, ks > 0 ? 1u : 0u);
                     }
+                    tc_commit(&s_full[sb]);
+                    if (info & 2) tc_commit(&q_free[span & 1]);
                 }
-                if (progress) {
-                    polls = 0;
-                } else if ((++polls & 255u) == 0) {
-                    const uint64_t now = global_timer_ns();
-                    if (polls == 256) t_progress = now;
-                    else if (now - t_progress > 1000000000ull) {   // about one second without progress
-                        s_dead = 1;
-                        atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-                        break;
-                    }
+                __syncwarp();
+                last_bar = &s_full[sb];
+                last_par = (uint32_t)(t / kTcSBuf) & 1;
+                first_bits = (info & 1) ? (first_bits | (1u << sb)) : (first_bits & ~(1u << sb));
+                return true;
+            };
+            auto issue_pv = [&](int t) -> bool {
+                const int st = t % kTcStages, sb = t % kTcSBuf;
+                if (!wait_all(&p_full[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) return false;
+                const bool first = (first_bits >> sb) & 1u;
+                if (first) {
+                    // the previous piece's epilogue has read O
+                    if (pv_piece > 0 && !wait_all(o_free, (uint32_t)(pv_piece - 1) & 1, &s_dead, p.status))
+                        return false;
+                    ++pv_piece;
                 }
-            }
-            // every MMA of this CTA completes before tensor memory is freed:
-            // the last PV of each S buffer is the latest phase of its barrier
-            for (int t = vt >= kTcSBuf ? vt - kTcSBuf : 0; t < vt; ++t)
-                if (!mbar_wait_bounded(&o_ready[t % kTcSBuf], (uint32_t)(t / kTcSBuf) & 1)) break;
+                tc_fence_after();
+                // O += P_t V_t, 4 steps of 16 keys, both dim halves per step
+                const uint64_t dv = dv0 + (uint64_t)((st * kStageBytes) >> 4);
+                if (elect_one()) {
+#pragma unroll
+                    for (int kk = 0; kk < kTileT / 16; ++kk)
+                        tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + kk * 8, dv + (uint64_t)(kk * ((16 * 128) >> 4)),
+                                  id_o, (first && kk == 0) ? 0u : 1u);
+                    tc_commit(&o_ready[sb]);
+                    tc_commit(&empty[st]);
+                }
+                __syncwarp();
+                last_bar = &o_ready[sb];
+                last_par = (uint32_t)(t / kTcSBuf) & 1;
+                return true;
+            };
+            bool ok = issue_qk(0) && (n_tiles < 2 || issue_qk(1));
+            for (int t = 0; ok && t < n_tiles; ++t) ok = issue_pv(t) && (t + 2 >= n_tiles || issue_qk(t + 2));
+            // every MMA of this CTA completes before tensor memory is freed
+            if (last_bar != nullptr && !mbar_wait_bounded(last_bar, last_par) && lane == 0)
+                atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
         }
     } else if (warp >= 4 && n_tiles > 0) {
         // ---------------------------------------------------- softmax, epilogue
@@ -525,11 +541,19 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 }
             } else {
                 const int lim_t = lim - ts;   // keys e < lim_t are visible
+                if (lim_t < 64) {
 #pragma unroll
-                for (int e = 0; e < 64; ++e) {
-                    if (e >= lim_t) s[e] = kNegInf;
-                    mt = fmaxf(mt, s[e]);
+                    for (int e = 0; e < 64; ++e)
+                        if (e >= lim_t) s[e] = kNegInf;
                 }
+                // eight independent chains: the maximum is exact in any order
+                float m8[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) m8[j] = fmaxf(s[j], s[j + 8]);
+#pragma unroll
+                for (int e = 16; e < 64; ++e) m8[e & 7] = fmaxf(m8[e & 7], s[e]);
+                mt = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                           fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
             }
             // ---- running max, lazily: O is rescaled only for a growth > 2^8
             float alpha = 1.f;
@@ -538,14 +562,15 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 m_run = mt;
             }
             const float neg = m_run == kNegInf ? 0.f : -m_run * c;
-            float rs = 0.f;
+            float r4[4] = {0.f, 0.f, 0.f, 0.f};
             uint32_t pk[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
                 const float p0 = ex2(fmaf(s[2 * e], c, neg)), p1 = ex2(fmaf(s[2 * e + 1], c, neg));
-                rs += p0 + p1;
+                r4[e & 3] += p0 + p1;
                 pk[e] = pack_f16x2(p0, p1);
             }
+            const float rs = (r4[0] + r4[1]) + (r4[2] + r4[3]);
             l_run = l_run * alpha + rs;
             // ---- a rescale of O waits for PV_{t-1}; the first tile of a piece
             // needs none (its PV overwrites O).  o_ready[b] completes once per
@@ -570,7 +595,12 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             tc_st32(t_row + sb * 64, pk);
             tc_wait_st();
             tc_fence_before();
-            __syncwarp();
+            // P_t goes to the MMA warp once the tile's V is in fp16 too (the
+            // PV reads both).  The next phase of `ready` needs the stage
+            // back, i.e. this PV, so the parity names one phase.
+            const bool v_ok = lane != 0 || tc_wait(&ready[t % kTcStages], (uint32_t)(t / kTcStages) & 1, &s_dead,
+                                                   p.status);
+            if (!__all_sync(0xffffffffu, v_ok)) break;
             if (lane == 0) mbar_arrive(&p_full[sb]);
 
             if (!piece_end) {
