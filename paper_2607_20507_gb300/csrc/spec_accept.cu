@@ -215,9 +215,9 @@ __device__ __forceinline__ long long range_lo(const AcceptParams& p, long long w
     return div_nn(w * p.N, p.W);
 }
 
-// Programmatic dependent launch: the draw kernel may start while the
-// statistics kernel runs; it waits here before reading what that kernel
-// wrote (a no-op when it was launched without the attribute).
+// Programmatic dependent launch: each kernel may start while the one before
+// it runs; it waits here before reading what that kernel wrote (a no-op
+// when it was launched without the attribute).
 __device__ __forceinline__ void wait_prior_grid() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void allow_dependent_launch() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -288,6 +288,10 @@ __global__ void __launch_bounds__(kThreads, 2) accept_stats_kernel(const AcceptP
     constexpr int kItem = kItemBytes / (int)sizeof(T);
     const int lane = threadIdx.x & 31;
     const long long w = (long long)blockIdx.x * kWarps + (threadIdx.x >> 5);
+    // launched as a programmatic dependent of the kernel before it: its
+    // inputs are read only past this wait, and the second kernel (which
+    // reads some inputs before its own wait) only starts after it
+    wait_prior_grid();
     allow_dependent_launch();
     if (w >= p.W) return;
     const long long lo = range_lo(p, w), hi = range_lo(p, w + 1);
@@ -747,6 +751,7 @@ __global__ void __launch_bounds__(kDrawThreads, 2) accept_draw_kernel(const Acce
 
     // ---- row statistics of the request (kernel 1's output), then the tests
     wait_prior_grid();
+    allow_dependent_launch();   // the next call's first kernel may start
     fold_rows<false, kRowsPerDrawWarp>(p, b, wid, kDrawWarps, p.R, lane, s_stat);
     __syncthreads();
     if (wid == 0) {
@@ -806,9 +811,10 @@ __global__ void __launch_bounds__(kThreads) accept_greedy_kernel(const AcceptPar
     __shared__ float2 s_stat[kWarps][kMaxRows];
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     const int b = blockIdx.x * kWarps + wid;
-    if (b >= p.B) return;
     const int k = p.k;
     wait_prior_grid();
+    allow_dependent_launch();   // the next call's first kernel may start
+    if (b >= p.B) return;
     fold_rows<true, 4>(p, b, 0, 1, k + 1, lane, s_stat[wid]);
     __syncwarp();
     int g = 0, x = -1;
@@ -905,6 +911,7 @@ __global__ void __launch_bounds__(kDrawThreads, 2) tree_draw_kernel(const Accept
         s_kids[u] = m;
     }
     wait_prior_grid();
+    allow_dependent_launch();   // the next call's first kernel may start
     fold_rows<false, 8>(p, b, tid >> 5, kDrawWarps, p.R, lane, s_stat);
     __syncthreads();
 
@@ -1015,6 +1022,7 @@ __global__ void __launch_bounds__(kThreads) tree_greedy_kernel(const AcceptParam
         }
     }
     wait_prior_grid();
+    allow_dependent_launch();   // the next call's first kernel may start
     fold_rows<true, 4>(p, b, 0, 1, n, lane, s_stat[wid]);
     __syncwarp();
     int32_t* out = p.out_tokens + (size_t)b * n;
@@ -1163,15 +1171,23 @@ AcceptPlan plan_accept(const cs_accept_dims& d, int n_draft, bool greedy, bool w
 
 template <typename T, bool G>
 cs_status launch_typed(AcceptParams p, const AcceptPlan& P, bool tree, cudaStream_t stream) {
-    accept_stats_kernel<T, G><<<P.grid1, kThreads, 0, stream>>>(p);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return cuda_fail(e, "accept_stats_kernel launch");
-    // the second kernel is launched as a programmatic dependent of the first:
-    // it may start early and waits (griddepcontrol.wait) before reading the
-    // partials
+    // both kernels are programmatic dependents of the kernel before them:
+    // each may start early and waits (griddepcontrol.wait) before it reads
+    // what that kernel wrote
     cudaLaunchAttribute attrs[2];
     attrs[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attrs[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaError_t e;
+    {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)P.grid1, 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.stream = stream;
+        cfg.attrs = attrs;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, accept_stats_kernel<T, G>, p);
+        if (e != cudaSuccess) return cuda_fail(e, "accept_stats_kernel launch");
+    }
     if (G) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3((p.B + kWarps - 1) / kWarps, 1, 1);

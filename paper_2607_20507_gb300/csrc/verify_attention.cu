@@ -190,10 +190,6 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nw = p.row_warps;
     const int nb = p.n_batch;
-    // the merge kernel is a programmatic dependent: let it start (and work out
-    // its schedule) while this kernel runs
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-
     // the page table of this launch into L2, spread over the CTAs, while the
     // schedule is computed (the producer's first lookups then hit L2)
     if (warp == kSplit * nw) {
@@ -215,6 +211,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         mbar_init(fold_b, nw);
         fence_barrier_init();
     }
+    // launched as a programmatic dependent of the kernel before it: the
+    // prologue above overlaps that kernel, every input is read below.  The
+    // merge kernel (this kernel's dependent) may then start and work out its
+    // schedule while this one runs.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     __syncthreads();
     const int l_cap = p.max_pages * p.ps;
     for (int base = 0; base < nb; base += blockDim.x) {
@@ -752,10 +754,14 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     }
     __syncthreads();
     const int n_p = s_np;
-    if (n_p <= 1) return;   // written whole by the main kernel
     // everything above depends only on the context lengths; the pieces are
-    // the main kernel's output
+    // the main kernel's output.  Every CTA waits, even one with nothing to
+    // merge, so that this grid never completes before the main kernel (a
+    // programmatic dependent of this kernel may rely on that), then lets the
+    // next kernel of the stream start.
     asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (n_p <= 1) return;   // written whole by the main kernel
 
     const int bg = p.b_base + bl;
     const int head = h / p.n_rb, rbase = (h - head * p.n_rb) * p.n_rows;
@@ -883,6 +889,24 @@ int tc_resident_per_sm() {
 }
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// A launch that may start while the kernel before it in the stream runs
+// (the kernel waits with griddepcontrol.wait before it reads its inputs).
+template <typename... Args, typename... Params>
+cudaError_t launch_dependent(void (*kern)(Params...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                             Args... args) {
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
 
 // The split merge as a programmatic dependent of the main kernel: it may
 // start early and waits (griddepcontrol.wait) before it reads the partials.
@@ -1051,8 +1075,7 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
         for (int b0 = 0; b0 < d.batch; b0 += kMaxBatchPerLaunch) {
             p.b_base = b0;
             p.n_batch = d.batch - b0 < kMaxBatchPerLaunch ? d.batch - b0 : kMaxBatchPerLaunch;
-            tk_fn<<<pl.grid, kTcThreads, smem_bytes, stream>>>(tk, tv, tq, p);
-            e = cudaGetLastError();
+            e = launch_dependent(tk_fn, dim3(pl.grid), dim3(kTcThreads), (size_t)smem_bytes, stream, tk, tv, tq, p);
             if (e != cudaSuccess) return cuda_fail(e, "verify_attention_tc_kernel launch");
             e = launch_merge(p, pl, stream);
             if (e != cudaSuccess) return cuda_fail(e, "verify_attention_merge_kernel launch");
@@ -1089,8 +1112,7 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     for (int b0 = 0; b0 < d.batch; b0 += kMaxBatchPerLaunch) {
         p.b_base = b0;
         p.n_batch = d.batch - b0 < kMaxBatchPerLaunch ? d.batch - b0 : kMaxBatchPerLaunch;
-        kern<<<pl.grid, block, kSmemBytes, stream>>>(tk, tv, p);
-        e = cudaGetLastError();
+        e = launch_dependent(kern, dim3(pl.grid), block, (size_t)kSmemBytes, stream, tk, tv, p);
         if (e != cudaSuccess) return cuda_fail(e, "verify_attention_kernel launch");
         e = launch_merge(p, pl, stream);
         if (e != cudaSuccess) return cuda_fail(e, "verify_attention_merge_kernel launch");

@@ -201,7 +201,6 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = p.n_batch;
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (warp == 0) {
         // the page table of this launch into L2 while the schedule is computed
@@ -236,6 +235,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         mbar_init(o_free, 4);
         fence_barrier_init();
     }
+    // a programmatic dependent of the kernel before it (inputs are read
+    // below); the merge kernel may start once every CTA is past this point
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     // ---- schedule: exclusive prefix of tiles per request (x spans), clamped L
     __syncthreads();
     const int l_cap = p.max_pages * p.ps;
