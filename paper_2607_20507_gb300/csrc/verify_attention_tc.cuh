@@ -15,17 +15,17 @@
 //           then holds (4-6), one box per page piece and dim half, so a tile
 //           lands as [dim half][64 keys][128 B], 128-byte swizzle; beside
 //           each stage it leaves whether the tile opens or closes a piece;
-//   warp 1  MMA issuer (the whole warp waits, one elected lane issues;
-//           fixed order): at a piece's start the query rows from shared into
-//           tensor memory (tcgen05.cp, one buffer per span parity), then per
-//           tile S_t = Q K_t^T into tensor memory (M = 128 padded rows,
-//           N = 64 keys, Q from tensor memory, K a K-major shared-memory
-//           operand, 8 steps of 16 dims) and O += P_t V_t
-//           (N = 128 dims, 4 steps of 16 keys) with P read from tensor
-//           memory and V an MN-major operand whose two dim halves lie one
-//           leading offset apart; QK runs two tiles ahead of PV, so that the
-//           tensor core computes S_{t+1} and S_{t+2} while the softmax works
-//           on S_t;
+//   warp 1  QK issuer (the whole warp waits, one elected lane issues): at
+//           a piece's start the query rows from shared into tensor memory
+//           (tcgen05.cp, one buffer per span parity), then per tile
+//           S_t = Q K_t^T into tensor memory (M = 128 padded rows, N = 64
+//           keys, Q from tensor memory, K a K-major shared-memory operand,
+//           8 steps of 16 dims) as soon as K_t has landed and one of four S
+//           buffers is free -- up to four tiles ahead of the softmax;
+//   warp 8  PV issuer: O += P_t V_t (N = 128 dims, 4 steps of 16 keys) as
+//           soon as the softmax releases P_t, with P read from tensor memory
+//           and V an MN-major operand whose two dim halves lie one leading
+//           offset apart;
 //   warp 2  tensor-memory allocation (512 columns: four S/P buffers of 64,
 //           O in 128, two query buffers of 64);
 //   warps 2-3  the V tile of every stage from bf16 into fp16, in place;
@@ -42,7 +42,8 @@
 // and a shared flag that ends every warp's loop.
 
 constexpr int kTcMaxStages = 6;
-constexpr int kTcThreads = 256;
+constexpr int kTcThreads = 288;                    // 9 warps
+constexpr int kTcPvWarp = 8;                       // the PV issuer
 constexpr int kTcRows = 128;                       // MMA M: query rows, padded
 constexpr int kTcMinRows = 48;                     // fewer query rows take the mma.sync form
 constexpr int kTcSBuf = 4;                         // S/P buffers in tensor memory
@@ -387,47 +388,51 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             __syncwarp();
             if (lane == 0) mbar_arrive(&ready[st]);
         }
-    } else if (warp == 1 && n_tiles > 0) {
+    } else if ((warp == 1 || warp == kTcPvWarp) && n_tiles > 0) {
         // ---------------------------------------------------------- MMA
-        // A fixed order: QK_0, QK_1, then PV_t followed by
-        // QK_{t+2} -- S_{t+1} is in tensor memory while the softmax works on
-        // S_t, and S_{t+2} is computed while it works on S_{t+1}.  Each wait
-        // names a phase its barrier can be at most one phase short of (the
-        // next phase needs an MMA this warp has not issued yet), so a parity
-        // wait is exact.  Descriptors advance by constant offsets (addresses
-        // stay below 256 KB, so the 14-bit start field cannot carry).  The
-        // whole warp runs the loop and waits; lane 0 issues the MMAs and the
-        // commits (a lone lane beside 31 parked at the block barrier pays
-        // hundreds of cycles per barrier probe and per tcgen05 instruction).
-        {
-            constexpr uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, true);
-            const uint64_t dq0 = tc_sw128_desc(smem_u32(sq));
-            const uint64_t qbuf16 = (uint64_t)(2 * qh) >> 4, qhalf16 = (uint64_t)qh >> 4;
-            const uint64_t dkv0 = tc_sw128_desc(smem_u32(skv)), dv0 = tc_mn_desc(smem_u32(skv + kTensorTileBytes));
-            uint32_t first_bits = 0;        // bit sb: the tile in S buffer sb opened its piece
-            int span = -1, pv_piece = 0;
-            uint64_t* last_bar = nullptr;   // the latest commit: completes after every MMA issued
-            uint32_t last_par = 0;
-            // every lane waits; the result is made warp-uniform, so that no lane
-            // leaves the loop while another still issues
-            auto wait_all = [&](uint64_t* bar, uint32_t par, volatile int* dead, int* status) -> bool {
-                return __all_sync(0xffffffffu, tc_wait(bar, par, dead, status));
-            };
-            auto issue_qk = [&](int t) -> bool {
-                const int st = t % kTcStages, sb = t % kTcSBuf;
-                if (!wait_all(&full[st], (uint32_t)(t / kTcStages) & 1, &s_dead, p.status)) return false;
+        // Two issuing warps, each running its loop with all lanes (the waits)
+        // and one elected lane issuing (a lone lane beside 31 parked at the
+        // block barrier pays hundreds of cycles per barrier probe and per
+        // tcgen05 instruction).  Each commit tracks the MMAs of its own
+        // thread only, and the two streams meet only through barriers:
+        //   warp 1 (QK): S_t = Q K_t^T as soon as K_t has landed and S buffer
+        //     t % 4 is free (PV_{t-4} done) -- up to four tiles ahead of the
+        //     softmax, whatever the PV stream is doing;
+        //   warp kTcPvWarp (PV): O += P_t V_t as soon as the softmax has
+        //     released P_t (and, opening a piece, the epilogue has read O).
+        // Each wait names a phase its barrier can be at most one phase short
+        // of (the next phase needs an MMA of this warp that is not issued
+        // yet), so a parity wait is exact.  Descriptors advance by constant
+        // offsets (addresses stay below 256 KB: the 14-bit start field cannot
+        // carry).
+        const bool qk_warp = warp == 1;
+        constexpr uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, true);
+        const uint64_t dq0 = tc_sw128_desc(smem_u32(sq));
+        const uint64_t qbuf16 = (uint64_t)(2 * qh) >> 4, qhalf16 = (uint64_t)qh >> 4;
+        const uint64_t dkv0 = tc_sw128_desc(smem_u32(skv)), dv0 = tc_mn_desc(smem_u32(skv + kTensorTileBytes));
+        int span = -1, pv_piece = 0;
+        Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);   // the PV warp's own view of the pieces
+        uint64_t* last_bar = nullptr;   // the warp's latest commit: completes after all its MMAs
+        uint32_t last_par = 0;
+        // every lane waits; the result is made warp-uniform, so that no lane
+        // leaves the loop while another still issues
+        auto wait_all = [&](uint64_t* bar, uint32_t par) -> bool {
+            return __all_sync(0xffffffffu, tc_wait(bar, par, &s_dead, p.status));
+        };
+        for (int t = 0; t < n_tiles; ++t) {
+            const int st = t % kTcStages, sb = t % kTcSBuf;
+            if (qk_warp) {
+                if (!wait_all(&full[st], (uint32_t)(t / kTcStages) & 1)) break;
                 const int info = s_info[st];
                 if (info & 1) {
                     // a new piece: its query rows landed, and the QKs of the
                     // piece two back are done reading the query buffer
                     ++span;
-                    if (!wait_all(&q_full[span & 1], (uint32_t)(span >> 1) & 1, &s_dead, p.status)) return false;
-                    if (span >= 2 && !wait_all(&q_free[span & 1], (uint32_t)((span - 2) >> 1) & 1, &s_dead, p.status))
-                        return false;
+                    if (!wait_all(&q_full[span & 1], (uint32_t)(span >> 1) & 1)) break;
+                    if (span >= 2 && !wait_all(&q_free[span & 1], (uint32_t)((span - 2) >> 1) & 1)) break;
                 }
                 // S buffer sb held S_{t-4}: PV_{t-4} is done with it
-                if (t >= kTcSBuf && !wait_all(&o_ready[sb], (uint32_t)((t - kTcSBuf) / kTcSBuf) & 1, &s_dead, p.status))
-                    return false;
+                if (t >= kTcSBuf && !wait_all(&o_ready[sb], (uint32_t)((t - kTcSBuf) / kTcSBuf) & 1)) break;
                 tc_fence_after();
                 const uint32_t tq = tmem + kTcQCol + (span & 1) * 64;
                 const uint64_t dk = dkv0 + (uint64_t)((st * kStageBytes) >> 4);
@@ -452,17 +457,13 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 __syncwarp();
                 last_bar = &s_full[sb];
                 last_par = (uint32_t)(t / kTcSBuf) & 1;
-                first_bits = (info & 1) ? (first_bits | (1u << sb)) : (first_bits & ~(1u << sb));
-                return true;
-            };
-            auto issue_pv = [&](int t) -> bool {
-                const int st = t % kTcStages, sb = t % kTcSBuf;
-                if (!wait_all(&p_full[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) return false;
-                const bool first = (first_bits >> sb) & 1u;
+            } else {
+                if (!wait_all(&p_full[sb], (uint32_t)(t / kTcSBuf) & 1)) break;
+                const bool first = t == 0 || cur.t == 0;
+                advance(cur, s_len, nb, p.n_vh);
                 if (first) {
                     // the previous piece's epilogue has read O
-                    if (pv_piece > 0 && !wait_all(o_free, (uint32_t)(pv_piece - 1) & 1, &s_dead, p.status))
-                        return false;
+                    if (pv_piece > 0 && !wait_all(o_free, (uint32_t)(pv_piece - 1) & 1)) break;
                     ++pv_piece;
                 }
                 tc_fence_after();
@@ -479,15 +480,12 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 __syncwarp();
                 last_bar = &o_ready[sb];
                 last_par = (uint32_t)(t / kTcSBuf) & 1;
-                return true;
-            };
-            bool ok = issue_qk(0) && (n_tiles < 2 || issue_qk(1));
-            for (int t = 0; ok && t < n_tiles; ++t) ok = issue_pv(t) && (t + 2 >= n_tiles || issue_qk(t + 2));
-            // every MMA of this CTA completes before tensor memory is freed
-            if (last_bar != nullptr && !mbar_wait_bounded(last_bar, last_par) && lane == 0)
-                atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+            }
         }
-    } else if (warp >= 4 && n_tiles > 0) {
+        // every MMA of this warp completes before tensor memory is freed
+        if (last_bar != nullptr && !mbar_wait_bounded(last_bar, last_par) && lane == 0)
+            atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+    } else if (warp >= 4 && warp < 8 && n_tiles > 0) {
         // ---------------------------------------------------- softmax, epilogue
         const int sub = warp & 3;
         const int row = sub * 32 + lane;                       // query row of the span = tensor-memory lane
