@@ -83,7 +83,8 @@ struct AttnParams {
     int n_rb;                    // row blocks per KV head (n_rows rows each)
     int n_vh;                    // Hkv * n_rb spans per request ("virtual heads")
     int n_rows_all;              // R * G query rows per KV head
-    int tc_stages, tc_q_half;    // tcgen05 kernel: K/V ring depth, bytes between query dim halves
+    int tc_stages, tc_vstages;   // tcgen05 kernel: K and V ring depths
+    int tc_q_half;               // tcgen05 kernel: bytes between query dim halves
     int b_base, n_batch;         // requests [b_base, b_base + n_batch) in this launch
     float scale_log2;            // sm_scale * log2(e)
 };
@@ -1067,7 +1068,8 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
              verify_attention_tc_kernel<true, 64>}};
         const int ti = box_t == 16 ? 0 : box_t == 32 ? 1 : 2;
         const TcKern tk_fn = tc_kerns[pl.tree][ti];
-        p.tc_stages = tc_stages(pl.n_rows_all);
+        p.tc_stages = tc_k_stages(pl.n_rows_all);
+        p.tc_vstages = tc_v_stages(pl.n_rows_all);
         p.tc_q_half = tc_q_half_bytes(pl.n_rows_all);
         const int smem_bytes = tc_smem_bytes(pl.n_rows_all);
         cudaError_t e = cudaFuncSetAttribute(tk_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);

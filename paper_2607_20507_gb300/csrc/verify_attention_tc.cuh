@@ -7,14 +7,19 @@
 // padding of every MMA costs more than it saves).  Same persistent schedule
 // (equal contiguous tile ranges, spans, two partial slots per CTA, merge
 // kernel), one CTA per SM, warp roles:
-//   warp 0  TMA producer: the span's query rows (one 4-D box per dim half,
+//   warp 0  K producer: the span's query rows (one 4-D box per dim half,
 //           double-buffered across spans, each half as many 128-byte rows as
 //           the span has: the MMA's 128-row window runs on into whatever
-//           follows, which only feeds padded rows) and the K/V tiles of the
-//           range through a ring of as many 32 KB stages as shared memory
-//           then holds (4-6), one box per page piece and dim half, so a tile
-//           lands as [dim half][64 keys][128 B], 128-byte swizzle; beside
-//           each stage it leaves whether the tile opens or closes a piece;
+//           follows, which only feeds padded rows) and the K tiles of the
+//           range through the K ring, one box per page piece and dim half, so
+//           a tile lands as [dim half][64 keys][128 B], 128-byte swizzle;
+//           beside each stage it leaves whether the tile opens or closes a
+//           piece;
+//   warp 9  V producer: the V tiles through the V ring, the same way.  The
+//           two rings share the 16 KB stages that shared memory holds beside
+//           the query buffers (a third for K, which is released as soon as
+//           its QK is done; the rest for V, held until its PV is done), so
+//           each side runs ahead as far as its own consumer allows;
 //   warp 1  QK issuer (the whole warp waits, one elected lane issues): at
 //           a piece's start the query rows from shared into tensor memory
 //           (tcgen05.cp, one buffer per span parity), then per tile
@@ -28,7 +33,7 @@
 //           offset apart;
 //   warp 2  tensor-memory allocation (512 columns: four S/P buffers of 64,
 //           O in 128, two query buffers of 64);
-//   warps 2-3  the V tile of every stage from bf16 into fp16, in place;
+//   warps 2-3  every V tile from bf16 into fp16, in place;
 //   warps 4-7  softmax and epilogue, one query row per thread (warp 4+s
 //           owns tensor-memory lanes 32s..32s+31): mask, running max, exp2,
 //           row sum, P written back over S as fp16 (warps 2-3 turn each V
@@ -41,9 +46,11 @@
 // Every mbarrier wait is bounded; a wait that gives up sets the status word
 // and a shared flag that ends every warp's loop.
 
-constexpr int kTcMaxStages = 6;
-constexpr int kTcThreads = 288;                    // 9 warps
+constexpr int kTcMaxK = 6;                         // K ring depth, at most
+constexpr int kTcMaxV = 10;                        // V ring depth, at most
+constexpr int kTcThreads = 320;                    // 10 warps
 constexpr int kTcPvWarp = 8;                       // the PV issuer
+constexpr int kTcVWarp = 9;                        // the V producer
 constexpr int kTcRows = 128;                       // MMA M: query rows, padded
 constexpr int kTcMinRows = 48;                     // fewer query rows take the mma.sync form
 constexpr int kTcSBuf = 4;                         // S/P buffers in tensor memory
@@ -56,16 +63,25 @@ constexpr int kTcSmemLimit = 232448 - 256;         // opt-in shared memory per b
 
 // Bytes between the two dim halves of a span's query rows (1024-aligned).
 __host__ __device__ constexpr int tc_q_half_bytes(int rows) { return (rows * 128 + 1023) / 1024 * 1024; }
-// K/V stages that fit beside two query buffers of `rows` rows.
-__host__ __device__ constexpr int tc_stages(int rows) {
-    return (kTcSmemLimit - kTcFixedSmem - 4 * tc_q_half_bytes(rows)) / kStageBytes < kTcMaxStages
-               ? (kTcSmemLimit - kTcFixedSmem - 4 * tc_q_half_bytes(rows)) / kStageBytes
-               : kTcMaxStages;
+// 16 KB tile stages (one K or one V tile each) that fit beside two query
+// buffers of `rows` rows, split between the K ring (a third: K is released
+// as soon as its QK is done) and the V ring (the rest: V waits for the
+// softmax).
+__host__ __device__ constexpr int tc_tile_stages(int rows) {
+    return (kTcSmemLimit - kTcFixedSmem - 4 * tc_q_half_bytes(rows)) / kTensorTileBytes;
+}
+__host__ __device__ constexpr int tc_k_stages(int rows) {
+    return (tc_tile_stages(rows) + 1) / 3 < 2 ? 2
+           : (tc_tile_stages(rows) + 1) / 3 > kTcMaxK ? kTcMaxK : (tc_tile_stages(rows) + 1) / 3;
+}
+__host__ __device__ constexpr int tc_v_stages(int rows) {
+    return tc_tile_stages(rows) - tc_k_stages(rows) > kTcMaxV ? kTcMaxV : tc_tile_stages(rows) - tc_k_stages(rows);
 }
 __host__ __device__ constexpr int tc_smem_bytes(int rows) {
-    return 4 * tc_q_half_bytes(rows) + tc_stages(rows) * kStageBytes + kTcFixedSmem;
+    return 4 * tc_q_half_bytes(rows) + (tc_k_stages(rows) + tc_v_stages(rows)) * kTensorTileBytes + kTcFixedSmem;
 }
-static_assert(tc_stages(kTcRows) >= 4, "ring too shallow for 128 query rows");
+static_assert(tc_k_stages(kTcRows) >= 2 && tc_v_stages(kTcRows) >= 4, "rings too shallow for 128 query rows");
+static_assert((2 * kTcMaxK + 3 * kTcMaxV + 4 + 3 * 4 + 1) * 8 <= 512, "barrier block too small");
 constexpr float kTcRescale = 8.f;                  // log2 growth of the max that forces a rescale of O
 
 __device__ __forceinline__ uint64_t tc_sw128_desc(uint32_t addr) {
@@ -174,18 +190,21 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __grid_constant__ CUtensorMap tmap_v,
                            const __grid_constant__ CUtensorMap tmap_q, const AttnParams p) {
     constexpr int kPieces = kTileT / kBoxT;
-    constexpr uint32_t kPieceBytes = (uint32_t)kBoxT * 256u;   // K and V bytes of one page piece each
+    constexpr uint32_t kPieceBytes = (uint32_t)kBoxT * 256u;   // bytes of one page piece of K (or of V)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    const int kTcStages = p.tc_stages;                      // K/V ring depth
+    const int SK = p.tc_stages, SV = p.tc_vstages;          // K and V ring depths
     const int qh = p.tc_q_half;                             // bytes between the dim halves of a span's rows
     uint8_t* sq = smem;                                     // [2 spans][2 halves][rows][128 B]
-    uint8_t* skv = smem + 4 * qh;                           // [stage][K | V][half][64 keys][128 B]
-    uint64_t* bars = reinterpret_cast<uint64_t*>(skv + kTcStages * kStageBytes);
-    uint64_t* full = bars;                                  // [stages] K/V landed
-    uint64_t* empty = bars + kTcMaxStages;                  // [stages] K/V consumed (PV done)
-    uint64_t* ready = bars + 2 * kTcMaxStages;              // [stages] the stage's V is in fp16
-    uint64_t* q_full = bars + 3 * kTcMaxStages;             // [2] Q of a span landed
+    uint8_t* sk = smem + 4 * qh;                            // [K stage][half][64 keys][128 B]
+    uint8_t* sv = sk + SK * kTensorTileBytes;               // [V stage][half][64 keys][128 B]
+    uint64_t* bars = reinterpret_cast<uint64_t*>(sv + SV * kTensorTileBytes);
+    uint64_t* kfull = bars;                                 // [SK] K tile landed
+    uint64_t* kempty = kfull + kTcMaxK;                     // [SK] K tile consumed (QK done)
+    uint64_t* vfull = kempty + kTcMaxK;                     // [SV] V tile landed
+    uint64_t* vempty = vfull + kTcMaxV;                     // [SV] V tile consumed (PV done)
+    uint64_t* ready = vempty + kTcMaxV;                     // [SV] the V tile is in fp16
+    uint64_t* q_full = ready + kTcMaxV;                     // [2] Q of a span landed
     uint64_t* q_free = q_full + 2;                          // [2] last QK of a span done
     uint64_t* s_full = q_free + 2;                          // [kTcSBuf] S_t in tensor memory
     uint64_t* p_full = s_full + kTcSBuf;                    // [kTcSBuf] P_t written (count 4 warps)
@@ -197,8 +216,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     __shared__ long long s_carry;
     __shared__ uint32_t s_tmem;
     __shared__ volatile int s_dead;
-    __shared__ int s_keys[kTcMaxStages];   // keys of the tile in each stage (V rows past are zeroed)
-    __shared__ int s_info[kTcMaxStages];   // bit 0: the stage's tile opens a span piece, bit 1: ends one
+    __shared__ int s_keys[kTcMaxV];   // keys of the tile in each V stage (V rows past are zeroed)
+    __shared__ int s_info[kTcMaxK];   // per K stage, bit 0: the tile opens a span piece, bit 1: ends one
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = p.n_batch;
@@ -219,9 +238,13 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     if (threadIdx.x == 0) {
         s_carry = 0;
         s_dead = 0;
-        for (int i = 0; i < kTcStages; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&empty[i], 1);
+        for (int i = 0; i < SK; ++i) {
+            mbar_init(&kfull[i], 1);
+            mbar_init(&kempty[i], 1);
+        }
+        for (int i = 0; i < SV; ++i) {
+            mbar_init(&vfull[i], 1);
+            mbar_init(&vempty[i], 1);
             mbar_init(&ready[i], 2);
         }
         for (int i = 0; i < 2; ++i) {
@@ -282,8 +305,17 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     const int n_tiles = (int)(f1 - f0);
     const uint32_t qrow_bytes = (uint32_t)(p.R * p.G) * 128u;   // one dim half of a span's rows
 
-    if (warp == 0 && n_tiles > 0) {
-        // ---------------------------------------------------------- producer
+    if ((warp == 0 || warp == kTcVWarp) && n_tiles > 0) {
+        // --------------------------------------------------------- producers
+        // warp 0: the K tiles (and, opening a piece, the query rows) through
+        // the K ring; warp kTcVWarp: the V tiles through the V ring.  Each
+        // runs ahead as far as its own ring allows.
+        const bool k_side = warp == 0;
+        const int S = k_side ? SK : SV;
+        uint8_t* const ring = k_side ? sk : sv;
+        uint64_t* const fullb = k_side ? kfull : vfull;
+        uint64_t* const emptyb = k_side ? kempty : vempty;
+        const CUtensorMap* const tmap = k_side ? &tmap_k : &tmap_v;
         constexpr int per_batch = 32 / kPieces;
         auto batch_pages = [&](int j0) -> int {
             const int jj = j0 + lane / kPieces;
@@ -294,24 +326,23 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             return __ldg(p.page_table + (size_t)(p.b_base + cc.b) * p.max_pages + tok / p.ps);
         };
         if (lane == 0) {
-            tma_prefetch_desc(&tmap_k);
-            tma_prefetch_desc(&tmap_v);
-            tma_prefetch_desc(&tmap_q);
+            tma_prefetch_desc(tmap);
+            if (k_side) tma_prefetch_desc(&tmap_q);
         }
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
         int pg_cur = batch_pages(0);
         int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
         int span = -1;
-        // tile jt goes out once its stage is free and, opening a piece, once
-        // the query buffer it reuses is free
+        // tile jt goes out once its stage is free and, K side opening a
+        // piece, once the query buffer it reuses is free
         int jt = 0;
         for (; jt < n_tiles; ++jt) {
-            const int st = jt % kTcStages;
+            const int st = jt % S;
             const bool first = jt == 0 || cur.t == 0;
             const bool last = jt + 1 == n_tiles || cur.t + 1 == cur.T;
             if (first) ++span;
-            bool go = jt < kTcStages || tc_wait(&empty[st], (uint32_t)(jt / kTcStages - 1) & 1, &s_dead, p.status);
-            if (go && first && span >= 2)
+            bool go = jt < S || tc_wait(&emptyb[st], (uint32_t)(jt / S - 1) & 1, &s_dead, p.status);
+            if (go && k_side && first && span >= 2)
                 go = tc_wait(&q_free[span & 1], (uint32_t)((span - 2) >> 1) & 1, &s_dead, p.status);
             if (!__all_sync(0xffffffffu, go)) break;
             const int jb = jt % per_batch;
@@ -323,7 +354,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             const int L = s_len[cur.b];
             const int ts = cur.t * kTileT;
             const int h_cur = cur.h / p.n_rb;
-            if (first && lane == 0) {
+            if (k_side && first && lane == 0) {
                 // a new span piece: its query rows into buffer span % 2
                 mbar_arrive_expect_tx(&q_full[span & 1], 2 * qrow_bytes);
                 const uint32_t qdst = smem_u32(sq + (span & 1) * 2 * qh);
@@ -336,27 +367,23 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             for (int pc = 0; pc < kPieces; ++pc)
                 if (ts + pc * kBoxT < L) ++valid;
             if (lane == 0) {
-                s_keys[st] = max(0, min(kTileT, L - ts));
-                s_info[st] = (first ? 1 : 0) | (last ? 2 : 0);
-                mbar_arrive_expect_tx(&full[st], (uint32_t)valid * kPieceBytes * 2u);
+                if (k_side) s_info[st] = (first ? 1 : 0) | (last ? 2 : 0);
+                else s_keys[st] = max(0, min(kTileT, L - ts));
+                mbar_arrive_expect_tx(&fullb[st], (uint32_t)valid * kPieceBytes);
             }
             __syncwarp();
             if (lane < valid) {
-                const uint32_t kdst = smem_u32(skv + st * kStageBytes) + (uint32_t)lane * (kBoxT * 128);
+                const uint32_t dst = smem_u32(ring + st * kTensorTileBytes) + (uint32_t)lane * (kBoxT * 128);
                 const int slot = (ts + lane * kBoxT) % p.ps;
 #pragma unroll
-                for (int hh = 0; hh < 2; ++hh) {
-                    tma_load_5d(kdst + hh * kTcHalfBytes, &tmap_k, &full[st], 0, slot, hh, h_cur, page);
-                    tma_load_5d(kdst + kTensorTileBytes + hh * kTcHalfBytes, &tmap_v, &full[st], 0, slot, hh, h_cur,
-                                page);
-                }
+                for (int hh = 0; hh < 2; ++hh)
+                    tma_load_5d(dst + hh * kTcHalfBytes, tmap, &fullb[st], 0, slot, hh, h_cur, page);
             }
         }
         // no copy in flight at exit: every issued tile has landed
         if (lane == 0)
-            for (int j = jt > kTcStages ? jt - kTcStages : 0; j < jt; ++j)
-                if (!mbar_wait_bounded(&full[j % kTcStages], (uint32_t)(j / kTcStages) & 1))
-                    atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
+            for (int j = jt > S ? jt - S : 0; j < jt; ++j)
+                if (!mbar_wait_bounded(&fullb[j % S], (uint32_t)(j / S) & 1)) atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
     } else if ((warp == 2 || warp == 3) && n_tiles > 0) {
         // ------------------------------------------------------- V to fp16
         // Each landed V tile is turned from bf16 into fp16 in place by these
@@ -366,10 +393,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // hands P_t to the MMA warp.
         const int ct = (warp - 2) * 32 + lane;
         for (int jc = 0; jc < n_tiles; ++jc) {
-            const int st = jc % kTcStages;
-            if (!tc_wait(&full[st], (uint32_t)(jc / kTcStages) & 1, &s_dead, p.status)) break;
+            const int st = jc % SV;
+            if (!tc_wait(&vfull[st], (uint32_t)(jc / SV) & 1, &s_dead, p.status)) break;
             const int keys = s_keys[st];
-            uint4* vt = reinterpret_cast<uint4*>(skv + st * kStageBytes + kTensorTileBytes);
+            uint4* vt = reinterpret_cast<uint4*>(sv + st * kTensorTileBytes);
 #pragma unroll 4
             for (int i = ct; i < kTensorTileBytes / 16; i += 64) {
                 uint4 v = make_uint4(0, 0, 0, 0);
@@ -409,7 +436,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         constexpr uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, true);
         const uint64_t dq0 = tc_sw128_desc(smem_u32(sq));
         const uint64_t qbuf16 = (uint64_t)(2 * qh) >> 4, qhalf16 = (uint64_t)qh >> 4;
-        const uint64_t dkv0 = tc_sw128_desc(smem_u32(skv)), dv0 = tc_mn_desc(smem_u32(skv + kTensorTileBytes));
+        const uint64_t dk0 = tc_sw128_desc(smem_u32(sk)), dv0 = tc_mn_desc(smem_u32(sv));
         int span = -1, pv_piece = 0;
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);   // the PV warp's own view of the pieces
         uint64_t* last_bar = nullptr;   // the warp's latest commit: completes after all its MMAs
@@ -420,9 +447,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             return __all_sync(0xffffffffu, tc_wait(bar, par, &s_dead, p.status));
         };
         for (int t = 0; t < n_tiles; ++t) {
-            const int st = t % kTcStages, sb = t % kTcSBuf;
+            const int sb = t % kTcSBuf;
             if (qk_warp) {
-                if (!wait_all(&full[st], (uint32_t)(t / kTcStages) & 1)) break;
+                const int st = t % SK;
+                if (!wait_all(&kfull[st], (uint32_t)(t / SK) & 1)) break;
                 const int info = s_info[st];
                 if (info & 1) {
                     // a new piece: its query rows landed, and the QKs of the
@@ -435,7 +463,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 if (t >= kTcSBuf && !wait_all(&o_ready[sb], (uint32_t)((t - kTcSBuf) / kTcSBuf) & 1)) break;
                 tc_fence_after();
                 const uint32_t tq = tmem + kTcQCol + (span & 1) * 64;
-                const uint64_t dk = dkv0 + (uint64_t)((st * kStageBytes) >> 4);
+                const uint64_t dk = dk0 + (uint64_t)((st * kTensorTileBytes) >> 4);
                 if (elect_one()) {
                     if (info & 1) {
                         // the query rows into tensor memory once per piece, 16
@@ -452,12 +480,14 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                         tc_mma_ts(tmem + sb * 64, tq + ks * 8, dk + ko, id_s, ks > 0 ? 1u : 0u);
                     }
                     tc_commit(&s_full[sb]);
+                    tc_commit(&kempty[st]);
                     if (info & 2) tc_commit(&q_free[span & 1]);
                 }
                 __syncwarp();
                 last_bar = &s_full[sb];
                 last_par = (uint32_t)(t / kTcSBuf) & 1;
             } else {
+                const int st = t % SV;
                 if (!wait_all(&p_full[sb], (uint32_t)(t / kTcSBuf) & 1)) break;
                 const bool first = t == 0 || cur.t == 0;
                 advance(cur, s_len, nb, p.n_vh);
@@ -468,14 +498,14 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 }
                 tc_fence_after();
                 // O += P_t V_t, 4 steps of 16 keys, both dim halves per step
-                const uint64_t dv = dv0 + (uint64_t)((st * kStageBytes) >> 4);
+                const uint64_t dv = dv0 + (uint64_t)((st * kTensorTileBytes) >> 4);
                 if (elect_one()) {
 #pragma unroll
                     for (int kk = 0; kk < kTileT / 16; ++kk)
                         tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + kk * 8, dv + (uint64_t)(kk * ((16 * 128) >> 4)),
                                   id_o, (first && kk == 0) ? 0u : 1u);
                     tc_commit(&o_ready[sb]);
-                    tc_commit(&empty[st]);
+                    tc_commit(&vempty[st]);
                 }
                 __syncwarp();
                 last_bar = &o_ready[sb];
@@ -599,8 +629,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             // P_t goes to the MMA warp once the tile's V is in fp16 too (the
             // PV reads both).  The next phase of `ready` needs the stage
             // back, i.e. this PV, so the parity names one phase.
-            const bool v_ok = lane != 0 || tc_wait(&ready[t % kTcStages], (uint32_t)(t / kTcStages) & 1, &s_dead,
-                                                   p.status);
+            const bool v_ok = lane != 0 || tc_wait(&ready[t % SV], (uint32_t)(t / SV) & 1, &s_dead, p.status);
             if (!__all_sync(0xffffffffu, v_ok)) break;
             if (lane == 0) mbar_arrive(&p_full[sb]);
 
