@@ -15,7 +15,7 @@
 //           a tile lands as [dim half][64 keys][128 B], 128-byte swizzle;
 //           beside each stage it leaves whether the tile opens or closes a
 //           piece;
-//   warp 9  V producer: the V tiles through the V ring, the same way.  The
+//   warp 13 V producer: the V tiles through the V ring, the same way.  The
 //           two rings share the 16 KB stages that shared memory holds beside
 //           the query buffers (a third for K, which is released as soon as
 //           its QK is done; the rest for V, held until its PV is done), so
@@ -27,30 +27,32 @@
 //           keys, Q from tensor memory, K a K-major shared-memory operand,
 //           8 steps of 16 dims) as soon as K_t has landed and one of four S
 //           buffers is free -- up to four tiles ahead of the softmax;
-//   warp 8  PV issuer: O += P_t V_t (N = 128 dims, 4 steps of 16 keys) as
+//   warp 12 PV issuer: O += P_t V_t (N = 128 dims, 4 steps of 16 keys) as
 //           soon as the softmax releases P_t, with P read from tensor memory
 //           and V an MN-major operand whose two dim halves lie one leading
 //           offset apart;
 //   warp 2  tensor-memory allocation (512 columns: four S/P buffers of 64,
 //           O in 128, two query buffers of 64);
 //   warps 2-3  every V tile from bf16 into fp16, in place;
-//   warps 4-7  softmax and epilogue, one query row per thread (warp 4+s
-//           owns tensor-memory lanes 32s..32s+31): mask, running max, exp2,
+//   warps 4-11 softmax and epilogue, two warps per query row (one row per
+//           lane; warps 4+q and 8+q own tensor-memory lanes 32q..32q+31 and
+//           take keys 0..31 and 32..63 of every tile): mask, running max
+//           (the two halves' maxima swapped through shared memory), exp2,
 //           row sum, P written back over S as fp16 (warps 2-3 turn each V
 //           tile into fp16, so PV multiplies fp16 by fp16: bf16 P alone can
 //           exceed the output tolerance on rows whose terms cancel); O is
-//           rescaled in tensor
-//           memory only when the running max grows by more than 2^8 (the
-//           stale max keeps every P below 256); at a span piece's end the
-//           row is normalised and written (bf16) or left as a partial.
+//           rescaled in tensor memory only when the running max grows by
+//           more than 2^8 (the stale max keeps every P below 256); at a span
+//           piece's end the row is normalised and written (bf16) or left as
+//           a partial, 64 dims by each warp of the pair.
 // Every mbarrier wait is bounded; a wait that gives up sets the status word
 // and a shared flag that ends every warp's loop.
 
 constexpr int kTcMaxK = 6;                         // K ring depth, at most
 constexpr int kTcMaxV = 10;                        // V ring depth, at most
-constexpr int kTcThreads = 320;                    // 10 warps
-constexpr int kTcPvWarp = 8;                       // the PV issuer
-constexpr int kTcVWarp = 9;                        // the V producer
+constexpr int kTcThreads = 448;                    // 14 warps
+constexpr int kTcPvWarp = 12;                      // the PV issuer
+constexpr int kTcVWarp = 13;                       // the V producer
 constexpr int kTcRows = 128;                       // MMA M: query rows, padded
 constexpr int kTcMinRows = 48;                     // fewer query rows take the mma.sync form
 constexpr int kTcSBuf = 4;                         // S/P buffers in tensor memory
@@ -59,7 +61,7 @@ constexpr int kTcQCol = kTcOCol + 128;             // first column of the two qu
 constexpr int kTcTmemCols = 512;                   // S/P [0, 256) in four buffers, O [256, 384), Q [384, 512)
 constexpr int kTcBarBytes = 512;
 constexpr int kTcFixedSmem = kTcBarBytes + (kMaxBatchPerLaunch + 1) * 8 + kMaxBatchPerLaunch * 4 + 1024;
-constexpr int kTcSmemLimit = 232448 - 256;         // opt-in shared memory per block, less the static part
+constexpr int kTcSmemLimit = 232448 - 2560;        // opt-in shared memory per block, less the static part
 
 // Bytes between the two dim halves of a span's query rows (1024-aligned).
 __host__ __device__ constexpr int tc_q_half_bytes(int rows) { return (rows * 128 + 1023) / 1024 * 1024; }
@@ -81,7 +83,7 @@ __host__ __device__ constexpr int tc_smem_bytes(int rows) {
     return 4 * tc_q_half_bytes(rows) + (tc_k_stages(rows) + tc_v_stages(rows)) * kTensorTileBytes + kTcFixedSmem;
 }
 static_assert(tc_k_stages(kTcRows) >= 2 && tc_v_stages(kTcRows) >= 4, "rings too shallow for 128 query rows");
-static_assert((2 * kTcMaxK + 3 * kTcMaxV + 4 + 3 * 4 + 1) * 8 <= 512, "barrier block too small");
+static_assert((2 * kTcMaxK + 3 * kTcMaxV + 4 + 3 * 4 + 1 + 4) * 8 <= 512, "barrier block too small");
 constexpr float kTcRescale = 8.f;                  // log2 growth of the max that forces a rescale of O
 
 __device__ __forceinline__ uint64_t tc_sw128_desc(uint32_t addr) {
@@ -169,6 +171,15 @@ __device__ __forceinline__ void tc_st32(uint32_t addr, const uint32_t (&r)[32]) 
         : "memory");
 }
 
+__device__ __forceinline__ void tc_st16(uint32_t addr, const uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+            addr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]),
+        "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+}
+
 __device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -207,9 +218,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     uint64_t* q_full = ready + kTcMaxV;                     // [2] Q of a span landed
     uint64_t* q_free = q_full + 2;                          // [2] last QK of a span done
     uint64_t* s_full = q_free + 2;                          // [kTcSBuf] S_t in tensor memory
-    uint64_t* p_full = s_full + kTcSBuf;                    // [kTcSBuf] P_t written (count 4 warps)
+    uint64_t* p_full = s_full + kTcSBuf;                    // [kTcSBuf] P_t written (count 8 warps)
     uint64_t* o_ready = p_full + kTcSBuf;                   // [kTcSBuf] PV_t done (S buffer free again)
-    uint64_t* o_free = o_ready + kTcSBuf;                   // O read out by the epilogue (count 4 warps)
+    uint64_t* o_free = o_ready + kTcSBuf;                   // O read out by the epilogue (count 8 warps)
+    uint64_t* pair_bar = o_free + 1;                        // [4] a softmax warp pair swapped values
     long long* s_prefix = reinterpret_cast<long long*>(reinterpret_cast<uint8_t*>(bars) + kTcBarBytes);
     int* s_len = reinterpret_cast<int*>(s_prefix + kMaxBatchPerLaunch + 1);
     __shared__ long long s_wtot[kTcThreads / 32];
@@ -218,6 +230,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     __shared__ volatile int s_dead;
     __shared__ int s_keys[kTcMaxV];   // keys of the tile in each V stage (V rows past are zeroed)
     __shared__ int s_info[kTcMaxK];   // per K stage, bit 0: the tile opens a span piece, bit 1: ends one
+    __shared__ float s_xch[4 * 2 * 2 * 32];   // softmax pair swaps: [pair][slot][half][lane]
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = p.n_batch;
@@ -253,10 +266,11 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         }
         for (int i = 0; i < kTcSBuf; ++i) {
             mbar_init(&s_full[i], 1);
-            mbar_init(&p_full[i], 4);
+            mbar_init(&p_full[i], 8);
             mbar_init(&o_ready[i], 1);
         }
-        mbar_init(o_free, 4);
+        mbar_init(o_free, 8);
+        for (int i = 0; i < 4; ++i) mbar_init(&pair_bar[i], 2);
         fence_barrier_init();
     }
     // a programmatic dependent of the kernel before it (inputs are read
@@ -515,22 +529,44 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // every MMA of this warp completes before tensor memory is freed
         if (last_bar != nullptr && !mbar_wait_bounded(last_bar, last_par) && lane == 0)
             atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-    } else if (warp >= 4 && warp < 8 && n_tiles > 0) {
+    } else if (warp >= 4 && warp < 12 && n_tiles > 0) {
         // ---------------------------------------------------- softmax, epilogue
-        const int sub = warp & 3;
+        // Two warps per tensor-memory lane quarter: warp 4+q (half 0) takes
+        // keys 0..31 of every tile, warp 8+q (half 1) keys 32..63, both for
+        // the query rows 32q..32q+31 (one per lane).  They swap their partial
+        // maxima of each tile (and their row sums at a piece's end) through
+        // shared memory, so both hold the same running max and make the same
+        // rescale decisions; each writes its half of P, rescales and writes
+        // its half of O, and keeps its half of the row sum.
+        const int sub = warp & 3, half = warp >= 8 ? 1 : 0;
+        const int kb = half * 32;                              // this warp's first key of a tile
         const int row = sub * 32 + lane;                       // query row of the span = tensor-memory lane
         const uint32_t t_row = tmem + ((uint32_t)(sub * 32) << 16);
         const float c = p.scale_log2;
+        uint32_t n_x = 0;                                      // swaps so far (the same count in both warps)
+        // the partner's value for this lane; false once a wait gave up
+        auto swap = [&](float mine, float& other) -> bool {
+            const int slot = (int)(n_x & 1);
+            s_xch[((sub * 2 + slot) * 2 + half) * 32 + lane] = mine;
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&pair_bar[sub]);
+            const bool ok = __all_sync(0xffffffffu, tc_wait(&pair_bar[sub], n_x & 1, &s_dead, p.status));
+            tc_fence_after();
+            ++n_x;
+            other = s_xch[((sub * 2 + slot) * 2 + (half ^ 1)) * 32 + lane];
+            return ok;
+        };
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
         int seg_t0 = cur.t;
         bool first_seg = true;
-        float m_run = kNegInf, l_run = 0.f;
+        float m_run = kNegInf, l_half = 0.f;
         int lim = 0, tree_base = 0, span_L = 0;
         uint64_t anc = ~0ull;
         auto begin_span = [&](const Cursor& cc) {
             const int L = s_len[cc.b];
             m_run = kNegInf;
-            l_run = 0.f;
+            l_half = 0.f;
             if (kTree) {
                 uint64_t ma, mb;
                 tree_ancestor_masks(p.parents + (size_t)(p.b_base + cc.b) * p.R, p.R, lane, ma, mb);
@@ -550,31 +586,30 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             const bool piece_end = t + 1 == n_tiles || cur.t + 1 == cur.T;
             if (!tc_wait(&s_full[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) break;
             tc_fence_after();
-            float s[64];
-            tc_ld32(t_row + sb * 64, *reinterpret_cast<float(*)[32]>(&s[0]));
-            tc_ld32(t_row + sb * 64 + 32, *reinterpret_cast<float(*)[32]>(&s[32]));
+            float s[32];
+            tc_ld32(t_row + sb * 64 + kb, s);
             // ---- mask (tree ancestors or the causal chain, and the context end);
             // padded rows see nothing
-            float mt = kNegInf;
+            float mh = kNegInf;
             if (row >= p.n_rows_all) {
 #pragma unroll
-                for (int e = 0; e < 64; ++e) s[e] = kNegInf;
+                for (int e = 0; e < 32; ++e) s[e] = kNegInf;
             } else if (kTree) {
                 const int d = ts - tree_base;
                 const uint64_t pre = d >= 0 ? 0ull : (d <= -64 ? ~0ull : (1ull << -d) - 1ull);
                 const uint64_t live = span_L - ts >= 64 ? ~0ull : (1ull << max(span_L - ts, 0)) - 1ull;
                 const uint64_t tr = d >= 64 ? 0ull : (d >= 0 ? anc >> d : (d <= -64 ? 0ull : anc << -d));
-                const uint64_t vis = (pre | tr) & live;
+                const uint32_t vis = (uint32_t)(((pre | tr) & live) >> kb);
 #pragma unroll
-                for (int e = 0; e < 64; ++e) {
-                    if (!((vis >> e) & 1ull)) s[e] = kNegInf;
-                    mt = fmaxf(mt, s[e]);
+                for (int e = 0; e < 32; ++e) {
+                    if (!((vis >> e) & 1u)) s[e] = kNegInf;
+                    mh = fmaxf(mh, s[e]);
                 }
             } else {
-                const int lim_t = lim - ts;   // keys e < lim_t are visible
-                if (lim_t < 64) {
+                const int lim_t = lim - ts - kb;   // keys e < lim_t of this half are visible
+                if (lim_t < 32) {
 #pragma unroll
-                    for (int e = 0; e < 64; ++e)
+                    for (int e = 0; e < 32; ++e)
                         if (e >= lim_t) s[e] = kNegInf;
                 }
                 // eight independent chains: the maximum is exact in any order
@@ -582,10 +617,13 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
 #pragma unroll
                 for (int j = 0; j < 8; ++j) m8[j] = fmaxf(s[j], s[j + 8]);
 #pragma unroll
-                for (int e = 16; e < 64; ++e) m8[e & 7] = fmaxf(m8[e & 7], s[e]);
-                mt = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
+                for (int e = 16; e < 32; ++e) m8[e & 7] = fmaxf(m8[e & 7], s[e]);
+                mh = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
                            fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
             }
+            float mo;
+            if (!swap(mh, mo)) break;
+            const float mt = fmaxf(mh, mo);   // the tile's row maximum, the same in both warps
             // ---- running max, lazily: O is rescaled only for a growth > 2^8
             float alpha = 1.f;
             if (mt != kNegInf && (m_run == kNegInf || (mt - m_run) * c > kTcRescale)) {
@@ -594,27 +632,26 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             }
             const float neg = m_run == kNegInf ? 0.f : -m_run * c;
             float r4[4] = {0.f, 0.f, 0.f, 0.f};
-            uint32_t pk[32];
+            uint32_t pk[16];
 #pragma unroll
-            for (int e = 0; e < 32; ++e) {
+            for (int e = 0; e < 16; ++e) {
                 const float p0 = ex2(fmaf(s[2 * e], c, neg)), p1 = ex2(fmaf(s[2 * e + 1], c, neg));
                 r4[e & 3] += p0 + p1;
                 pk[e] = pack_f16x2(p0, p1);
             }
-            const float rs = (r4[0] + r4[1]) + (r4[2] + r4[3]);
-            l_run = l_run * alpha + rs;
-            // ---- a rescale of O waits for PV_{t-1}; the first tile of a piece
-            // needs none (its PV overwrites O).  o_ready[b] completes once per
-            // tile of S buffer b: PV_{t-5} is complete (QK_t waited for
-            // PV_{t-4}) and PV_{t+3} is not issued, so the parity of PV_{t-1}'s
-            // phase is unambiguous.
+            l_half = l_half * alpha + ((r4[0] + r4[1]) + (r4[2] + r4[3]));
+            // ---- a rescale of O (this warp's 64 dims) waits for PV_{t-1}; the
+            // first tile of a piece needs none (its PV overwrites O).
+            // o_ready[b] completes once per tile of S buffer b: PV_{t-5} is
+            // complete (QK_t waited for PV_{t-4}) and PV_{t+3} is not issued,
+            // so the parity of PV_{t-1}'s phase is unambiguous.
             const unsigned need = __ballot_sync(0xffffffffu, alpha != 1.f && cur.t != seg_t0);
             if (need) {
                 const int tp = t - 1;
                 if (!tc_wait(&o_ready[tp % kTcSBuf], (uint32_t)(tp / kTcSBuf) & 1, &s_dead, p.status)) break;
                 tc_fence_after();
 #pragma unroll 1
-                for (int c0 = 0; c0 < 128; c0 += 32) {
+                for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
                     float o[32];
                     tc_ld32(t_row + kTcOCol + c0, o);
                     uint32_t r[32];
@@ -623,13 +660,16 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                     tc_st32(t_row + kTcOCol + c0, r);
                 }
             }
-            tc_st32(t_row + sb * 64, pk);
+            // P as fp16 pairs: keys kb..kb+31 are columns kb/2 .. kb/2+15 of the
+            // buffer (the partner's S columns there were loaded before the swap)
+            tc_st16(t_row + sb * 64 + half * 16, pk);
             tc_wait_st();
             tc_fence_before();
             // P_t goes to the MMA warp once the tile's V is in fp16 too (the
             // PV reads both).  The next phase of `ready` needs the stage
             // back, i.e. this PV, so the parity names one phase.
-            const bool v_ok = lane != 0 || tc_wait(&ready[t % SV], (uint32_t)(t / SV) & 1, &s_dead, p.status);
+            const bool v_ok = lane != 0 || half != 0 || tc_wait(&ready[t % SV], (uint32_t)(t / SV) & 1, &s_dead,
+                                                                p.status);
             if (!__all_sync(0xffffffffu, v_ok)) break;
             if (lane == 0) mbar_arrive(&p_full[sb]);
 
@@ -638,9 +678,14 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 continue;
             }
             // ---- end of a span piece: O after its last PV (every earlier MMA
-            // completes before that commit), then written
+            // completes before that commit), then written, each warp its 64
+            // dims; the row sum is the two halves' sum, added in the same
+            // order in both warps
             if (!tc_wait(&o_ready[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) break;
             tc_fence_after();
+            float lo;
+            if (!swap(l_half, lo)) break;
+            const float l_run = half == 0 ? l_half + lo : lo + l_half;
             const int bg = p.b_base + cur.b;
             const int head = cur.h / p.n_rb;
             const bool complete = seg_t0 == 0 && cur.t + 1 == cur.T;
@@ -648,7 +693,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             const bool live_row = row < p.n_rows_all;
             const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
 #pragma unroll 1
-            for (int c0 = 0; c0 < 128; c0 += 32) {
+            for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
                 float o[32];
                 tc_ld32(t_row + kTcOCol + c0, o);
                 if (!live_row) continue;
@@ -672,7 +717,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                             make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
                 }
             }
-            if (live_row && !complete)
+            if (live_row && !complete && half == 0)
                 p.part_ml[slot * p.n_rows + row] = make_float2(m_run == kNegInf ? kNegInf : m_run * c, l_run);
             tc_fence_before();
             __syncwarp();
