@@ -7,8 +7,9 @@
 // padding of every MMA costs more than it saves).  Same persistent schedule
 // (equal contiguous tile ranges, spans, two partial slots per CTA, merge
 // kernel), one CTA per SM, warp roles:
-//   warp 0  K producer: the span's query rows (one 4-D box per dim half,
-//           double-buffered across spans, each half as many 128-byte rows as
+//   warp 0  K producer: the span's query rows (one 4-D box per dim half into
+//           one buffer, refilled once the previous span's rows have been
+//           copied into tensor memory; each half as many 128-byte rows as
 //           the span has: the MMA's 128-row window runs on into whatever
 //           follows, which only feeds padded rows) and the K tiles of the
 //           range through the K ring, one box per page piece and dim half, so
@@ -17,7 +18,7 @@
 //           piece;
 //   warp 13 V producer: the V tiles through the V ring, the same way.  The
 //           two rings share the 16 KB stages that shared memory holds beside
-//           the query buffers (a third for K, which is released as soon as
+//           the query buffer (a third for K, which is released as soon as
 //           its QK is done; the rest for V, held until its PV is done), so
 //           each side runs ahead as far as its own consumer allows;
 //   warp 1  QK issuer (the whole warp waits, one elected lane issues): at
@@ -65,12 +66,12 @@ constexpr int kTcSmemLimit = 232448 - 2560;        // opt-in shared memory per b
 
 // Bytes between the two dim halves of a span's query rows (1024-aligned).
 __host__ __device__ constexpr int tc_q_half_bytes(int rows) { return (rows * 128 + 1023) / 1024 * 1024; }
-// 16 KB tile stages (one K or one V tile each) that fit beside two query
-// buffers of `rows` rows, split between the K ring (a third: K is released
+// 16 KB tile stages (one K or one V tile each) that fit beside the query
+// buffer of `rows` rows, split between the K ring (a third: K is released
 // as soon as its QK is done) and the V ring (the rest: V waits for the
 // softmax).
 __host__ __device__ constexpr int tc_tile_stages(int rows) {
-    return (kTcSmemLimit - kTcFixedSmem - 4 * tc_q_half_bytes(rows)) / kTensorTileBytes;
+    return (kTcSmemLimit - kTcFixedSmem - 2 * tc_q_half_bytes(rows)) / kTensorTileBytes;
 }
 __host__ __device__ constexpr int tc_k_stages(int rows) {
     return (tc_tile_stages(rows) + 1) / 3 < 2 ? 2
@@ -80,10 +81,10 @@ __host__ __device__ constexpr int tc_v_stages(int rows) {
     return tc_tile_stages(rows) - tc_k_stages(rows) > kTcMaxV ? kTcMaxV : tc_tile_stages(rows) - tc_k_stages(rows);
 }
 __host__ __device__ constexpr int tc_smem_bytes(int rows) {
-    return 4 * tc_q_half_bytes(rows) + (tc_k_stages(rows) + tc_v_stages(rows)) * kTensorTileBytes + kTcFixedSmem;
+    return 2 * tc_q_half_bytes(rows) + (tc_k_stages(rows) + tc_v_stages(rows)) * kTensorTileBytes + kTcFixedSmem;
 }
 static_assert(tc_k_stages(kTcRows) >= 2 && tc_v_stages(kTcRows) >= 4, "rings too shallow for 128 query rows");
-static_assert((2 * kTcMaxK + 3 * kTcMaxV + 4 + 3 * 4 + 1 + 4) * 8 <= 512, "barrier block too small");
+static_assert((2 * kTcMaxK + 3 * kTcMaxV + 5 + 3 * 4 + 1 + 4) * 8 <= 512, "barrier block too small");
 constexpr float kTcRescale = 8.f;                  // log2 growth of the max that forces a rescale of O
 
 __device__ __forceinline__ uint64_t tc_sw128_desc(uint32_t addr) {
@@ -206,8 +207,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int SK = p.tc_stages, SV = p.tc_vstages;          // K and V ring depths
     const int qh = p.tc_q_half;                             // bytes between the dim halves of a span's rows
-    uint8_t* sq = smem;                                     // [2 spans][2 halves][rows][128 B]
-    uint8_t* sk = smem + 4 * qh;                            // [K stage][half][64 keys][128 B]
+    uint8_t* sq = smem;                                     // [2 halves][rows][128 B]: one span's query rows
+    uint8_t* sk = smem + 2 * qh;                            // [K stage][half][64 keys][128 B]
     uint8_t* sv = sk + SK * kTensorTileBytes;               // [V stage][half][64 keys][128 B]
     uint64_t* bars = reinterpret_cast<uint64_t*>(sv + SV * kTensorTileBytes);
     uint64_t* kfull = bars;                                 // [SK] K tile landed
@@ -215,8 +216,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     uint64_t* vfull = kempty + kTcMaxK;                     // [SV] V tile landed
     uint64_t* vempty = vfull + kTcMaxV;                     // [SV] V tile consumed (PV done)
     uint64_t* ready = vempty + kTcMaxV;                     // [SV] the V tile is in fp16
-    uint64_t* q_full = ready + kTcMaxV;                     // [2] Q of a span landed
-    uint64_t* q_free = q_full + 2;                          // [2] last QK of a span done
+    uint64_t* q_full = ready + kTcMaxV;                     // a span's query rows landed in shared memory
+    uint64_t* q_cp = q_full + 1;                            // ... and were copied into tensor memory
+    uint64_t* q_free = q_cp + 1;                            // [2] last QK of a span done (tensor-memory buffer)
     uint64_t* s_full = q_free + 2;                          // [kTcSBuf] S_t in tensor memory
     uint64_t* p_full = s_full + kTcSBuf;                    // [kTcSBuf] P_t written (count 8 warps)
     uint64_t* o_ready = p_full + kTcSBuf;                   // [kTcSBuf] PV_t done (S buffer free again)
@@ -260,10 +262,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             mbar_init(&vempty[i], 1);
             mbar_init(&ready[i], 2);
         }
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(&q_full[i], 1);
-            mbar_init(&q_free[i], 1);
-        }
+        mbar_init(q_full, 1);
+        mbar_init(q_cp, 1);
+        for (int i = 0; i < 2; ++i) mbar_init(&q_free[i], 1);
         for (int i = 0; i < kTcSBuf; ++i) {
             mbar_init(&s_full[i], 1);
             mbar_init(&p_full[i], 8);
@@ -348,7 +349,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
         int span = -1;
         // tile jt goes out once its stage is free and, K side opening a
-        // piece, once the query buffer it reuses is free
+        // piece, once the query buffer is free
         int jt = 0;
         for (; jt < n_tiles; ++jt) {
             const int st = jt % S;
@@ -356,8 +357,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             const bool last = jt + 1 == n_tiles || cur.t + 1 == cur.T;
             if (first) ++span;
             bool go = jt < S || tc_wait(&emptyb[st], (uint32_t)(jt / S - 1) & 1, &s_dead, p.status);
-            if (go && k_side && first && span >= 2)
-                go = tc_wait(&q_free[span & 1], (uint32_t)((span - 2) >> 1) & 1, &s_dead, p.status);
+            // the query buffer is free once the previous span's rows are in tensor memory
+            if (go && k_side && first && span >= 1)
+                go = tc_wait(q_cp, (uint32_t)(span - 1) & 1, &s_dead, p.status);
             if (!__all_sync(0xffffffffu, go)) break;
             const int jb = jt % per_batch;
             if (jt > 0 && jb == 0) {
@@ -369,12 +371,12 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             const int ts = cur.t * kTileT;
             const int h_cur = cur.h / p.n_rb;
             if (k_side && first && lane == 0) {
-                // a new span piece: its query rows into buffer span % 2
-                mbar_arrive_expect_tx(&q_full[span & 1], 2 * qrow_bytes);
-                const uint32_t qdst = smem_u32(sq + (span & 1) * 2 * qh);
+                // a new span piece: its query rows into the query buffer
+                mbar_arrive_expect_tx(q_full, 2 * qrow_bytes);
+                const uint32_t qdst = smem_u32(sq);
 #pragma unroll
                 for (int hh = 0; hh < 2; ++hh)
-                    tma_load_4d(qdst + hh * qh, &tmap_q, &q_full[span & 1], hh * 64, h_cur * p.G, 0, p.b_base + cur.b);
+                    tma_load_4d(qdst + hh * qh, &tmap_q, q_full, hh * 64, h_cur * p.G, 0, p.b_base + cur.b);
             }
             advance(cur, s_len, nb, p.n_vh);
             int valid = 0;
@@ -449,7 +451,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         const bool qk_warp = warp == 1;
         constexpr uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, true);
         const uint64_t dq0 = tc_sw128_desc(smem_u32(sq));
-        const uint64_t qbuf16 = (uint64_t)(2 * qh) >> 4, qhalf16 = (uint64_t)qh >> 4;
+        const uint64_t qhalf16 = (uint64_t)qh >> 4;
         const uint64_t dk0 = tc_sw128_desc(smem_u32(sk)), dv0 = tc_mn_desc(smem_u32(sv));
         int span = -1, pv_piece = 0;
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);   // the PV warp's own view of the pieces
@@ -470,7 +472,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                     // a new piece: its query rows landed, and the QKs of the
                     // piece two back are done reading the query buffer
                     ++span;
-                    if (!wait_all(&q_full[span & 1], (uint32_t)(span >> 1) & 1)) break;
+                    if (!wait_all(q_full, (uint32_t)span & 1)) break;
                     if (span >= 2 && !wait_all(&q_free[span & 1], (uint32_t)((span - 2) >> 1) & 1)) break;
                 }
                 // S buffer sb held S_{t-4}: PV_{t-4} is done with it
@@ -483,10 +485,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                         // the query rows into tensor memory once per piece, 16
                         // dims (8 columns) per copy; every QK of the piece then
                         // reads only K from shared memory
-                        const uint64_t dq = dq0 + (span & 1) * qbuf16;
 #pragma unroll
                         for (int ks = 0; ks < kD / 16; ++ks)
-                            tc_cp_128x256b(tq + ks * 8, dq + (ks >> 2) * qhalf16 + (uint64_t)((ks & 3) * 2));
+                            tc_cp_128x256b(tq + ks * 8, dq0 + (ks >> 2) * qhalf16 + (uint64_t)((ks & 3) * 2));
+                        tc_commit(q_cp);   // the producer may refill the query buffer
                     }
 #pragma unroll
                     for (int ks = 0; ks < kD / 16; ++ks) {
