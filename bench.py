@@ -41,10 +41,14 @@ UNIT = "verified draft tokens/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 512 << 20
-KERNEL_SOURCES = ("paper_2607_20507_gb300/csrc/verify_attention.cu",
-                  "paper_2607_20507_gb300/csrc/verify_attention_tc.cuh",
-                  "paper_2607_20507_gb300/csrc/spec_accept.cu",
-                  "paper_2607_20507_gb300/csrc/cs_device.cuh")
+# the sources of each kernel pair whose DRAM traffic profiles/traffic.json records
+KERNEL_SOURCES = {
+    "verify_attention": ("paper_2607_20507_gb300/csrc/verify_attention.cu",
+                         "paper_2607_20507_gb300/csrc/verify_attention_tc.cuh",
+                         "paper_2607_20507_gb300/csrc/cs_device.cuh"),
+    "spec_accept": ("paper_2607_20507_gb300/csrc/spec_accept.cu",
+                    "paper_2607_20507_gb300/csrc/cs_device.cuh"),
+}
 
 
 # --------------------------------------------------------------------------
@@ -120,9 +124,9 @@ def measured_peaks() -> tuple[dict, str]:
         return {"hbm_gbs": FALLBACK_HBM_GBS}, "of fallback"
 
 
-def kernel_source_hash() -> str:
+def kernel_source_hash(kernel: str) -> str:
     h = hashlib.sha256()
-    for rel in KERNEL_SOURCES:
+    for rel in KERNEL_SOURCES[kernel]:
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
@@ -138,7 +142,7 @@ def recorded_traffic(kernel: str, workload: str) -> int | None:
     except Exception:
         return None
     e = rec.get(kernel, {}).get(workload)
-    if not e or e.get("source_hash") != kernel_source_hash():
+    if not e or e.get("source_hash") != kernel_source_hash(kernel):
         return None
     return int(e["dram_bytes_per_launch"])
 

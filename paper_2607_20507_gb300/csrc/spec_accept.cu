@@ -596,6 +596,77 @@ __device__ __forceinline__ PassScan pass_scan(const DrawRow<T>& d, bool residual
                     : pass_scan_t<T, false>(d, pass_start, end, w, s_wsum, s_wlast);
 }
 
+// Per-warp pass totals of a slice (one block-wide buffer per kernel).
+__device__ __forceinline__ float* draw_warp_pass_totals() {
+    __shared__ float s_wpass[kDrawWarps * kMaxPasses];
+    return s_wpass;
+}
+
+struct SliceMass {
+    float mass;   // the slice's mass: the pass totals added in pass order
+    int last;     // largest id of the slice with positive weight, -1 if none
+};
+
+// All n_pass passes of this CTA's slice [c0, c1), streamed without a block
+// barrier per pass: each warp folds its runs with the warp scan of pass_scan
+// and leaves its total for the pass; one barrier at the end, then every pass
+// total is the warp totals added in warp order, bit for bit the total that
+// pass_scan computes when the pass is walked again.  s_pass[ps] receives
+// them.
+template <typename T, bool kResidual>
+__device__ __forceinline__ SliceMass slice_passes_t(const DrawRow<T>& d, int c0, int c1, int n_pass, float* s_pass,
+                                                    int (&s_wlast)[kDrawWarps]) {
+    constexpr int kRun = kRunVecs * 16 / (int)sizeof(T);
+    constexpr int kPass = kDrawThreads * kRun;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    float* s_wpass = draw_warp_pass_totals();
+    float w[kRun];
+    int last = -1;
+    for (int ps = 0; ps < n_pass; ++ps) {
+        const int nx = c0 + (ps + 1) * kPass + tid * kRun;
+        if (ps + 1 < n_pass && (tid & 3) == 0 && nx < c1) {
+            // the next pass into L1 while this one is reduced (a 128-byte
+            // line holds the runs of four threads); only addresses inside the
+            // slice are touched
+            asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rt + nx));
+            if (kResidual) asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rd + nx));
+        }
+        const int start = c0 + ps * kPass + tid * kRun;
+        run_weights<T, kResidual>(d, start, c1, w);
+        float ls = 0.f;
+#pragma unroll
+        for (int e = 0; e < kRun; ++e) {
+            ls += w[e];
+            if (w[e] > 0.f) last = start + e;
+        }
+        const float incl = warp_incl_scan(ls, lane);
+        if (lane == 31) s_wpass[wid * kMaxPasses + ps] = incl;
+    }
+    last = warp_max_int(last);
+    if (lane == 0) s_wlast[wid] = last;
+    __syncthreads();
+    if (tid < n_pass) {
+        float tot = 0.f;
+#pragma unroll
+        for (int j = 0; j < kDrawWarps; ++j) tot += s_wpass[j * kMaxPasses + tid];
+        s_pass[tid] = tot;
+    }
+    SliceMass r{0.f, -1};
+#pragma unroll
+    for (int j = 0; j < kDrawWarps; ++j) r.last = max(r.last, s_wlast[j]);
+    __syncthreads();
+    for (int ps = 0; ps < n_pass; ++ps) r.mass += s_pass[ps];
+    __syncthreads();   // s_wlast / s_pass stay unchanged until every thread has read them
+    return r;
+}
+
+template <typename T>
+__device__ __forceinline__ SliceMass slice_passes(const DrawRow<T>& d, bool residual, int c0, int c1, int n_pass,
+                                                  float* s_pass, int (&s_wlast)[kDrawWarps]) {
+    return residual ? slice_passes_t<T, true>(d, c0, c1, n_pass, s_pass, s_wlast)
+                    : slice_passes_t<T, false>(d, c0, c1, n_pass, s_pass, s_wlast);
+}
+
 // ------------------------------------------------------------ the draw
 // Inverse-CDF draw of one token from the weights of row pair d -- p, or
 // max(p - rho q, 0) when `residual` (rho as folded into d) -- over the
@@ -620,23 +691,20 @@ __device__ __forceinline__ void cluster_draw(const DrawRow<T>& d, bool residual,
     token = 0;
     writer = -1;
     for (int round = 0; round < 2; ++round) {
-        float mass = 0.f;
-        int last = -1;
-        PassScan kept{0.f, 0.f, 0.f, 0.f, -1};   // the last pass, whose weights stay in w
-        for (int ps = 0; ps < n_pass; ++ps) {
-            const int nx = c0 + (ps + 1) * kPass + tid * kRun;
-            if (ps + 1 < n_pass && (tid & 3) == 0 && nx < c1) {
-                // the next pass into L1 while this one is reduced (a 128-byte
-                // line holds the runs of four threads); only addresses inside
-                // the slice are touched
-                asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rt + nx));
-                if (residual) asm volatile("prefetch.global.L1 [%0];" ::"l"(d.rd + nx));
-            }
-            kept = pass_scan<T>(d, residual, c0 + ps * kPass, c1, w, s_wsum, s_wlast);
-            if (tid == 0) s_pass[ps] = kept.total;
-            mass += kept.total;
-            last = max(last, kept.last);
+        // one pass: scanned at once, its weights and prefixes kept for the
+        // walk; several: streamed, and the owning pass walked again
+        PassScan kept{0.f, 0.f, 0.f, 0.f, -1};
+        SliceMass sm{0.f, -1};
+        if (n_pass == 1) {
+            kept = pass_scan<T>(d, residual, c0, c1, w, s_wsum, s_wlast);
+            if (tid == 0) s_pass[0] = kept.total;
+            sm.mass = kept.total;
+            sm.last = kept.last;
+        } else {
+            sm = slice_passes<T>(d, residual, c0, c1, n_pass, s_pass, s_wlast);
         }
+        const float mass = sm.mass;
+        const int last = sm.last;
         const int slot = xr & 1;
         ++xr;
         if (tid == 0) s_x[slot] = make_float2(mass, __int_as_float(last));
@@ -682,8 +750,8 @@ __device__ __forceinline__ void cluster_draw(const DrawRow<T>& d, bool residual,
             break;
         }
         tt -= cum;
-        // the weights of the last pass are still in registers; others are recomputed
-        const PassScan sc = pj == n_pass - 1 ? kept : pass_scan<T>(d, residual, c0 + pj * kPass, c1, w, s_wsum, s_wlast);
+        // walked again, the pass's scan reproduces its total bit for bit
+        const PassScan sc = n_pass == 1 ? kept : pass_scan<T>(d, residual, c0 + pj * kPass, c1, w, s_wsum, s_wlast);
         // the first run with positive mass whose prefix passes tt (a run of
         // zero weights can come first through rounding; it never owns the draw)
         const unsigned cross = __ballot_sync(0xffffffffu, sc.own > 0.f && sc.incl > tt);
@@ -841,9 +909,9 @@ __device__ __forceinline__ float cluster_mass(const DrawRow<T>& d, bool residual
                                               int (&s_wlast)[kDrawWarps], float2* s_x, int& xr) {
     constexpr int kRun = kRunVecs * 16 / (int)sizeof(T);
     constexpr int kPass = kDrawThreads * kRun;
-    float w[kRun];
-    float mass = 0.f;
-    for (int ps = 0; ps < n_pass; ++ps) mass += pass_scan<T>(d, residual, c0 + ps * kPass, c1, w, s_wsum, s_wlast).total;
+    __shared__ float s_tpass[kMaxPasses];
+    const float mass = slice_passes<T>(d, residual, c0, c1, n_pass, s_tpass, s_wlast).mass;
+    (void)s_wsum;
     const int slot = xr & 1;
     ++xr;
     if (threadIdx.x == 0) s_x[slot] = make_float2(mass, 0.f);
