@@ -417,6 +417,18 @@ cs_status cs_kv_commit_tree(const cs_attn_dims* dims, void* k_pages, void* v_pag
 #define CS_DEVICE_WAIT_TIMEOUT 1
 cs_status cs_read_device_status(const void* workspace, int32_t* status_out, cs_stream_t stream);
 
+/*
+ * Failure-detection self-test.  Enqueues one kernel whose single thread runs
+ * the bounded mbarrier wait that every wait of the attention kernels uses, on
+ * a barrier that nothing completes.  After about one second the wait gives up
+ * and the thread sets CS_DEVICE_WAIT_TIMEOUT in the status word, the first 4
+ * bytes of `workspace` (a device buffer of at least 4 bytes, 4-byte aligned,
+ * owned by the caller; nothing else in it is touched).  Read the word with
+ * cs_read_device_status.  No fault, trap or hang: the context stays usable.
+ * CS_ERR_INVALID_ARG for a NULL or misaligned workspace.
+ */
+cs_status cs_selftest_wait_timeout(void* workspace, cs_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

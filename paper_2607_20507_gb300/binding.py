@@ -18,6 +18,7 @@ from . import build as _build
 
 CS_OK, CS_ERR_INVALID_ARG, CS_ERR_UNSUPPORTED, CS_ERR_CUDA, CS_ERR_WORKSPACE = range(5)
 CS_F32, CS_BF16 = 0, 1
+CS_DEVICE_WAIT_TIMEOUT = 1   # device status bit: a bounded wait inside a kernel gave up
 STATUS_NAMES = {0: "CS_OK", 1: "CS_ERR_INVALID_ARG", 2: "CS_ERR_UNSUPPORTED", 3: "CS_ERR_CUDA",
                 4: "CS_ERR_WORKSPACE"}
 EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_workspace_bytes",
@@ -26,7 +27,7 @@ EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_work
                     "cs_sample", "cs_kv_append", "cs_kv_commit", "cs_route_workspace_bytes",
                     "cs_route_norms", "cs_route", "cs_tree_verify_attention_workspace_bytes",
                     "cs_tree_verify_attention", "cs_tree_accept_workspace_bytes", "cs_tree_accept",
-                    "cs_kv_commit_tree")
+                    "cs_kv_commit_tree", "cs_selftest_wait_timeout")
 
 
 class RouteDims(ctypes.Structure):
@@ -88,6 +89,8 @@ def load_library(path: str | None = None):
                                                     i32, vp, vp]
         lib.cs_read_device_status.restype = ctypes.c_int
         lib.cs_read_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_int32), vp]
+        lib.cs_selftest_wait_timeout.restype = ctypes.c_int
+        lib.cs_selftest_wait_timeout.argtypes = [vp, vp]
         lib.cs_kv_append.restype = ctypes.c_int
         lib.cs_kv_append.argtypes = [ctypes.POINTER(AttnDims), vp, vp, vp, vp, vp, vp, i32, vp]
         lib.cs_kv_commit.restype = ctypes.c_int
@@ -476,6 +479,14 @@ def cs_verify_attention_noalloc(q, k_pages, v_pages, page_table, ctx_lens, n_dra
                                          _stream(dev) if stream is None else stream)
     _check(lib, st)
     return out
+
+
+def cs_selftest_wait_timeout(workspace: torch.Tensor, stream: int | None = None) -> None:
+    """Runs the kernels' bounded wait on a barrier nothing completes (about one
+    second); it sets CS_DEVICE_WAIT_TIMEOUT in the workspace's status word."""
+    lib = load_library()
+    _check(lib, lib.cs_selftest_wait_timeout(_ptr(workspace),
+                                             _stream(workspace.device) if stream is None else stream))
 
 
 def cs_read_device_status(workspace: torch.Tensor, stream: int | None = None) -> int:

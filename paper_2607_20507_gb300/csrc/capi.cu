@@ -389,6 +389,14 @@ cs_status cs_sample(const cs_accept_dims* dims, const void* logits, const float*
                               nullptr, workspace, reinterpret_cast<cudaStream_t>(stream));
 }
 
+cs_status cs_selftest_wait_timeout(void* workspace, cs_stream_t stream) {
+    if (!workspace) return fail(CS_ERR_INVALID_ARG, "workspace is NULL");
+    if (!aligned(workspace, 4)) return fail(CS_ERR_INVALID_ARG, "workspace must be 4-byte aligned");
+    const cudaError_t e = launch_wait_selftest(static_cast<int*>(workspace), reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "wait self-test launch");
+    return CS_OK;
+}
+
 cs_status cs_read_device_status(const void* workspace, int32_t* status_out, cs_stream_t stream) {
     if (!workspace || !status_out) return fail(CS_ERR_INVALID_ARG, "NULL argument");
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);

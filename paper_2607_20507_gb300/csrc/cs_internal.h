@@ -36,6 +36,9 @@ AttnPlan plan_tree_attention(const cs_attn_dims& d, int n_nodes, int sm_count);
 
 // parents: NULL for the causal chain, the [B, rows] parent array for a tree
 // (must match plan.tree)
+// The failure-detection self-test (cs_selftest_wait_timeout).
+cudaError_t launch_wait_selftest(int* status, cudaStream_t stream);
+
 cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& plan, const void* q,
                                   const void* k_pages, const void* v_pages,
                                   const int32_t* page_table, const int32_t* ctx_lens,

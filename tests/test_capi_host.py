@@ -292,3 +292,9 @@ def test_tree_argument_checks(lib):
 def test_binding_fails_loudly_without_library(tmp_path):
     with pytest.raises(RuntimeError, match="not found"):
         binding.load_library(str(tmp_path / "missing.so"))
+
+
+def test_wait_selftest_argument_checks(lib):
+    # rejected on the host before anything is enqueued
+    assert lib.cs_selftest_wait_timeout(None, None) == binding.CS_ERR_INVALID_ARG
+    assert lib.cs_selftest_wait_timeout(FAKE + 2, None) == binding.CS_ERR_INVALID_ARG
