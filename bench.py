@@ -624,6 +624,78 @@ def run_reference(args) -> dict | None:
                     "d2h_bytes_per_step": 0}}
 
 
+def run_sweep(args) -> None:
+    """The sweep's cells at B >= 64 (one JSON line each): verify attention over
+    k x B at context 4096, and the acceptance over k x B x V at draft sigma
+    1.0 (the sigma changes how many positions are accepted, not the bytes the
+    kernels read).  Each cell: inputs generated on the device, the C-ABI call
+    captured in a CUDA graph, 5 untimed replays, then the median of `steps`
+    replays with the L2 flushed before each (outside the events)."""
+    from paper_2607_20507_gb300 import binding
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    binding.load_library()
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+
+    def median_us(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr):
+            fn()
+        for _ in range(5):
+            flush.zero_()
+            gr.replay()
+        ts = []
+        for _ in range(args.steps):
+            flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            gr.replay()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1) * 1e3)
+        return statistics.median(ts)
+
+    def line(kind, w, us, nbytes, extra):
+        gbs = nbytes / us / 1e3
+        print(json.dumps({"sweep": kind, "cell": w.name, "batch": w.batch, "n_draft": w.n_draft,
+                          "vocab": w.vocab if kind == "spec_accept" else None, "us": round(us, 2),
+                          "bytes": nbytes, "gbs": round(gbs, 1), "frac_of_8tbs": round(gbs / NOMINAL_HBM_GBS, 4),
+                          "frac_of_peak": round(gbs / hbm_peak, 4), "peak_source": peak_src} | extra), flush=True)
+
+    for w in W.sweep_attention_cells():
+        if w.batch < 64:
+            continue
+        att = W.attention_inputs(w, dev)
+        ws = binding.verify_attention_workspace(binding.attn_dims(att["q"], att["k_pages"], att["page_table"]),
+                                                w.n_draft, dev)
+        out = torch.empty_like(att["q"])
+        us = median_us(lambda: binding.cs_verify_attention(att["q"], att["k_pages"], att["v_pages"],
+                                                           att["page_table"], att["ctx_lens"], w.n_draft,
+                                                           out=out, workspace=ws))
+        line("verify_attention", w, us, attention_bytes(att["ctx_lens"].cpu().numpy(), w), {})
+        del att, ws, out
+        torch.cuda.empty_cache()
+    for w in W.sweep_accept_cells():
+        if w.batch < 64 or w.draft_sigma != 1.0:
+            continue
+        T = W.SWEEP_TEMPERATURE
+        acc = W.accept_inputs(w, T, dev)
+        ot = torch.empty((w.batch, w.n_draft + 1), dtype=torch.int32, device=dev)
+        on = torch.empty((w.batch,), dtype=torch.int32, device=dev)
+        us = median_us(lambda: binding.cs_spec_accept(acc["target"], acc["draft"], acc["draft_tokens"],
+                                                      acc["uniforms"], T, ot, on))
+        n_acc = on.cpu().numpy()
+        line("spec_accept", w, us, accept_bytes(n_acc, w, T)[1], {"mean_accepted": float(n_acc.mean())})
+        del acc, ot, on
+        torch.cuda.empty_cache()
+
+
 def main(argv=None) -> int:
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -637,9 +709,14 @@ def main(argv=None) -> int:
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--warmup-seconds", type=float, default=1.0,
                     help="keep warming up (and sampling clocks) for at least this long")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time the sweep's cells at B >= 64 instead (one JSON line per cell)")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)
     args.steps = max(1, args.steps)
+    if args.sweep:
+        run_sweep(args)
+        return 0
     res = run_reference(args) if args.impl == "reference" else run_gb300(args)
     if res is not None:
         print(json.dumps(res), flush=True)
