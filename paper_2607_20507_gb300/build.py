@@ -15,7 +15,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libcachespec.so")
-SOURCES = ["capi.cu", "verify_attention.cu", "spec_accept.cu", "noalloc.cu", "kv_cache.cu", "route.cu"]
+SOURCES = ["capi.cu", "verify_attention.cu", "spec_accept.cu", "noalloc.cu", "kv_cache.cu", "route.cu", "selftest.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

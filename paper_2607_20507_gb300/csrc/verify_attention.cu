@@ -1122,22 +1122,4 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     return CS_OK;
 }
 
-namespace {
-// One thread runs the bounded mbarrier wait of the kernels above on a
-// barrier that nothing arrives at: after about one second the wait gives up
-// and the thread records CS_DEVICE_WAIT_TIMEOUT, as a kernel's role would.
-__global__ void wait_selftest_kernel(int* status) {
-    __shared__ uint64_t bar;
-    if (threadIdx.x != 0) return;
-    mbar_init(&bar, 1);
-    fence_barrier_init();
-    if (!mbar_wait_bounded(&bar, 0)) atomicOr(status, CS_DEVICE_WAIT_TIMEOUT);
-}
-}  // namespace
-
-cudaError_t launch_wait_selftest(int* status, cudaStream_t stream) {
-    wait_selftest_kernel<<<1, 32, 0, stream>>>(status);
-    return cudaGetLastError();
-}
-
 }  // namespace cs
