@@ -320,6 +320,27 @@ def run_gb300(args) -> dict | None:
     t_attn = [e0.elapsed_time(e1) * 1e-3 for e0, e1, _ in ev]
     t_acc = [e1.elapsed_time(e2) * 1e-3 for _, e1, e2 in ev]
     t_step = [e0.elapsed_time(e1) * 1e-3 for e0, e1 in evs]
+
+    # configurations 1-2 also report hot-L2 times (the same graphs replayed
+    # back to back with no flush: inputs stay in the 129 MB L2); the JSON
+    # line's value stays the flushed one
+    hot_l2 = None
+    if args.workload in (1, 2):
+        def hot_mean_us(gr):
+            for _ in range(3):
+                gr.replay()
+            torch.cuda.synchronize()
+            evh = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(args.steps)]
+            for e0, e1 in evh:
+                e0.record(stream)
+                gr.replay()
+                e1.record(stream)
+            torch.cuda.synchronize()
+            return 1e3 * statistics.mean(e0.elapsed_time(e1) for e0, e1 in evh)
+        hot_l2 = {"step_us": round(hot_mean_us(g_step), 2), "attention_us": round(hot_mean_us(g_attn), 2),
+                  "accept_us": round(hot_mean_us(g_acc), 2),
+                  "note": "no L2 flush between replays: the inputs stay L2-resident; not the headline"}
     value, t_max = aggregate_throughput(float(B * k * args.steps), sum(t_step), world, dev)
     n_acc = out_n.cpu().numpy()
 
@@ -499,6 +520,7 @@ def run_gb300(args) -> dict | None:
                        "per_call_graphs_step_us": round(1e6 * statistics.mean(a + b for a, b in zip(t_attn, t_acc)), 2),
                        "direct_call_step_us": round(direct_us, 2)},
             "greedy": greedy,
+            "hot_l2": hot_l2,
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
