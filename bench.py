@@ -8,7 +8,12 @@ temperature).  The metric is verified draft tokens per second (B*k per step)
 with the achieved HBM bandwidth of the dominant kernel against the measured
 copy peak.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 2] [--impl gb300|reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 4] [--impl gb300|reference]
+
+The headline workload is configuration 4 (B = 256, k = 8, V = 128256, 64 query
+/ 8 KV heads, contexts 2K-16K, 32-token pages), the largest single-GPU
+configuration; the other serving configurations are timed in the same run
+and reported under ``per_workload``.
 
 Under torchrun (N > 1) every rank runs an independent replica on its own GPU
 with its own requests (the step shards by request; there is no collective on
@@ -41,6 +46,9 @@ UNIT = "verified draft tokens/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 512 << 20
+ATT_ATOL, ATT_RTOL = 2e-3, 1e-2      # attention output tolerance against the oracle
+NEAR_TIE_ACCEPT = 1e-5               # accept test: |u_i - p_i(x_i)/q_i(x_i)|
+NEAR_TIE_DRAW = 1e-6                 # final draw: |u_k - C/Z| at an edge of the drawn cell
 # the sources of each kernel pair whose DRAM traffic profiles/traffic.json records
 KERNEL_SOURCES = {
     "verify_attention": ("paper_2607_20507_gb300/csrc/verify_attention.cu",
@@ -212,6 +220,115 @@ class ClockSampler:
 # the GB300 arm
 # --------------------------------------------------------------------------
 
+def _events(n):
+    return [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+
+
+def capture(fn):
+    """fn run three times, then captured into a CUDA graph (host enqueue time
+    -- Python, ctypes, tensor-map encoding -- stays out of the timed replays)."""
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize()
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gr):
+        fn()
+    torch.cuda.synchronize()
+    return gr
+
+
+def flushed_times(gr, steps, flush, stream) -> list[float]:
+    """Seconds of `steps` replays of graph `gr`, the L2 flushed before each
+    (outside the events)."""
+    ev = _events(steps)
+    for e0, e1 in ev:
+        flush.zero_()
+        e0.record(stream)
+        gr.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return [e0.elapsed_time(e1) * 1e-3 for e0, e1 in ev]
+
+
+def serving_calls(w, T, dev):
+    """Inputs, output buffers and the two C-ABI calls of one workload's step."""
+    from paper_2607_20507_gb300 import binding
+    att = W.attention_inputs(w, dev)
+    acc = W.accept_inputs(w, T, dev)
+    k, B = w.n_draft, w.batch
+    ws = binding.verify_attention_workspace(binding.attn_dims(att["q"], att["k_pages"], att["page_table"]),
+                                            k, dev)
+    bufs = {"out": torch.empty_like(att["q"]),
+            "out_tok": torch.empty((B, k + 1), dtype=torch.int32, device=dev),
+            "out_n": torch.empty((B,), dtype=torch.int32, device=dev)}
+
+    def attention():
+        binding.cs_verify_attention(att["q"], att["k_pages"], att["v_pages"], att["page_table"],
+                                    att["ctx_lens"], k, out=bufs["out"], workspace=ws)
+
+    def accept(inp=acc, temp=T):
+        binding.cs_spec_accept(inp["target"], inp["draft"] if temp > 0 else None,
+                               inp["draft_tokens"], inp["uniforms"], temp, bufs["out_tok"], bufs["out_n"])
+
+    return att, acc, bufs, attention, accept
+
+
+def kernel_figures(w, T, lens, n_acc, t_attn, t_acc, hbm_peak) -> dict:
+    """Per-call time, algorithmic bytes and bandwidth of both calls of a step."""
+    ab = attention_bytes(lens, w)
+    acc_need, acc_full = accept_bytes(n_acc, w, T)
+    m_attn, m_acc = statistics.mean(t_attn), statistics.mean(t_acc)
+    return {
+        "verify_attention": {"us": round(1e6 * m_attn, 2), "bytes": ab, "gbs": round(ab / m_attn / 1e9, 1),
+                             "frac": round(ab / m_attn / 1e9 / hbm_peak, 4),
+                             "frac_of_nominal_8tbs": round(ab / m_attn / 1e9 / NOMINAL_HBM_GBS, 4),
+                             "tflops": round(attention_flops(lens, w) / m_attn / 1e12, 1)},
+        # the acceptance kernels read every row once (all positions in parallel);
+        # `needed_bytes` (rows 0..a) is what a rejection-ordered pass would touch
+        "spec_accept": {"us": round(1e6 * m_acc, 2), "bytes": acc_full, "gbs": round(acc_full / m_acc / 1e9, 1),
+                        "frac": round(acc_full / m_acc / 1e9 / hbm_peak, 4),
+                        "frac_of_nominal_8tbs": round(acc_full / m_acc / 1e9 / NOMINAL_HBM_GBS, 4),
+                        "needed_bytes": acc_need, "mean_accepted": round(float(n_acc.mean()), 4)},
+    }
+
+
+def other_workload(wid, steps, flush, stream, dev, hbm_peak) -> dict:
+    """One serving workload besides the headline one: each call in its own
+    graph, `steps` flushed replays each, and the step as one graph."""
+    w = W.WORKLOADS[wid]
+    T = max(w.temperatures)
+    att, acc, bufs, attention, accept = serving_calls(w, T, dev)
+
+    def step():
+        attention()
+        accept()
+
+    g_a, g_c, g_s = capture(attention), capture(accept), capture(step)
+    for _ in range(3):
+        flush.zero_()
+        g_s.replay()
+    t_s = flushed_times(g_s, steps, flush, stream)
+    t_a = flushed_times(g_a, steps, flush, stream)
+    t_c = flushed_times(g_c, steps, flush, stream)
+    lens = att["ctx_lens"].cpu().numpy()
+    n_acc = bufs["out_n"].cpu().numpy()
+    step_s = statistics.mean(t_s)
+    res = {"temperature": T, "batch": w.batch, "n_draft": w.n_draft,
+           "step_us": round(1e6 * step_s, 2),
+           "verified_tokens_per_s": round(w.batch * w.n_draft / step_s, 1),
+           "kernels": kernel_figures(w, T, lens, n_acc, t_a, t_c, hbm_peak)}
+    if 0.0 in w.temperatures and T > 0:
+        acc0 = W.accept_inputs(w, 0.0, dev)
+        g0 = capture(lambda: accept(acc0, 0.0))
+        t0 = flushed_times(g0, steps, flush, stream)
+        ng = bufs["out_n"].cpu().numpy()
+        res["greedy"] = kernel_figures(w, 0.0, lens, ng, t_a, t0, hbm_peak)["spec_accept"]
+        del acc0, g0
+    del att, acc, bufs, g_a, g_c, g_s
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_gb300(args) -> dict | None:
     import torch.distributed as dist
     from paper_2607_20507_gb300 import binding
@@ -222,51 +339,28 @@ def run_gb300(args) -> dict | None:
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     binding.load_library()
+    peaks, peak_src = measured_peaks()
+    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
 
     w = replica_workload(W.WORKLOADS[args.workload], rank)
     if args.batch:
         w = w.with_(batch=args.batch)
     T = args.temperature if args.temperature is not None else max(w.temperatures)
-    att = W.attention_inputs(w, dev)
-    acc = W.accept_inputs(w, T, dev)
-    acc_greedy = W.accept_inputs(w, 0.0, dev) if 0.0 in w.temperatures else None
+    att, acc, bufs, attention, accept = serving_calls(w, T, dev)
     k, B = w.n_draft, w.batch
-    ws = binding.verify_attention_workspace(binding.attn_dims(att["q"], att["k_pages"], att["page_table"]),
-                                            k, dev)
-    out = torch.empty_like(att["q"])
-    out_tok = torch.empty((B, k + 1), dtype=torch.int32, device=dev)
-    out_n = torch.empty((B,), dtype=torch.int32, device=dev)
+    out, out_tok, out_n = bufs["out"], bufs["out_tok"], bufs["out_n"]
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
 
-    def attention():
-        binding.cs_verify_attention(att["q"], att["k_pages"], att["v_pages"], att["page_table"],
-                                    att["ctx_lens"], k, out=out, workspace=ws)
-
-    def accept(inp, temp):
-        binding.cs_spec_accept(inp["target"], inp["draft"] if temp > 0 else None,
-                               inp["draft_tokens"], inp["uniforms"], temp, out_tok, out_n)
-
     def step():
         attention()
-        accept(acc, T)
+        accept()
 
     # The step is captured once into a CUDA graph (both C-ABI calls, whose
-    # kernels chain by programmatic dependent launch): the device-timed steps
-    # replay it, so that host-side enqueue time (Python, ctypes, tensor-map
-    # encoding) cannot open gaps inside the timed events.  Each call is also
-    # captured on its own, to time the two kernels' shares of the step.
-    for _ in range(3):
-        step()
-    torch.cuda.synchronize()
-    g_step, g_attn, g_acc = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_step):
-        step()
-    with torch.cuda.graph(g_attn):
-        attention()
-    with torch.cuda.graph(g_acc):
-        accept(acc, T)
-    torch.cuda.synchronize()
+    # kernels chain by programmatic dependent launch) and the timed steps
+    # replay it.  Each call is also captured on its own, to time the two
+    # calls' shares of the step.
+    g_step, g_attn, g_acc = capture(step), capture(attention), capture(accept)
 
     # warm-up: at least W steps and about a second of work, with clocks sampled
     sampler = ClockSampler(local)
@@ -282,8 +376,7 @@ def run_gb300(args) -> dict | None:
         torch.cuda.synchronize()
 
         # timed region: exactly K steps, L2 flushed between steps (outside the events)
-        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(args.steps)]
+        evs = _events(args.steps)
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
@@ -308,8 +401,7 @@ def run_gb300(args) -> dict | None:
             e2.record(stream)
         torch.cuda.synchronize()
     # the same K steps through the direct API calls (host enqueue on the path)
-    evd = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(args.steps)]
+    evd = _events(args.steps)
     for e0, e1 in evd:
         flush.zero_()
         e0.record(stream)
@@ -320,18 +412,19 @@ def run_gb300(args) -> dict | None:
     t_attn = [e0.elapsed_time(e1) * 1e-3 for e0, e1, _ in ev]
     t_acc = [e1.elapsed_time(e2) * 1e-3 for _, e1, e2 in ev]
     t_step = [e0.elapsed_time(e1) * 1e-3 for e0, e1 in evs]
+    value, t_max = aggregate_throughput(float(B * k * args.steps), sum(t_step), world, dev)
+    n_acc = out_n.cpu().numpy()
+    lens = att["ctx_lens"].cpu().numpy()
+    kernels = kernel_figures(w, T, lens, n_acc, t_attn, t_acc, hbm_peak)
 
-    # configurations 1-2 also report hot-L2 times (the same graphs replayed
-    # back to back with no flush: inputs stay in the 129 MB L2); the JSON
-    # line's value stays the flushed one
+    # hot-L2 times of the small workloads (inputs stay in the 129 MB L2)
     hot_l2 = None
-    if args.workload in (1, 2):
+    if w.wid in (1, 2):
         def hot_mean_us(gr):
             for _ in range(3):
                 gr.replay()
             torch.cuda.synchronize()
-            evh = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                   for _ in range(args.steps)]
+            evh = _events(args.steps)
             for e0, e1 in evh:
                 e0.record(stream)
                 gr.replay()
@@ -341,55 +434,20 @@ def run_gb300(args) -> dict | None:
         hot_l2 = {"step_us": round(hot_mean_us(g_step), 2), "attention_us": round(hot_mean_us(g_attn), 2),
                   "accept_us": round(hot_mean_us(g_acc), 2),
                   "note": "no L2 flush between replays: the inputs stay L2-resident; not the headline"}
-    value, t_max = aggregate_throughput(float(B * k * args.steps), sum(t_step), world, dev)
-    n_acc = out_n.cpu().numpy()
 
-    # greedy mode of the same workload (its temperature list names it)
-    greedy = None
-    if acc_greedy is not None:
-        evg = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(args.steps)]
-        for _ in range(3):
-            accept(acc_greedy, 0.0)
-        torch.cuda.synchronize()
-        g_gr = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g_gr):
-            accept(acc_greedy, 0.0)
-        for e0, e1 in evg:
-            flush.zero_()
-            e0.record(stream)
-            g_gr.replay()
-            e1.record(stream)
-        torch.cuda.synchronize()
-        tg = [e0.elapsed_time(e1) * 1e-3 for e0, e1 in evg]
-        ng = out_n.cpu().numpy()
-        gb, gfull = accept_bytes(ng, w, 0.0)
-        greedy = {"accept_us": 1e6 * statistics.mean(tg), "mean_accepted": float(ng.mean()),
-                  "gbs": gfull / statistics.mean(tg) / 1e9}
-
-    # the next rows of the path, timed on their own at this workload's shape:
-    # the KV append of the k+1 verify rows and one drafter sampling step
+    # the next rows of the path at the headline workload's shape: the KV
+    # append of the k+1 verify rows and one drafter sampling step
     def timed_graph(fn):
-        for _ in range(3):
-            fn()
-        torch.cuda.synchronize()
-        gr = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(gr):
-            fn()
-        evn = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(args.steps)]
-        for e0, e1 in evn:
-            flush.zero_()
-            e0.record(stream)
-            gr.replay()
-            e1.record(stream)
-        torch.cuda.synchronize()
-        return statistics.mean(e0.elapsed_time(e1) * 1e-3 for e0, e1 in evn)
+        return statistics.mean(flushed_times(capture(fn), args.steps, flush, stream))
 
-    gen = torch.Generator(device=dev).manual_seed(17)
-    Hkv_, D_ = att["k_pages"].shape[1], att["k_pages"].shape[3]
-    new_k = torch.randn(B, k + 1, Hkv_, D_, generator=gen, device=dev).to(torch.bfloat16)
-    new_v = torch.randn(B, k + 1, Hkv_, D_, generator=gen, device=dev).to(torch.bfloat16)
+    # the append writes back the rows the pool already holds at the k+1
+    # verify positions (the same bytes move; the pool, which the parity
+    # sample below reads, stays as the timed steps saw it)
+    Hkv_ = att["k_pages"].shape[1]
+    pos = att["ctx_lens"].long()[:, None] - (k + 1) + torch.arange(k + 1, device=dev)[None, :]
+    pg = att["page_table"].long().gather(1, pos // w.page_size)
+    new_k = att["k_pages"][pg, :, pos % w.page_size, :].contiguous()
+    new_v = att["v_pages"][pg, :, pos % w.page_size, :].contiguous()
     t_app = timed_graph(lambda: binding.cs_kv_append(new_k, new_v, att["k_pages"], att["v_pages"],
                                                      att["page_table"], att["ctx_lens"]))
     app_bytes = 2 * 2 * new_k.numel() * 2            # K and V, read the new rows and write the slots
@@ -398,10 +456,12 @@ def run_gb300(args) -> dict | None:
     d_out = torch.empty(B, dtype=torch.int32, device=dev)
     t_smp = timed_graph(lambda: binding.cs_sample(d_logits, d_u, T if T > 0 else 0.7, d_out))
     smp_bytes = d_logits.numel() * d_logits.element_size()
-    next_rows = {"kv_append": {"us": 1e6 * t_app, "bytes": app_bytes, "gbs": app_bytes / t_app / 1e9,
-                               "rows": int(B * (k + 1) * Hkv_)},
-                 "draft_sample": {"us": 1e6 * t_smp, "bytes": smp_bytes, "gbs": smp_bytes / t_smp / 1e9,
-                                  "rows": B, "vocab": int(d_logits.shape[1])}}
+    next_rows = {"kv_append": {"us": round(1e6 * t_app, 2), "bytes": app_bytes,
+                               "gbs": round(app_bytes / t_app / 1e9, 1), "rows": int(B * (k + 1) * Hkv_)},
+                 "draft_sample": {"us": round(1e6 * t_smp, 2), "bytes": smp_bytes,
+                                  "gbs": round(smp_bytes / t_smp / 1e9, 1), "rows": B,
+                                  "vocab": int(d_logits.shape[1])}}
+    del new_k, new_v, d_logits, d_u, d_out
     # the front end's semantic routing (one batch of request embeddings
     # against the group centroids), at two group-index sizes
     for rw in (W.ROUTE_WORKLOADS[2], W.ROUTE_WORKLOADS[3]):
@@ -412,11 +472,12 @@ def run_gb300(args) -> dict | None:
         flops = 2.0 * rw.batch * rw.n_groups * rw.dim
         r_bytes = (rw.batch + rw.n_groups) * rw.dim * 2 + rw.n_groups * 4 + rw.batch * 12
         next_rows[f"route_b{rw.batch}_g{rw.n_groups}"] = {
-            "us": 1e6 * t_rt, "tflops": flops / t_rt / 1e12, "flops": flops, "bytes": r_bytes,
+            "us": round(1e6 * t_rt, 2), "tflops": round(flops / t_rt / 1e12, 1), "flops": flops, "bytes": r_bytes,
+            "frac_of_bf16_peak": round(flops / t_rt / 1e12 / float(peaks.get("bf16_tflops", 1900.0)), 4),
             "hit_rate": float((r_out[0] >= 0).float().mean().item())}
         del rx, r_inv, r_out
-    # token-tree verification at the same attention geometry and vocabulary:
-    # tree attention over the paged cache and the acceptance walk
+    # token-tree verification at the B = 8 workload's attention geometry and
+    # vocabulary: tree attention over the paged cache and the acceptance walk
     tw = W.TREE_WORKLOADS[2]
     ta = W.tree_attention_inputs(tw, dev)
     t_out = torch.empty_like(ta["q"])
@@ -437,15 +498,25 @@ def run_gb300(args) -> dict | None:
     tac_bytes = tw.batch * (tw.n_nodes + internal) * tw.vocab * s_log
     next_rows[f"tree_{tw.name}"] = {
         "nodes": tw.n_nodes, "branching": list(tw.branching), "temperature": T_tree,
-        "attention_us": 1e6 * t_tat, "attention_bytes": tat_bytes, "attention_gbs": tat_bytes / t_tat / 1e9,
-        "accept_us": 1e6 * t_tac, "accept_bytes": tac_bytes, "accept_gbs": tac_bytes / t_tac / 1e9,
+        "attention_us": round(1e6 * t_tat, 2), "attention_bytes": tat_bytes,
+        "attention_gbs": round(tat_bytes / t_tat / 1e9, 1),
+        "attention_frac": round(tat_bytes / t_tat / 1e9 / hbm_peak, 4),
+        "accept_us": round(1e6 * t_tac, 2), "accept_bytes": tac_bytes,
+        "accept_gbs": round(tac_bytes / t_tac / 1e9, 1),
         "mean_accepted": float(t_na.float().mean().item())}
     del ta, tc, t_out, t_bufs
 
-    # end to end through the public API: inputs start in pinned host memory
-    host = {name: t.cpu().pin_memory() for name, t in
-            list(att.items()) + list(acc.items()) if isinstance(t, torch.Tensor)}
-    dev_bufs = {name: (att.get(name) if name in att else acc[name]) for name in host}
+    # end to end through the public API.  Every step's inputs -- the query
+    # rows, the page table and context lengths, both logit tensors, the draft
+    # tokens and the uniforms -- are copied from pinned host memory, and the
+    # emitted tokens and counts are read back.  The paged KV cache stays
+    # resident on the device (serving state that earlier steps wrote, not a
+    # per-step input).
+    step_inputs = {"q": att["q"], "page_table": att["page_table"], "ctx_lens": att["ctx_lens"],
+                   "target": acc["target"], "draft_tokens": acc["draft_tokens"], "uniforms": acc["uniforms"]}
+    if T > 0:
+        step_inputs["draft"] = acc["draft"]
+    host = {name: t.cpu().pin_memory() for name, t in step_inputs.items()}
     h2d = sum(t.numel() * t.element_size() for t in host.values())
     res_host = (torch.empty((B, k + 1), dtype=torch.int32).pin_memory(),
                 torch.empty((B,), dtype=torch.int32).pin_memory())
@@ -453,7 +524,7 @@ def run_gb300(args) -> dict | None:
 
     def e2e_step():
         for name, t in host.items():
-            dev_bufs[name].copy_(t, non_blocking=True)
+            step_inputs[name].copy_(t, non_blocking=True)
         step()
         res_host[0].copy_(out_tok, non_blocking=True)
         res_host[1].copy_(out_n, non_blocking=True)
@@ -469,36 +540,32 @@ def run_gb300(args) -> dict | None:
         e2e_step()
     e_end.record(stream)
     torch.cuda.synchronize()
-    e2e_value, _ = aggregate_throughput(float(B * k * args.steps), e_start.elapsed_time(e_end) * 1e-3,
-                                        world, dev)
+    e2e_s = e_start.elapsed_time(e_end) * 1e-3
+    e2e_value, _ = aggregate_throughput(float(B * k * args.steps), e2e_s, world, dev)
+
+    # the other serving workloads, each timed the same way (not the headline)
+    per_workload = {}
+    if not args.no_per_workload:
+        for wid in sorted(W.WORKLOADS):
+            if wid != w.wid:
+                per_workload[W.WORKLOADS[wid].name] = other_workload(wid, args.steps, flush, stream, dev, hbm_peak)
 
     # roofline of the dominant kernel (the one with the larger share of the step)
-    lens = att["ctx_lens"].cpu().numpy()
-    peaks, peak_src = measured_peaks()
-    hbm_peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
-    ab = attention_bytes(lens, w)
-    acc_need, acc_full = accept_bytes(n_acc, w, T)
-    m_attn, m_acc = statistics.mean(t_attn), statistics.mean(t_acc)
-    kernels = {
-        "verify_attention": {"us": 1e6 * m_attn, "bytes": ab, "gbs": ab / m_attn / 1e9,
-                             "tflops": attention_flops(lens, w) / m_attn / 1e12},
-        # the acceptance kernels read every row once (all positions in parallel);
-        # `needed_bytes` (rows 0..a) is what a rejection-ordered pass would touch
-        "spec_accept": {"us": 1e6 * m_acc, "bytes": acc_full, "gbs": acc_full / m_acc / 1e9,
-                        "needed_bytes": acc_need, "mean_accepted": float(n_acc.mean())},
-    }
-    dom = "verify_attention" if m_attn >= m_acc else "spec_accept"
-    dom_bytes = ab if dom == "verify_attention" else acc_full
-    dom_t = m_attn if dom == "verify_attention" else m_acc
-    achieved = dom_bytes / dom_t / 1e9
+    dom = "verify_attention" if kernels["verify_attention"]["us"] >= kernels["spec_accept"]["us"] else "spec_accept"
+    achieved = kernels[dom]["bytes"] / (kernels[dom]["us"] * 1e-6) / 1e9
     roofline = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
                 "unit": "GB/s", "frac": round(achieved / hbm_peak, 4), "peak_source": peak_src,
                 "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
-                "traffic": recorded_traffic(dom, w.name)}
+                "traffic": recorded_traffic(dom, w.name),
+                "algorithmic_bytes_per_launch": kernels[dom]["bytes"],
+                "us_per_launch": kernels[dom]["us"]}
 
     result = None
     if rank == 0:
-        cpu = None if args.no_cpu_baseline else oracle_baseline(w, T, att, acc, seconds_budget=20.0)
+        cpu, parity = (None, None)
+        if not args.no_cpu_baseline:
+            cpu, parity = oracle_baseline(w, T, att, acc, out, out_tok, out_n,
+                                          seconds_budget=args.cpu_seconds)
         result = {
             "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup,
@@ -513,20 +580,24 @@ def run_gb300(args) -> dict | None:
                        "l2": "flushed between steps (512 MiB memset outside the timed events)",
                        "parallelism": f"replicas x{world} (requests shard; no collective)"},
             "kernels": kernels,
+            "emitted_tokens_per_s": round(float((n_acc + 1).sum()) * args.steps / t_max, 1),
+            "per_workload": per_workload,
             "next_rows": next_rows,
             "launch": {"timed_steps": "CUDA-graph replay of one step (both C-ABI calls in one graph; "
                                       "kernels chained by programmatic dependent launch)",
                        "kernel_times": "each C-ABI call in its own graph, the same K steps",
                        "per_call_graphs_step_us": round(1e6 * statistics.mean(a + b for a, b in zip(t_attn, t_acc)), 2),
                        "direct_call_step_us": round(direct_us, 2)},
-            "greedy": greedy,
             "hot_l2": hot_l2,
             "roofline": roofline,
             "cpu_baseline": cpu,
+            "parity_sample": parity,
             "e2e": {"value": round(e2e_value, 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h,
-                    "note": "host->device copy of every input from pinned memory and device->host "
-                            "read of the emitted tokens inside the timed region"},
+                    "d2h_bytes_per_step": d2h, "ms_per_step": round(1e3 * e2e_s / args.steps, 4),
+                    "note": "per step: host->device copy from pinned memory of the query rows, page table, "
+                            "context lengths, target and draft logits, draft tokens and uniforms; the two "
+                            "C-ABI calls; device->host read of the emitted tokens and counts.  The paged KV "
+                            "cache stays resident on the device (serving state, not a per-step input)"},
             # per step: the verify-attention kernel and its split merge (one pair per
             # 1024-request slice), the acceptance statistics kernel and the draw
             # kernel (one launch per 65535 requests)
@@ -539,19 +610,41 @@ def run_gb300(args) -> dict | None:
     return result
 
 
-def oracle_baseline(w, T, att, acc, seconds_budget=20.0) -> dict:
-    """The fp64 oracle on the host cores over a bounded sample of the workload."""
+def parity_counts(out_tok, out_n, e_tok, e_n, accept_margin, draw_margin) -> dict:
+    """Acceptance parity of GPU outputs against the oracle's on the same
+    requests: near-ties (accept tests with |u - p/q| < 1e-5, draws with u_k
+    within 1e-6 of an edge of the drawn cell) are counted, and so are the
+    requests that differ inside and outside those bands."""
+    mism = np.any(out_tok != e_tok, axis=1) | (out_n != e_n)
+    tie_a = accept_margin < NEAR_TIE_ACCEPT
+    tie_d = draw_margin < NEAR_TIE_DRAW
+    tie = tie_a | tie_d
+    return {"requests": int(len(e_n)), "near_ties_accept": int(tie_a.sum()), "near_ties_draw": int(tie_d.sum()),
+            "near_ties_differ": int((mism & tie).sum()), "differ_outside_band": int((mism & ~tie).sum())}
+
+
+def oracle_baseline(w, T, att, acc, out, out_tok, out_n, seconds_budget=15.0) -> tuple[dict, dict]:
+    """The fp64 oracle on the host cores over a bounded, seeded request sample
+    of the workload: its throughput (the cpu_baseline), and the GPU outputs of
+    the same requests compared with its results (attention element by
+    element against 2e-3 + 1e-2|ref|; tokens and counts exactly, near-ties
+    counted)."""
     import oracle
     cores = os.cpu_count() or 1
     oracle.set_threads(cores)
     B = w.batch
-    # grow the request sample until the budget is used (at least one request)
+    g_out = out.float().cpu().numpy()
+    g_tok, g_n = out_tok.cpu().numpy(), out_n.cpu().numpy()
     n = 1
     spent = 0.0
     done = 0
     rng = np.random.default_rng(0)
     order = rng.permutation(B)
-    while done < B and spent < seconds_budget:
+    att_bad = att_n = 0
+    worst = 0.0
+    cmp_tok, cmp_n, cmp_am, cmp_dm, cmp_et, cmp_en = [], [], [], [], [], []
+    passes = 0
+    while spent < seconds_budget and (done < B or passes == 0):
         take = order[done:done + n].tolist()
         sa = W.attention_subset(att, take)
         sc = W.accept_subset(acc, take)
@@ -560,31 +653,46 @@ def oracle_baseline(w, T, att, acc, seconds_budget=20.0) -> dict:
         c_host = (W.host_bits(sc["target"]), W.host_bits(sc["draft"]) if T > 0 else None,
                   sc["draft_tokens"].cpu().numpy(), sc["uniforms"].cpu().numpy())
         t0 = time.perf_counter()
-        oracle.verify_attention(*a_host, w.n_draft)
-        oracle.spec_accept(*c_host, T)
+        e_out = oracle.verify_attention(*a_host, w.n_draft)
+        e_tok, e_n, am, dm = oracle.spec_accept(*c_host, T, with_draw_margin=True)
         spent += time.perf_counter() - t0
+        err = np.abs(g_out[take] - e_out)
+        tol = ATT_ATOL + ATT_RTOL * np.abs(e_out)
+        att_bad += int((err > tol).sum()) + int((~np.isfinite(g_out[take])).sum())
+        att_n += err.size
+        worst = max(worst, float((err / tol).max()) if err.size else 0.0)
+        cmp_tok.append(g_tok[take])
+        cmp_n.append(g_n[take])
+        cmp_et.append(e_tok)
+        cmp_en.append(e_n)
+        cmp_am.append(am)
+        cmp_dm.append(dm)
         done += len(take)
-        n = min(2 * n, B - done) if done < B else n
-    # a workload the oracle finishes quickly is repeated until about ten
-    # seconds of CPU work are measured
-    passes = 1 if done >= B else 0
-    if done >= B and spent < 10.0:
-        a_host = (W.host_bits(att["q"]), W.host_bits(att["k_pages"]), W.host_bits(att["v_pages"]),
-                  att["page_table"].cpu().numpy(), att["ctx_lens"].cpu().numpy())
-        c_host = (W.host_bits(acc["target"]), W.host_bits(acc["draft"]) if T > 0 else None,
-                  acc["draft_tokens"].cpu().numpy(), acc["uniforms"].cpu().numpy())
-        while spent < 10.0:
-            t0 = time.perf_counter()
-            oracle.verify_attention(*a_host, w.n_draft)
-            oracle.spec_accept(*c_host, T)
-            spent += time.perf_counter() - t0
-            done += B
+        if done >= B:
+            # a workload the oracle finishes quickly is repeated until about
+            # ten seconds of CPU work are measured
             passes += 1
-    value = done * w.n_draft / spent
-    what = (f"{passes} passes over all {B} requests" if passes else f"{done} of {B} requests")
-    return {"value": round(value, 2), "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{what} of {w.name} (attention + acceptance, fp64, "
-                      f"OpenMP over requests/heads), {spent:.2f} s"}
+            if spent >= 10.0:
+                break
+            done = 0
+            n = B
+        else:
+            n = min(2 * n, B - done)
+    n_req = sum(len(x) for x in cmp_n)
+    value = n_req * w.n_draft / spent
+    what = (f"{passes} passes over all {B} requests" if passes else
+            f"a seeded sample of {n_req} of {B} requests")
+    cpu = {"value": round(value, 2), "unit": UNIT, "cores": cores, "kind": "oracle",
+           "sample": f"{what} of {w.name} (attention + acceptance, fp64, "
+                     f"OpenMP over requests/heads), {spent:.2f} s"}
+    acc_par = parity_counts(np.concatenate(cmp_tok), np.concatenate(cmp_n), np.concatenate(cmp_et),
+                            np.concatenate(cmp_en), np.concatenate(cmp_am), np.concatenate(cmp_dm))
+    parity = {"sample": what,
+              "verify_attention": {"requests": n_req, "elements": att_n, "outside_tolerance": att_bad,
+                                   "worst_err_over_tol": round(worst, 4),
+                                   "tolerance": "|gpu - oracle| <= 2e-3 + 1e-2|oracle|"},
+              "spec_accept": acc_par | {"bands": "accept |u - p/q| < 1e-5; draw |u_k - C/Z| < 1e-6"}}
+    return cpu, parity
 
 
 # --------------------------------------------------------------------------
@@ -600,13 +708,17 @@ def run_reference(args) -> dict | None:
     T = args.temperature if args.temperature is not None else max(w.temperatures)
     cores = os.cpu_count() or 1
     oracle.set_threads(cores)
-    att = W.attention_inputs(w, "cpu")
-    acc = W.accept_inputs(w, T, "cpu")
+    # inputs drawn where the GPU arm draws them (the same seeded values; on a
+    # host without a GPU, the CPU generators); only the sampled requests are
+    # copied to the host, and the timing covers the oracle alone
+    gen_dev = "cuda" if torch.cuda.is_available() else "cpu"
+    att = W.attention_inputs(w, gen_dev)
+    acc = W.accept_inputs(w, T, gen_dev)
     # each step is a bounded sample: as many requests as fit about 2 s of oracle work
-    take = list(range(w.batch))
+    take = np.random.default_rng(0).permutation(w.batch).tolist()
     probe = W.attention_subset(att, take[:1])
     ph = (W.host_bits(probe["q"]), W.host_bits(probe["k_pages"]), W.host_bits(probe["v_pages"]),
-          probe["page_table"].numpy(), probe["ctx_lens"].numpy())
+          probe["page_table"].cpu().numpy(), probe["ctx_lens"].cpu().numpy())
     t0 = time.perf_counter()
     oracle.verify_attention(*ph, w.n_draft)
     per_req = max(time.perf_counter() - t0, 1e-4)
@@ -614,9 +726,10 @@ def run_reference(args) -> dict | None:
     sa = W.attention_subset(att, take[:n_req])
     sc = W.accept_subset(acc, take[:n_req])
     a_host = (W.host_bits(sa["q"]), W.host_bits(sa["k_pages"]), W.host_bits(sa["v_pages"]),
-              sa["page_table"].numpy(), sa["ctx_lens"].numpy())
+              sa["page_table"].cpu().numpy(), sa["ctx_lens"].cpu().numpy())
     c_host = (W.host_bits(sc["target"]), W.host_bits(sc["draft"]) if T > 0 else None,
-              sc["draft_tokens"].numpy(), sc["uniforms"].numpy())
+              sc["draft_tokens"].cpu().numpy(), sc["uniforms"].cpu().numpy())
+    del att, acc
 
     def step():
         oracle.verify_attention(*a_host, w.n_draft)
@@ -631,7 +744,7 @@ def run_reference(args) -> dict | None:
         times.append(time.perf_counter() - t0)
     total = sum(times)
     value = n_req * w.n_draft * args.steps / total
-    sample = (f"{n_req} of {w.batch} requests of {w.name} per step (attention + acceptance, fp64, "
+    sample = (f"a seeded sample of {n_req} of {w.batch} requests of {w.name} per step (attention + acceptance, fp64, "
               f"OpenMP on {cores} host threads)")
     return {"impl": "reference", "metric": METRIC, "value": round(value, 3), "unit": UNIT,
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
@@ -721,14 +834,19 @@ def run_sweep(args) -> None:
 def main(argv=None) -> int:
     ap = argparse.ArgumentParser(description=__doc__.splitlines()[0])
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--workload", type=int, default=2, choices=sorted(W.WORKLOADS))
+    ap.add_argument("--workload", type=int, default=4, choices=sorted(W.WORKLOADS),
+                    help="the headline workload (default 4: B = 256, the largest single-GPU configuration)")
     ap.add_argument("--temperature", type=float, default=None)
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (smaller cases for profiling)")
     ap.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-per-workload", action="store_true",
+                    help="skip timing the other serving workloads")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0,
+                    help="budget of the oracle's request sample (cpu_baseline and parity_sample)")
     ap.add_argument("--warmup-seconds", type=float, default=1.0,
                     help="keep warming up (and sampling clocks) for at least this long")
     ap.add_argument("--sweep", action="store_true",

@@ -36,7 +36,8 @@
  * Conventions for every entry point
  *   - All tensor arguments are DEVICE pointers owned by the caller, dense
  *     row-major in the layouts stated below.  The library never allocates,
- *     frees or synchronises (except cs_read_device_status, which says so).
+ *     frees or synchronises (except the status reads cs_read_device_status
+ *     and cs_verify_attention_noalloc_status, which say so).
  *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL is the legacy
  *     default stream) and return once the work is enqueued.
  *   - Arguments are checked on the host before anything is enqueued; a bad
@@ -225,6 +226,18 @@ cs_status cs_verify_attention_noalloc(const cs_attn_dims* dims, const void* q, c
                                       const void* v_pages, const int32_t* page_table,
                                       const int32_t* ctx_lens, int32_t n_draft, void* out,
                                       cs_stream_t stream);
+
+/*
+ * Device status word of the allocation-free entry point on the current
+ * device (the counterpart of cs_read_device_status, whose workspace the
+ * caller of cs_verify_attention_noalloc does not have): 0, or the CS_DEVICE_*
+ * bits of the latest cs_verify_attention_noalloc call enqueued before it on
+ * `stream` (each call clears the word first, so a bit names that call's
+ * failure: its output is invalid).  Copies 4 bytes to the host and
+ * SYNCHRONISES `stream`; allocates nothing.  The paper has no counterpart.
+ * CS_ERR_INVALID_ARG for a NULL status_out, CS_ERR_CUDA on a copy failure.
+ */
+cs_status cs_verify_attention_noalloc_status(int32_t* status_out, cs_stream_t stream);
 
 /*
  * Paged KV cache around the verify pass (Sec. 3.4's draft-and-verify step).

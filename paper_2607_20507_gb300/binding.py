@@ -23,7 +23,8 @@ STATUS_NAMES = {0: "CS_OK", 1: "CS_ERR_INVALID_ARG", 2: "CS_ERR_UNSUPPORTED", 3:
                 4: "CS_ERR_WORKSPACE"}
 EXPORTED_SYMBOLS = ("cs_abi_version", "cs_last_error", "cs_verify_attention_workspace_bytes",
                     "cs_verify_attention", "cs_spec_accept_workspace_bytes", "cs_spec_accept",
-                    "cs_read_device_status", "cs_verify_attention_noalloc", "cs_sample_workspace_bytes",
+                    "cs_read_device_status", "cs_verify_attention_noalloc", "cs_verify_attention_noalloc_status",
+                    "cs_sample_workspace_bytes",
                     "cs_sample", "cs_kv_append", "cs_kv_commit", "cs_route_workspace_bytes",
                     "cs_route_norms", "cs_route", "cs_tree_verify_attention_workspace_bytes",
                     "cs_tree_verify_attention", "cs_tree_accept_workspace_bytes", "cs_tree_accept",
@@ -87,6 +88,8 @@ def load_library(path: str | None = None):
         lib.cs_verify_attention_noalloc.restype = ctypes.c_int
         lib.cs_verify_attention_noalloc.argtypes = [ctypes.POINTER(AttnDims), vp, vp, vp, vp, vp,
                                                     i32, vp, vp]
+        lib.cs_verify_attention_noalloc_status.restype = ctypes.c_int
+        lib.cs_verify_attention_noalloc_status.argtypes = [ctypes.POINTER(ctypes.c_int32), vp]
         lib.cs_read_device_status.restype = ctypes.c_int
         lib.cs_read_device_status.argtypes = [vp, ctypes.POINTER(ctypes.c_int32), vp]
         lib.cs_selftest_wait_timeout.restype = ctypes.c_int
@@ -495,4 +498,14 @@ def cs_read_device_status(workspace: torch.Tensor, stream: int | None = None) ->
     v = ctypes.c_int32(0)
     _check(lib, lib.cs_read_device_status(_ptr(workspace), ctypes.byref(v),
                                           _stream(workspace.device) if stream is None else stream))
+    return int(v.value)
+
+
+def cs_verify_attention_noalloc_status(device=None, stream: int | None = None) -> int:
+    """Status word of the allocation-free entry point on the current device: the
+    CS_DEVICE_* bits of its latest call (synchronises the stream)."""
+    lib = load_library()
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    v = ctypes.c_int32(0)
+    _check(lib, lib.cs_verify_attention_noalloc_status(ctypes.byref(v), _stream(dev) if stream is None else stream))
     return int(v.value)

@@ -76,3 +76,19 @@ extern "C" cs_status cs_verify_attention_noalloc(const cs_attn_dims* dims, const
     return cs_verify_attention(dims, q, k_pages, v_pages, page_table, ctx_lens, n_draft, out,
                                scratch, CS_NOALLOC_SCRATCH_BYTES, stream);
 }
+
+// The status word at the start of the scratch array, read back for the
+// caller (who never sees the array's address): the CS_DEVICE_* bits of the
+// latest allocation-free call on this device.
+extern "C" cs_status cs_verify_attention_noalloc_status(int32_t* status_out, cs_stream_t stream) {
+    if (!status_out) return cs::fail(CS_ERR_INVALID_ARG, "status_out is NULL");
+    void* scratch = nullptr;
+    cs_status st = scratch_address(&scratch);
+    if (st != CS_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(status_out, scratch, sizeof(int32_t), cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return cs::cuda_fail(e, "cudaMemcpyAsync(noalloc status)");
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cs::cuda_fail(e, "cudaStreamSynchronize");
+    return CS_OK;
+}

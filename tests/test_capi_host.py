@@ -298,3 +298,8 @@ def test_wait_selftest_argument_checks(lib):
     # rejected on the host before anything is enqueued
     assert lib.cs_selftest_wait_timeout(None, None) == binding.CS_ERR_INVALID_ARG
     assert lib.cs_selftest_wait_timeout(FAKE + 2, None) == binding.CS_ERR_INVALID_ARG
+
+
+def test_noalloc_status_rejects_a_null_output(lib):
+    assert lib.cs_verify_attention_noalloc_status(None, None) == binding.CS_ERR_INVALID_ARG
+    assert b"NULL" in lib.cs_last_error()

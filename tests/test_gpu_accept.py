@@ -24,8 +24,7 @@ from paper_2607_20507_gb300 import workloads as W
 pytestmark = pytest.mark.gpu
 
 DEV = "cuda:0"
-NEAR_TIE = 1e-5          # accept test: |u - p/q|
-DRAW_TIE = 1e-6          # draw: |u_k - C/Z| at the edges of the drawn cell
+from parity_bands import DRAW_TIE, NEAR_TIE, check_tie_rate
 
 
 def gpu(inp, T):
@@ -52,6 +51,7 @@ def assert_parity(inp, T, what=""):
     assert not bad.any(), (f"{what}: {int(bad.sum())} requests differ outside the near-tie band; "
                            f"first {np.nonzero(bad)[0][:5].tolist()}")
     print(f"{what}: {len(n)} requests, near-ties {int(tie.sum())}, of which differ {int((mism & tie).sum())}")
+    check_tie_rate(int(tie.sum()), len(n), what)
     # structure of every GPU output, ties included
     k = out.shape[1] - 1
     V = inp["target"].shape[2]
@@ -81,6 +81,35 @@ def test_sweep_cells(sigma, k, B, V):
              if c.draft_sigma == sigma and c.n_draft == k and c.batch == B and c.vocab == V)
     inp = W.accept_inputs(w, W.SWEEP_TEMPERATURE, DEV)
     assert_parity(inp, W.SWEEP_TEMPERATURE, w.name)
+
+
+def stratified_sweep_cells():
+    """At each of B = 64, 256 and 512: five cells that between them take every
+    k, every draft sigma and every vocabulary of the sweep once."""
+    cells = []
+    for bi, B in enumerate((64, 256, 512)):
+        for i, k in enumerate(W.SWEEP_KS):
+            sigma = W.SWEEP_SIGMAS[(i + bi) % 5]
+            V = W.SWEEP_VOCABS[(i + bi) % 3]
+            cells.append((sigma, k, B, V))
+    return cells
+
+
+@pytest.mark.parametrize("sigma,k,B,V", stratified_sweep_cells())
+def test_sweep_stratified_at_serving_batches(sigma, k, B, V):
+    """The launch at full size; the oracle on a seeded sample of 24 requests."""
+    w = next(c for c in W.sweep_accept_cells()
+             if c.draft_sigma == sigma and c.n_draft == k and c.batch == B and c.vocab == V)
+    T = W.SWEEP_TEMPERATURE
+    inp = W.accept_inputs(w, T, DEV)
+    out, n = gpu(inp, T)
+    idx = sorted(np.random.default_rng(w.cell).choice(B, 24, replace=False).tolist())
+    sub = W.accept_subset(inp, idx)
+    eo, en, tie = ref(sub, T)
+    mism = np.any(out[idx] != eo, axis=1) | (n[idx] != en)
+    assert not (mism & ~tie).any(), f"{w.name}: requests {np.nonzero(mism & ~tie)[0].tolist()} differ"
+    check_tie_rate(int(tie.sum()), len(idx), w.name)
+    assert (out[np.arange(B), n] >= 0).all() and (n >= 0).all() and (n <= k).all()
 
 
 def custom(B, k, V, dtype, T, sigma=1.0, cell=0):

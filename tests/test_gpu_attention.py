@@ -76,17 +76,20 @@ def test_workload_4_sampled_requests():
     w = W.WORKLOADS[4]
     inp = W.attention_inputs(w, DEV)
     out = gpu(inp)
-    idx = sorted(np.random.default_rng(4).choice(w.batch, 8, replace=False).tolist())
+    idx = sorted(np.random.default_rng(4).choice(w.batch, 24, replace=False).tolist())
     sub = W.attention_subset(inp, idx)
     assert_parity(out[idx], ref(sub), "workload 4 sample")
 
 
-@pytest.mark.parametrize("k,B", [(16, 512), (1, 512), (8, 64)])
+@pytest.mark.parametrize("k,B", [(k, B) for k in W.SWEEP_KS for B in W.SWEEP_BATCHES])
 def test_sweep_attention_cells_sampled(k, B):
+    """Every attention cell of the sweep (context 4096): the launch at full
+    size, the oracle on a seeded sample of up to 3 requests."""
     w = next(c for c in W.sweep_attention_cells() if c.n_draft == k and c.batch == B)
     inp = W.attention_inputs(w, DEV)
     out = gpu(inp)
-    idx = sorted(np.random.default_rng(k * 1000 + B).choice(B, 4, replace=False).tolist())
+    n = min(3, B)
+    idx = sorted(np.random.default_rng(k * 1000 + B).choice(B, n, replace=False).tolist())
     assert_parity(out[idx], ref(W.attention_subset(inp, idx)), w.name)
 
 

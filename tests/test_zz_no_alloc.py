@@ -32,6 +32,12 @@ def noalloc(lib, inp, out):
                                          torch.cuda.current_stream().cuda_stream)
     assert st == binding.CS_OK, lib.cs_last_error().decode()
     torch.cuda.synchronize()
+    # the call's device status word (in the library's scratch, which the
+    # caller cannot address): no bounded wait gave up
+    status = ctypes.c_int32(-1)
+    st = lib.cs_verify_attention_noalloc_status(ctypes.byref(status), torch.cuda.current_stream().cuda_stream)
+    assert st == binding.CS_OK, lib.cs_last_error().decode()
+    assert status.value == 0
     return out
 
 
