@@ -5,11 +5,18 @@ two narrow bands where fp32 and fp64 may legitimately decide differently:
 * an accept test with |u_i - p_i(x_i)/q_i(x_i)| < 1e-5 (the band the
   acceptance rule's tolerance names);
 * a final draw with u_k within 1e-6 of either CDF value that brackets the
-  drawn token (the kernels' fp32 running sums resolve the CDF to ~1e-8).
-Requests in a band are counted; they must stay rare, so that a kernel that
-drifts into the bands still fails: at most 1% of the requests (at least 2
-allowed, for small samples).  With uniform u the expected rate is about
-2e-5 per accept test, far below that bound.
+  drawn token.  The kernels weigh each token by 2^((z - m) c) in fp32: the
+  rounding of the exponent's argument alone moves a weight by up to ~1e-6
+  relative, so the CDF may move by that much where a few tokens carry most
+  of the mass (measured mismatches sit below 1e-7).
+
+Which requests fall in a band is a property of the inputs (the oracle's own
+fp64 margins), not of the kernel: with V tokens a uniform lands within 1e-6
+of one of the V + 1 CDF edges with probability up to 2e-6 (V + 1), so at
+V = 128K several percent of the draws are near-ties.  What a drifting kernel
+changes is how many of those requests come out DIFFERENT: that count is
+bounded (at most 1% of the requests compared, and at least 2 allowed for
+small samples); in measurements it is about 0.2% at V = 256000.
 """
 import math
 
@@ -17,11 +24,11 @@ NEAR_TIE = 1e-5
 DRAW_TIE = 1e-6
 
 
-def max_near_ties(n_requests: int) -> int:
+def max_band_mismatches(n_requests: int) -> int:
     return max(2, math.ceil(0.01 * n_requests))
 
 
-def check_tie_rate(n_ties: int, n_requests: int, what: str = "") -> None:
-    assert n_ties <= max_near_ties(n_requests), (
-        f"{what}: {n_ties} of {n_requests} requests fall in a near-tie band "
-        f"(at most {max_near_ties(n_requests)} allowed)")
+def check_band_mismatches(n_differ: int, n_requests: int, what: str = "") -> None:
+    assert n_differ <= max_band_mismatches(n_requests), (
+        f"{what}: {n_differ} of {n_requests} requests differ from the oracle inside a near-tie band "
+        f"(at most {max_band_mismatches(n_requests)} allowed)")

@@ -58,6 +58,9 @@ def one(w, T) -> dict:
     del inp, sub
     torch.cuda.empty_cache()
     return {"config": w.name, "temperature": T, "batch": B, "compared": len(idx),
+            "draw_margin_le_1e-7": int((dm < 1e-7).sum()), "draw_margin_le_1e-8": int((dm < 1e-8).sum()),
+            "differ_max_draw_margin": float(dm[mism].max()) if mism.any() else None,
+            "differ_max_accept_margin": float(am[mism].max()) if mism.any() else None,
             "near_ties_accept": int(ta.sum()), "near_ties_draw": int(td.sum()),
             "near_ties_differ": int((mism & tie).sum()), "differ_outside_band": int((mism & ~tie).sum()),
             "mean_accepted": float(en.mean())}

@@ -18,7 +18,7 @@ from paper_2607_20507_gb300 import workloads as W
 pytestmark = pytest.mark.gpu
 
 DEV = "cuda:0"
-from parity_bands import DRAW_TIE, NEAR_TIE, check_tie_rate
+from parity_bands import DRAW_TIE, NEAR_TIE, check_band_mismatches
 
 
 def random_parents(rng, B, n, detach=0.0):
@@ -121,7 +121,7 @@ def assert_accept_parity(inp, T, what):
     mism = np.any(tok != r["tokens"], axis=1) | np.any(path != r["path"], axis=1) | (n != r["n_accepted"])
     bad = mism & ~tie
     assert not bad.any(), f"{what}: {int(bad.sum())} requests differ outside the near-tie band"
-    check_tie_rate(int(tie.sum()), len(n), what)
+    check_band_mismatches(int((mism & tie).sum()), len(n), what)
     print(f"{what}: {len(n)} requests, mean accepted {n.mean():.2f}, near-ties {int(tie.sum())}, "
           f"of which differ {int((mism & tie).sum())}")
     nn = tok.shape[1]
