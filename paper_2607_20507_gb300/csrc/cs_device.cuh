@@ -161,6 +161,21 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Two fp32 values (low half first) as the sum of two bf16 pairs: hi = bf16(x),
+// lo = bf16(x - hi).  The pair carries ~16 significant bits of x, so a product
+// against bf16 data taken as hi.V + lo.V is finer than an fp16 operand
+// (11 bits) and, unlike fp16, covers bf16's whole exponent range.
+__device__ __forceinline__ void split_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+    hi = pack_bf16x2(x0, x1);
+    lo = pack_bf16x2(x0 - __uint_as_float(hi << 16), x1 - __uint_as_float(hi & 0xffff0000u));
+}
+
+// The attention weights P are formed as 2^(x - kPShift) with x <= 8: P * 2^-64.
+// The row sum carries the same factor, so it cancels in the normalised output,
+// and no partial sum of P.V can overflow fp32 even for V entries near bf16's
+// largest value (~3.39e38); weights below 2^-62 of the row's largest vanish.
+constexpr float kPShift = 64.f;
+
 // ------------------------------------------------------------- MUFU math
 // 2^x on the special-function unit (flushes subnormal results to zero).
 __device__ __forceinline__ float ex2(float x) {

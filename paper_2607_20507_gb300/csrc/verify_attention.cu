@@ -9,10 +9,10 @@
 // takes the contiguous tile range [c*W/G, (c+1)*W/G) of the W tiles, so every
 // CTA streams the same number of tiles whatever the context lengths.  A span
 // that lies inside one CTA's range is finished there and written in bf16;
-// a span cut by range boundaries leaves one (O, m, l) partial per piece (each
-// CTA writes at most two: its first and its last piece), and a second small
-// kernel merges the pieces of every cut span with log-sum-exp weights, all
-// spans in parallel.
+// a span cut by range boundaries leaves one partial per piece -- the piece's
+// own normalised output and its (m, l) -- (each CTA writes at most two: its
+// first and its last piece), and a second small kernel merges the pieces of
+// every cut span with log-sum-exp weights, all spans in parallel.
 //
 // Token trees (the multi-candidate verification variant) use the same
 // kernel with a different mask: node i of a request's tree sees every prefix
@@ -34,18 +34,20 @@
 // of up to 64 keys of one page and head, landing as [half][key][64 dims]
 // with the 128-byte swizzle, so a 16-token page is one 4 KB copy.  The page
 // ids of the next 32 / pieces tiles come from one warp-wide load issued a
-// batch ahead, and the page table is prefetched into L2 at launch.  Consumer warps own 16 of the (k+1)*G query rows of
-// the current span each (draft row i = r / G, query head h*G + r % G), so
-// every K/V byte staged in shared memory serves all rows; they run S = Q K^T
-// on bf16 tensor cores and O += P V on fp16 ones (mma.sync m16n8k16, fp32
-// accumulate; P rounded to fp16, V converted from bf16 -- in shared memory by
-// the producer warp, or in registers by key-split consumers -- which is exact
-// for values inside fp16's range) with an fp32 online softmax in the log2
-// domain.  fp16 P is eight times finer than bf16: with bf16 P the
-// rounding of the weights alone can exceed 2e-3 + 1e-2|o| on rows whose
-// terms cancel.
+// batch ahead, and the page table is prefetched into L2 at launch.
+// Consumer warps own 16 of the (k+1)*G query rows of the current span each
+// (draft row i = r / G, query head h*G + r % G), so every K/V byte staged in
+// shared memory serves all rows; they run S = Q K^T and O += P V on bf16
+// tensor cores (mma.sync m16n8k16, fp32 accumulate) with an fp32 online
+// softmax in the log2 domain.  V is used as stored; P enters the product as
+// the sum of two bf16 terms (hi + lo, ~16 significant bits: bf16 P alone
+// rounds the weights coarsely enough to exceed 2e-3 + 1e-2|o| on rows whose
+// terms cancel), and it is formed as P * 2^-64, a factor the row sum carries
+// too, so that no partial sum of P.V can overflow fp32 for any finite bf16 V.
 #include <math.h>
 #include <stdio.h>
+
+#include <type_traits>
 
 #include <cudaTypedefs.h>
 
@@ -180,9 +182,6 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     uint64_t* empty = full + kStages;
     uint64_t* fold_a = empty + kStages;   // key-split: every consumer is done with the stage
     uint64_t* fold_b = fold_a + 1;        // key-split: the second group's state is in the stage
-    uint64_t* ready = fold_b + 1;         // [kStages] the producer converted the stage's V (no key split)
-    constexpr bool kConvert = kSplit == 1;
-    __shared__ int s_keys[kStages];       // keys of the tile in each stage (rows past are zeroed)
     long long* s_prefix = reinterpret_cast<long long*>(smem + kStages * kStageBytes + kBarrierBytes);
     int* s_len = reinterpret_cast<int*>(s_prefix + kMaxBatchPerLaunch + 1);
     __shared__ long long s_wtot[kMaxRowWarps + 1];
@@ -206,7 +205,6 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         for (int i = 0; i < kStages; ++i) {
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], kSplit * nw);
-            mbar_init(&ready[i], 1);
         }
         mbar_init(fold_a, kSplit * nw);
         mbar_init(fold_b, nw);
@@ -263,11 +261,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         // ------------------------------------------------------ producer
         // The whole warp produces: the next tile is issued once its stage is
         // free (lane pc owns page piece pc; the page ids of 32/pieces tiles
-        // come from one warp-wide load issued a batch ahead).  Without the
-        // key split (three or more row warps, whose tensor throughput paces
-        // them) the producer also turns each landed V tile into fp16 in
-        // place before `ready` releases it; with it, the consumers convert
-        // their V fragments in registers, which adds less to their latency.
+        // come from one warp-wide load issued a batch ahead).
         if (lane == 0) {
             tma_prefetch_desc(&tmap_k);
             tma_prefetch_desc(&tmap_v);
@@ -287,10 +281,10 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
         int pg_cur = batch_pages(0);
         int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
-        int jt = 0, jc = 0;   // next tile to issue, next tile to convert
+        int jt = 0;   // next tile to issue
         uint32_t polls = 0;
         uint64_t t_idle = 0;
-        while (kConvert ? jc < n_tiles : jt < n_tiles) {
+        while (jt < n_tiles) {
             bool progress = false;
             if (jt < n_tiles) {
                 const int st = jt % kStages;
@@ -310,10 +304,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                     int valid = 0;
                     for (int pc = 0; pc < pieces; ++pc)
                         if (ts + pc * kBoxT < L) ++valid;
-                    if (lane == 0) {
-                        s_keys[st] = max(0, min(kTileT, L - ts));
-                        mbar_arrive_expect_tx(&full[st], (uint32_t)valid * piece_bytes * 2u);
-                    }
+                    if (lane == 0) mbar_arrive_expect_tx(&full[st], (uint32_t)valid * piece_bytes * 2u);
                     __syncwarp();
                     if (lane < valid) {
                         const uint32_t kdst = smem_base + st * kStageBytes + (uint32_t)lane * piece_bytes;
@@ -323,37 +314,6 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                         tma_load_5d(vdst, &tmap_v, &full[st], 0, slot, 0, h_cur, page);
                     }
                     ++jt;
-                    progress = true;
-                }
-            }
-            if (kConvert && jc < jt) {
-                const int st = jc % kStages;
-                int landed = 0;
-                if (lane == 0) landed = mbar_test_wait(&full[st], (uint32_t)(jc / kStages) & 1);
-                if (__shfl_sync(0xffffffffu, landed, 0)) {
-                    // V tile rows are [piece][dim half][key]: row r holds key
-                    // (r / (2 kBoxT)) kBoxT + r % kBoxT; rows past L_b are zeroed
-                    const int keys = s_keys[st];
-                    uint4* vt = reinterpret_cast<uint4*>(smem + st * kStageBytes + kTensorTileBytes);
-#pragma unroll 4
-                    for (int i = lane; i < kTensorTileBytes / 16; i += 32) {
-                        const int r = i >> 3;
-                        const int key = (r / (2 * kBoxT)) * kBoxT + r % kBoxT;
-                        uint4 v = make_uint4(0, 0, 0, 0);
-                        if (key < keys) {
-                            v = vt[i];
-                            v.x = bf16x2_to_f16x2(v.x);
-                            v.y = bf16x2_to_f16x2(v.y);
-                            v.z = bf16x2_to_f16x2(v.z);
-                            v.w = bf16x2_to_f16x2(v.w);
-                        }
-                        vt[i] = v;
-                    }
-                    // these generic writes precede the next TMA write into the stage
-                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&ready[st]);
-                    ++jc;
                     progress = true;
                 }
             }
@@ -445,13 +405,13 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     for (int j = 0; j < n_tiles; ++j) {
         const int st = j % kStages;
         const uint32_t use = (uint32_t)(j / kStages);
-        if (!mbar_wait_bounded(kConvert ? &ready[st] : &full[st], use & 1)) {
+        if (!mbar_wait_bounded(&full[st], use & 1)) {
             flag_timeout(p.status);
             break;
         }
         const int L = s_len[cur.b];
         const int ts = cur.t * kTileT;
-        if (!kConvert && ts + kTileT > L) {
+        if (ts + kTileT > L) {
             // keys past L_b (pages not loaded, or slots past the context) may
             // hold any bits: zero their V rows so that P = 0 cannot meet NaN
             const int first = max(0, L - ts);
@@ -528,7 +488,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             const float m_use = m_new == kNegInf ? 0.f : m_new;
             const float alpha = ex2((m_raw[rh] - m_use) * c);
             m_raw[rh] = m_new;
-            const float neg = -m_use * c;
+            const float neg = -m_use * c - kPShift;   // P * 2^-64 (the row sum carries the same factor)
             float rs = 0.f;
 #pragma unroll
             for (int nt = 0; nt < kNT; ++nt) {
@@ -545,30 +505,26 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                 o[dn][2 * rh + 1] *= alpha;
             }
         }
-        // ---- O += P V over this warp's keys: k-steps of 16 keys
+        // ---- O += P V over this warp's keys: k-steps of 16 keys.  P as the sum
+        // of two bf16 terms (hi + lo) against V as stored (bf16)
 #pragma unroll
         for (int kk = 0; kk < kNT / 2; ++kk) {
-            uint32_t a[4];
-            a[0] = pack_f16x2(sc[2 * kk][0], sc[2 * kk][1]);
-            a[1] = pack_f16x2(sc[2 * kk][2], sc[2 * kk][3]);
-            a[2] = pack_f16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-            a[3] = pack_f16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
+            uint32_t ah[4], al[4];
+            split_bf16x2(sc[2 * kk][0], sc[2 * kk][1], ah[0], al[0]);
+            split_bf16x2(sc[2 * kk][2], sc[2 * kk][3], ah[1], al[1]);
+            split_bf16x2(sc[2 * kk + 1][0], sc[2 * kk + 1][1], ah[2], al[2]);
+            split_bf16x2(sc[2 * kk + 1][2], sc[2 * kk + 1][3], ah[3], al[3]);
             const int key = key0 + kk * 16 + (lm & 1) * 8 + lr;
 #pragma unroll
             for (int dp = 0; dp < 8; ++dp) {
                 const int dblk = 2 * dp + (lm >> 1);
                 const int ch = dblk & 7;
                 uint32_t b0, b1, b2, b3;
-                ldsm_x4_trans(vb + key_row(key, dblk >> 3) * 128 + ((ch ^ (key & 7)) << 4), b0,
-                              b1, b2, b3);
-                if (!kConvert) {   // V fragments from bf16 to fp16
-                    b0 = bf16x2_to_f16x2(b0);
-                    b1 = bf16x2_to_f16x2(b1);
-                    b2 = bf16x2_to_f16x2(b2);
-                    b3 = bf16x2_to_f16x2(b3);
-                }
-                mma_f16_16816(o[2 * dp], a, b0, b1);
-                mma_f16_16816(o[2 * dp + 1], a, b2, b3);
+                ldsm_x4_trans(vb + key_row(key, dblk >> 3) * 128 + ((ch ^ (key & 7)) << 4), b0, b1, b2, b3);
+                mma_bf16_16816(o[2 * dp], ah, b0, b1);
+                mma_bf16_16816(o[2 * dp + 1], ah, b2, b3);
+                mma_bf16_16816(o[2 * dp], al, b0, b1);
+                mma_bf16_16816(o[2 * dp + 1], al, b2, b3);
             }
         }
         const bool piece_end = !(j + 1 < n_tiles && cur.t + 1 < cur.T);
@@ -621,7 +577,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         }
         // generic-proxy writes (zeroed rows, the fold's scratch) must be
         // ordered before the next TMA write into this stage
-        if ((!kConvert && ts + kTileT > L) || (kSplit > 1 && piece_end))
+        if (ts + kTileT > L || (kSplit > 1 && piece_end))
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[st]);
@@ -670,10 +626,13 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
             for (int rh = 0; rh < 2; ++rh) {
                 const int row = rh ? row1 : row0;
                 if (row >= p.n_rows || (rh ? grow1 : grow0) >= p.n_rows_all) continue;
+                // the piece's own normalised output and (m, l): the merge takes
+                // a convex combination, which no V value can overflow
+                const float inv = lt[rh] > 0.f ? 1.f / lt[rh] : 0.f;
                 float* dst = p.part_o + (slot * p.n_rows + row) * kD + tq * 2;
 #pragma unroll
                 for (int dn = 0; dn < 16; ++dn)
-                    *reinterpret_cast<float2*>(dst + dn * 8) = make_float2(o[dn][2 * rh], o[dn][2 * rh + 1]);
+                    *reinterpret_cast<float2*>(dst + dn * 8) = make_float2(o[dn][2 * rh] * inv, o[dn][2 * rh + 1] * inv);
                 if (tq == 0)
                     p.part_ml[slot * p.n_rows + row] =
                         make_float2(m_raw[rh] == kNegInf ? kNegInf : m_raw[rh] * c, lt[rh]);
@@ -692,10 +651,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 // Merge of split spans.  Every CTA recomputes the schedule of the main kernel
 // from the context lengths, so it knows which CTAs cut its span (b, h) and in
 // which slots their pieces are; a span with a single piece was written by the
-// main kernel and is skipped.  The pieces are folded with log-sum-exp weights:
-// one warp per query row (a CTA holds 8 rows of one span, so all rows of a
-// span merge at once), lanes across the 128 dims (one coalesced 512-byte
-// read per piece), every piece's loads issued before any is used.
+// main kernel and is skipped.  Each piece left its own normalised output and
+// (m, l); the pieces are combined with log-sum-exp weights normalised to sum
+// to one (a convex combination: no value can overflow): one warp per query
+// row (a CTA holds 8 rows of one span, so all rows of a span merge at once),
+// lanes across the 128 dims (one coalesced 512-byte read per piece), eight
+// pieces' loads issued before any is used.
 // ---------------------------------------------------------------------------
 constexpr int kMergeThreads = 256;
 constexpr int kMergeRows = kMergeThreads / 32;   // query rows per merge CTA
@@ -768,47 +729,58 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     const int head = h / p.n_rb, rbase = (h - head * p.n_rb) * p.n_rows;
     const int row = blockIdx.z * kMergeRows + warp;
     if (row < p.n_rows && rbase + row < p.n_rows_all) {
-        float M = kNegInf, lsum = 0.f;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int q0 = 0; q0 < n_p; q0 += kMergePieces) {
-            float2 ml[kMergePieces];
-            float4 v[kMergePieces];
+        // Every piece left its own normalised output o_q and (m_q, l_q); the
+        // row's output is sum_q w_q o_q with w_q = l_q 2^(m_q - M) / sum_r
+        // l_r 2^(m_r - M), a convex combination.  Pass 1 (lanes across the
+        // pieces): M and the total weight.  Pass 2 (lanes across the 128
+        // dims, one 512-byte read per piece, eight pieces in flight): the sum.
+        float M = kNegInf;
+        for (int q = lane; q < n_p; q += 32) M = fmaxf(M, __ldcg(&p.part_ml[(size_t)s_slots[q] * p.n_rows + row]).x);
 #pragma unroll
-            for (int qq = 0; qq < kMergePieces; ++qq) {
-                const bool ok = q0 + qq < n_p;
-                const size_t sl = (size_t)s_slots[ok ? q0 + qq : 0];
-                ml[qq] = ok ? __ldcg(&p.part_ml[sl * p.n_rows + row]) : make_float2(kNegInf, 0.f);
-                v[qq] = ok ? __ldcg(reinterpret_cast<const float4*>(p.part_o + (sl * p.n_rows + row) * kD +
-                                                                    lane * 4))
-                           : make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+        float lsum = 0.f;
+        if (M != kNegInf)
+            for (int q = lane; q < n_p; q += 32) {
+                const float2 ml = __ldcg(&p.part_ml[(size_t)s_slots[q] * p.n_rows + row]);
+                if (ml.x != kNegInf) lsum = fmaf(ml.y, ex2(ml.x - M), lsum);
             }
-            float Mn = M;
 #pragma unroll
-            for (int qq = 0; qq < kMergePieces; ++qq) Mn = fmaxf(Mn, ml[qq].x);
-            if (Mn == kNegInf) continue;
-            const float sc_old = M == kNegInf ? 0.f : ex2(M - Mn);
-            lsum *= sc_old;
-            acc.x *= sc_old;
-            acc.y *= sc_old;
-            acc.z *= sc_old;
-            acc.w *= sc_old;
-#pragma unroll
-            for (int qq = 0; qq < kMergePieces; ++qq) {
-                const float wgt = ml[qq].x == kNegInf ? 0.f : ex2(ml[qq].x - Mn);
-                lsum = fmaf(wgt, ml[qq].y, lsum);
-                acc.x = fmaf(wgt, v[qq].x, acc.x);
-                acc.y = fmaf(wgt, v[qq].y, acc.y);
-                acc.z = fmaf(wgt, v[qq].z, acc.z);
-                acc.w = fmaf(wgt, v[qq].w, acc.w);
-            }
-            M = Mn;
-        }
+        for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
         const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int q0 = 0; q0 < n_p && inv > 0.f; q0 += 32) {
+            float wq = 0.f;   // the weight of piece q0 + lane
+            if (q0 + lane < n_p) {
+                const float2 ml = __ldcg(&p.part_ml[(size_t)s_slots[q0 + lane] * p.n_rows + row]);
+                wq = ml.x == kNegInf ? 0.f : ml.y * ex2(ml.x - M) * inv;
+            }
+            const int nq = min(32, n_p - q0);
+            for (int qq = 0; qq < nq; qq += kMergePieces) {
+                float4 v[kMergePieces];
+                float wgt[kMergePieces];
+#pragma unroll
+                for (int j = 0; j < kMergePieces; ++j) {
+                    const bool ok = qq + j < nq;
+                    wgt[j] = __shfl_sync(0xffffffffu, wq, (qq + j) & 31);
+                    const size_t sl = (size_t)s_slots[q0 + (ok ? qq + j : 0)];
+                    v[j] = ok ? __ldcg(reinterpret_cast<const float4*>(p.part_o + (sl * p.n_rows + row) * kD + lane * 4))
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (!ok) wgt[j] = 0.f;
+                }
+#pragma unroll
+                for (int j = 0; j < kMergePieces; ++j) {
+                    acc.x = fmaf(wgt[j], v[j].x, acc.x);
+                    acc.y = fmaf(wgt[j], v[j].y, acc.y);
+                    acc.z = fmaf(wgt[j], v[j].z, acc.z);
+                    acc.w = fmaf(wgt[j], v[j].w, acc.w);
+                }
+            }
+        }
         const int i = (rbase + row) / p.G, gi = (rbase + row) % p.G;
         __nv_bfloat16* dst = p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + lane * 4;
         uint2 pk;
-        pk.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-        pk.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+        pk.x = pack_bf16x2(acc.x, acc.y);
+        pk.y = pack_bf16x2(acc.z, acc.w);
         *reinterpret_cast<uint2*>(dst) = pk;
     }
 }

@@ -28,24 +28,26 @@
 //           keys, Q from tensor memory, K a K-major shared-memory operand,
 //           8 steps of 16 dims) as soon as K_t has landed and one of four S
 //           buffers is free -- up to four tiles ahead of the softmax;
-//   warp 12 PV issuer: O += P_t V_t (N = 128 dims, 4 steps of 16 keys) as
-//           soon as the softmax releases P_t, with P read from tensor memory
-//           and V an MN-major operand whose two dim halves lie one leading
-//           offset apart;
+//   warp 12 PV issuer: O += P_t V_t (N = 128 dims, 8 steps of 16 keys: 4
+//           with P_hi, 4 with P_lo) as soon as the softmax releases P_t and
+//           V_t has landed, with P read from tensor memory and V, as stored
+//           in bf16, an MN-major operand whose two dim halves lie one leading
+//           offset apart; in a span's last tile it first zeroes the V rows
+//           past L_b (their slots may hold any bits);
 //   warp 2  tensor-memory allocation (512 columns: four S/P buffers of 64,
 //           O in 128, two query buffers of 64);
-//   warps 2-3  every V tile from bf16 into fp16, in place;
 //   warps 4-11 softmax and epilogue, two warps per query row (one row per
 //           lane; warps 4+q and 8+q own tensor-memory lanes 32q..32q+31 and
 //           take keys 0..31 and 32..63 of every tile): mask, running max
 //           (the two halves' maxima swapped through shared memory), exp2,
-//           row sum, P written back over S as fp16 (warps 2-3 turn each V
-//           tile into fp16, so PV multiplies fp16 by fp16: bf16 P alone can
-//           exceed the output tolerance on rows whose terms cancel); O is
-//           rescaled in tensor memory only when the running max grows by
-//           more than 2^8 (the stale max keeps every P below 256); at a span
-//           piece's end the row is normalised and written (bf16) or left as
-//           a partial, 64 dims by each warp of the pair.
+//           row sum, P written back over S as two bf16 terms, hi and lo
+//           (bf16 P alone can exceed the output tolerance on rows whose terms
+//           cancel), formed as P * 2^-64 so that no partial sum of P.V
+//           overflows fp32 for any finite bf16 V; O is rescaled in tensor
+//           memory only when the running max grows by more than 2^8 (the
+//           stale max keeps every P below 256); at a span piece's end the row
+//           is normalised and written (bf16) or left as a partial, 64 dims by
+//           each warp of the pair.
 // Every mbarrier wait is bounded; a wait that gives up sets the status word
 // and a shared flag that ends every warp's loop.
 
@@ -84,7 +86,7 @@ __host__ __device__ constexpr int tc_smem_bytes(int rows) {
     return 2 * tc_q_half_bytes(rows) + (tc_k_stages(rows) + tc_v_stages(rows)) * kTensorTileBytes + kTcFixedSmem;
 }
 static_assert(tc_k_stages(kTcRows) >= 2 && tc_v_stages(kTcRows) >= 4, "rings too shallow for 128 query rows");
-static_assert((2 * kTcMaxK + 3 * kTcMaxV + 5 + 3 * 4 + 1 + 4) * 8 <= 512, "barrier block too small");
+static_assert((2 * kTcMaxK + 2 * kTcMaxV + 5 + 3 * 4 + 1 + 4) * 8 <= kTcBarBytes, "barrier block too small");
 constexpr float kTcRescale = 8.f;                  // log2 growth of the max that forces a rescale of O
 
 __device__ __forceinline__ uint64_t tc_sw128_desc(uint32_t addr) {
@@ -102,7 +104,7 @@ __device__ __forceinline__ uint64_t tc_mn_desc(uint32_t addr) {
 }
 
 // kind::f16 instruction descriptor: fp32 D, M = 128, N = n, A and B both
-// bf16 (QK) or both fp16 (PV); b_mn: B is MN-major (its N index contiguous)
+// bf16 (f16 = false) or both fp16; b_mn: B is MN-major (its N index contiguous)
 __host__ __device__ constexpr uint32_t tc_idesc(int n, bool b_mn, bool f16) {
     return (1u << 4) | (f16 ? 0u : (1u << 7) | (1u << 10)) | (b_mn ? (1u << 16) : 0u) | ((uint32_t)(n >> 3) << 17) |
            ((uint32_t)(kTcRows >> 4) << 24);
@@ -215,8 +217,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     uint64_t* kempty = kfull + kTcMaxK;                     // [SK] K tile consumed (QK done)
     uint64_t* vfull = kempty + kTcMaxK;                     // [SV] V tile landed
     uint64_t* vempty = vfull + kTcMaxV;                     // [SV] V tile consumed (PV done)
-    uint64_t* ready = vempty + kTcMaxV;                     // [SV] the V tile is in fp16
-    uint64_t* q_full = ready + kTcMaxV;                     // a span's query rows landed in shared memory
+    uint64_t* q_full = vempty + kTcMaxV;                    // a span's query rows landed in shared memory
     uint64_t* q_cp = q_full + 1;                            // ... and were copied into tensor memory
     uint64_t* q_free = q_cp + 1;                            // [2] last QK of a span done (tensor-memory buffer)
     uint64_t* s_full = q_free + 2;                          // [kTcSBuf] S_t in tensor memory
@@ -260,7 +261,6 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         for (int i = 0; i < SV; ++i) {
             mbar_init(&vfull[i], 1);
             mbar_init(&vempty[i], 1);
-            mbar_init(&ready[i], 2);
         }
         mbar_init(q_full, 1);
         mbar_init(q_cp, 1);
@@ -400,37 +400,6 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         if (lane == 0)
             for (int j = jt > S ? jt - S : 0; j < jt; ++j)
                 if (!mbar_wait_bounded(&fullb[j % S], (uint32_t)(j / S) & 1)) atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-    } else if ((warp == 2 || warp == 3) && n_tiles > 0) {
-        // ------------------------------------------------------- V to fp16
-        // Each landed V tile is turned from bf16 into fp16 in place by these
-        // two warps (16-byte chunk i of the tile, laid out [dim half][64
-        // keys][128 B], holds key (i / 8) % 64; rows past L_b are zeroed),
-        // then released through `ready`, which the softmax checks before it
-        // hands P_t to the MMA warp.
-        const int ct = (warp - 2) * 32 + lane;
-        for (int jc = 0; jc < n_tiles; ++jc) {
-            const int st = jc % SV;
-            if (!tc_wait(&vfull[st], (uint32_t)(jc / SV) & 1, &s_dead, p.status)) break;
-            const int keys = s_keys[st];
-            uint4* vt = reinterpret_cast<uint4*>(sv + st * kTensorTileBytes);
-#pragma unroll 4
-            for (int i = ct; i < kTensorTileBytes / 16; i += 64) {
-                uint4 v = make_uint4(0, 0, 0, 0);
-                if (((i >> 3) & (kTileT - 1)) < keys) {
-                    v = vt[i];
-                    v.x = bf16x2_to_f16x2(v.x);
-                    v.y = bf16x2_to_f16x2(v.y);
-                    v.z = bf16x2_to_f16x2(v.z);
-                    v.w = bf16x2_to_f16x2(v.w);
-                }
-                vt[i] = v;
-            }
-            // generic writes the tensor core reads next (and the next TMA
-            // write into the stage follows them)
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&ready[st]);
-        }
     } else if ((warp == 1 || warp == kTcPvWarp) && n_tiles > 0) {
         // ---------------------------------------------------------- MMA
         // Two issuing warps, each running its loop with all lanes (the waits)
@@ -449,7 +418,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // offsets (addresses stay below 256 KB: the 14-bit start field cannot
         // carry).
         const bool qk_warp = warp == 1;
-        constexpr uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, true);
+        // QK and PV both bf16: P enters as two bf16 terms (hi + lo) against V as stored
+        constexpr uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, false);
         const uint64_t dq0 = tc_sw128_desc(smem_u32(sq));
         const uint64_t qhalf16 = (uint64_t)qh >> 4;
         const uint64_t dk0 = tc_sw128_desc(smem_u32(sk)), dv0 = tc_mn_desc(smem_u32(sv));
@@ -505,6 +475,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             } else {
                 const int st = t % SV;
                 if (!wait_all(&p_full[sb], (uint32_t)(t / kTcSBuf) & 1)) break;
+                // V_t has landed (the stage's next landing needs this PV first)
+                if (!wait_all(&vfull[st], (uint32_t)(t / SV) & 1)) break;
                 const bool first = t == 0 || cur.t == 0;
                 advance(cur, s_len, nb, p.n_vh);
                 if (first) {
@@ -512,14 +484,31 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                     if (pv_piece > 0 && !wait_all(o_free, (uint32_t)(pv_piece - 1) & 1)) break;
                     ++pv_piece;
                 }
+                // a span's last tile: the slots past L_b may hold any bits (NaN
+                // included) and P is 0 there, so their V rows are zeroed (chunk i
+                // of the tile holds key (i / 8) % 64)
+                const int keys = s_keys[st];
+                if (keys < kTileT) {
+                    uint4* vt = reinterpret_cast<uint4*>(sv + st * kTensorTileBytes);
+                    for (int i = lane; i < kTensorTileBytes / 16; i += 32)
+                        if (((i >> 3) & (kTileT - 1)) >= keys) vt[i] = make_uint4(0, 0, 0, 0);
+                    // generic writes the tensor core reads next
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    __syncwarp();
+                }
                 tc_fence_after();
-                // O += P_t V_t, 4 steps of 16 keys, both dim halves per step
+                // O += P_t V_t: 4 steps of 16 keys with P_hi (columns 0..31 of
+                // the buffer), 4 with P_lo (columns 32..63), both dim halves per step
                 const uint64_t dv = dv0 + (uint64_t)((st * kTensorTileBytes) >> 4);
                 if (elect_one()) {
 #pragma unroll
                     for (int kk = 0; kk < kTileT / 16; ++kk)
                         tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + kk * 8, dv + (uint64_t)(kk * ((16 * 128) >> 4)),
                                   id_o, (first && kk == 0) ? 0u : 1u);
+#pragma unroll
+                    for (int kk = 0; kk < kTileT / 16; ++kk)
+                        tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + 32 + kk * 8,
+                                  dv + (uint64_t)(kk * ((16 * 128) >> 4)), id_o, 1u);
                     tc_commit(&o_ready[sb]);
                     tc_commit(&vempty[st]);
                 }
@@ -632,14 +621,16 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 alpha = m_run == kNegInf ? 0.f : ex2((m_run - mt) * c);
                 m_run = mt;
             }
-            const float neg = m_run == kNegInf ? 0.f : -m_run * c;
+            // ---- P = 2^((s - m) c - 64) (the row sum carries the same 2^-64),
+            // as the sum of two bf16 terms
+            const float neg = m_run == kNegInf ? 0.f : -m_run * c - kPShift;
             float r4[4] = {0.f, 0.f, 0.f, 0.f};
-            uint32_t pk[16];
+            uint32_t ph[16], pl[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
                 const float p0 = ex2(fmaf(s[2 * e], c, neg)), p1 = ex2(fmaf(s[2 * e + 1], c, neg));
                 r4[e & 3] += p0 + p1;
-                pk[e] = pack_f16x2(p0, p1);
+                split_bf16x2(p0, p1, ph[e], pl[e]);
             }
             l_half = l_half * alpha + ((r4[0] + r4[1]) + (r4[2] + r4[3]));
             // ---- a rescale of O (this warp's 64 dims) waits for PV_{t-1}; the
@@ -662,17 +653,14 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                     tc_st32(t_row + kTcOCol + c0, r);
                 }
             }
-            // P as fp16 pairs: keys kb..kb+31 are columns kb/2 .. kb/2+15 of the
-            // buffer (the partner's S columns there were loaded before the swap)
-            tc_st16(t_row + sb * 64 + half * 16, pk);
+            // P as bf16 pairs: keys kb..kb+31 are columns kb/2 .. kb/2+15 of the
+            // buffer (hi) and 32 + kb/2 .. (lo); the S columns there were loaded
+            // by both warps of the pair before the swap
+            tc_st16(t_row + sb * 64 + half * 16, ph);
+            tc_st16(t_row + sb * 64 + 32 + half * 16, pl);
             tc_wait_st();
             tc_fence_before();
-            // P_t goes to the MMA warp once the tile's V is in fp16 too (the
-            // PV reads both).  The next phase of `ready` needs the stage
-            // back, i.e. this PV, so the parity names one phase.
-            const bool v_ok = lane != 0 || half != 0 || tc_wait(&ready[t % SV], (uint32_t)(t / SV) & 1, &s_dead,
-                                                                p.status);
-            if (!__all_sync(0xffffffffu, v_ok)) break;
+            __syncwarp();
             if (lane == 0) mbar_arrive(&p_full[sb]);
 
             if (!piece_end) {
@@ -693,6 +681,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             const bool complete = seg_t0 == 0 && cur.t + 1 == cur.T;
             const size_t slot = 2 * (size_t)cta + (first_seg ? 0 : 1);
             const bool live_row = row < p.n_rows_all;
+            // normalised output; a partial is the piece's own normalised output
+            // (the merge takes a convex combination)
             const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
 #pragma unroll 1
             for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
@@ -716,7 +706,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
                         *reinterpret_cast<float4*>(dst + 4 * q) =
-                            make_float4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                            make_float4(o[4 * q] * inv, o[4 * q + 1] * inv, o[4 * q + 2] * inv, o[4 * q + 3] * inv);
                 }
             }
             if (live_row && !complete && half == 0)

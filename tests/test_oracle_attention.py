@@ -263,3 +263,25 @@ def test_bf16_widening_is_exact():
     out = oracle.verify_attention(q, kp, vp, np.zeros((1, 1), np.int32), np.array([1], np.int32), 0)
     assert out[0, 0, 0, :3].tolist() == [1.0, -2.0, 0.125]
     assert math.isclose(out[0, 0, 0, 3], 0.0)
+
+
+def test_large_values_match_torch_sdpa():
+    """V entries across bf16's whole range (up to ~3.39e38, far beyond fp16's
+    65504) are exact in fp64: the oracle still equals torch's float64 SDPA."""
+    rng = np.random.default_rng(77)
+    B, k, Hq, Hkv, D, ps = 2, 3, 4, 2, 8, 4
+    c = make_case(rng, B, k, Hq, Hkv, D, ps, [29, 38])
+    big = [3.3e38, -3.0e38, 1.0e5, -65536.0, 65280.0, 2.0e20]
+    for b in range(B):
+        L = int(c["lens"][b])
+        for h in range(Hkv):
+            for val, d in zip(big, rng.choice(D, len(big), replace=False)):
+                key = int(rng.integers(0, L))
+                bits, exact = bf16_round(np.array([val]))
+                page, slot = int(c["table"][b, key // ps]), key % ps
+                c["vpool"][page, h, slot, d] = bits[0]
+                c["v_dense"][b, h, key, d] = exact[0]
+    got = run_oracle(c)
+    ref = sdpa_masked(c, Hq, Hkv)
+    assert np.isfinite(got).all() and np.abs(ref).max() > 1e37
+    np.testing.assert_allclose(got, ref, rtol=1e-12, atol=1e-13 * np.abs(ref).max())
