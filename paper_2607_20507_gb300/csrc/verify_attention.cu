@@ -1028,10 +1028,8 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
         CUtensorMap tq;
         st = encode_q_map(&tq, q, d, pl.rows);
         if (st != CS_OK) return st;
-        st = encode_pool_map(&tk, k_pages, d, box_t, 1);
-        if (st != CS_OK) return st;
-        st = encode_pool_map(&tv, v_pages, d, box_t, 1);
-        if (st != CS_OK) return st;
+        // one box per page piece with both dim halves, as for the other form
+
         using TcKern = void (*)(const CUtensorMap, const CUtensorMap, const CUtensorMap, const AttnParams);
         static const TcKern tc_kerns[2][3] = {
             {verify_attention_tc_kernel<false, 16>, verify_attention_tc_kernel<false, 32>,

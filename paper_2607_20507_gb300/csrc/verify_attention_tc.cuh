@@ -95,11 +95,11 @@ __device__ __forceinline__ uint64_t tc_sw128_desc(uint32_t addr) {
            (2ull << 61);
 }
 
-// MN-major, 128-byte swizzle, for the V tile [dim half][64 keys][128 B]:
-// 8-key groups 1024 bytes apart (stride), the two 64-dim halves one half
-// tile apart (leading offset)
-__device__ __forceinline__ uint64_t tc_mn_desc(uint32_t addr) {
-    return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)((kTileT * 128) >> 4) << 16) |
+// MN-major, 128-byte swizzle, for a V page piece [dim half][keys][128 B]:
+// 8-key groups 1024 bytes apart (stride), the two 64-dim halves
+// `half_bytes` apart (leading offset)
+__device__ __forceinline__ uint64_t tc_mn_desc(uint32_t addr, uint32_t half_bytes) {
+    return (uint64_t)((addr >> 4) & 0x3FFF) | ((uint64_t)(half_bytes >> 4) << 16) |
            ((uint64_t)(1024 >> 4) << 32) | (1ull << 46) | (2ull << 61);
 }
 
@@ -197,7 +197,6 @@ __device__ __forceinline__ bool tc_wait(uint64_t* bar, uint32_t parity, volatile
     return false;
 }
 
-constexpr int kTcHalfBytes = kTileT * 128;       // one dim half of a 64-key K or V tile
 
 template <bool kTree, int kBoxT>
 __global__ void __launch_bounds__(kTcThreads, 1)
@@ -205,6 +204,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                            const __grid_constant__ CUtensorMap tmap_q, const AttnParams p) {
     constexpr int kPieces = kTileT / kBoxT;
     constexpr uint32_t kPieceBytes = (uint32_t)kBoxT * 256u;   // bytes of one page piece of K (or of V)
+    constexpr uint32_t kPieceHalf = (uint32_t)kBoxT * 128u;    // one dim half of a page piece
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int SK = p.tc_stages, SV = p.tc_vstages;          // K and V ring depths
@@ -389,11 +389,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             }
             __syncwarp();
             if (lane < valid) {
-                const uint32_t dst = smem_u32(ring + st * kTensorTileBytes) + (uint32_t)lane * (kBoxT * 128);
+                // one box per page piece, both dim halves: [half][kBoxT keys][128 B]
+                const uint32_t dst = smem_u32(ring + st * kTensorTileBytes) + (uint32_t)lane * kPieceBytes;
                 const int slot = (ts + lane * kBoxT) % p.ps;
-#pragma unroll
-                for (int hh = 0; hh < 2; ++hh)
-                    tma_load_5d(dst + hh * kTcHalfBytes, tmap, &fullb[st], 0, slot, hh, h_cur, page);
+                tma_load_5d(dst, tmap, &fullb[st], 0, slot, 0, h_cur, page);
             }
         }
         // no copy in flight at exit: every issued tile has landed
@@ -419,10 +418,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // carry).
         const bool qk_warp = warp == 1;
         // QK and PV both bf16: P enters as two bf16 terms (hi + lo) against V as stored
-        constexpr uint32_t id_s = tc_idesc(kTileT, false, false), id_o = tc_idesc(kD, true, false);
+        constexpr uint32_t id_s = tc_idesc(kBoxT, false, false), id_o = tc_idesc(kD, true, false);
         const uint64_t dq0 = tc_sw128_desc(smem_u32(sq));
         const uint64_t qhalf16 = (uint64_t)qh >> 4;
-        const uint64_t dk0 = tc_sw128_desc(smem_u32(sk)), dv0 = tc_mn_desc(smem_u32(sv));
+        const uint64_t dk0 = tc_sw128_desc(smem_u32(sk)), dv0 = tc_mn_desc(smem_u32(sv), kPieceHalf);
         int span = -1, pv_piece = 0;
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);   // the PV warp's own view of the pieces
         uint64_t* last_bar = nullptr;   // the warp's latest commit: completes after all its MMAs
@@ -460,10 +459,16 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                             tc_cp_128x256b(tq + ks * 8, dq0 + (ks >> 2) * qhalf16 + (uint64_t)((ks & 3) * 2));
                         tc_commit(q_cp);   // the producer may refill the query buffer
                     }
+                    // per page piece (N = kBoxT keys, S columns pc*kBoxT..), 8
+                    // steps of 16 dims
 #pragma unroll
-                    for (int ks = 0; ks < kD / 16; ++ks) {
-                        const uint64_t ko = (uint64_t)((((ks >> 2) * kTcHalfBytes) >> 4) + (ks & 3) * 2);
-                        tc_mma_ts(tmem + sb * 64, tq + ks * 8, dk + ko, id_s, ks > 0 ? 1u : 0u);
+                    for (int pc = 0; pc < kPieces; ++pc) {
+#pragma unroll
+                        for (int ks = 0; ks < kD / 16; ++ks) {
+                            const uint64_t ko =
+                                (uint64_t)(((pc * kPieceBytes + (ks >> 2) * kPieceHalf) >> 4) + (ks & 3) * 2);
+                            tc_mma_ts(tmem + sb * 64 + pc * kBoxT, tq + ks * 8, dk + ko, id_s, ks > 0 ? 1u : 0u);
+                        }
                     }
                     tc_commit(&s_full[sb]);
                     tc_commit(&kempty[st]);
@@ -485,13 +490,16 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                     ++pv_piece;
                 }
                 // a span's last tile: the slots past L_b may hold any bits (NaN
-                // included) and P is 0 there, so their V rows are zeroed (chunk i
-                // of the tile holds key (i / 8) % 64)
+                // included) and P is 0 there, so their V rows are zeroed (128-byte
+                // row r of the tile, [piece][half][kBoxT keys], holds key
+                // (r / (2 kBoxT)) kBoxT + r % kBoxT)
                 const int keys = s_keys[st];
                 if (keys < kTileT) {
                     uint4* vt = reinterpret_cast<uint4*>(sv + st * kTensorTileBytes);
-                    for (int i = lane; i < kTensorTileBytes / 16; i += 32)
-                        if (((i >> 3) & (kTileT - 1)) >= keys) vt[i] = make_uint4(0, 0, 0, 0);
+                    for (int i = lane; i < kTensorTileBytes / 16; i += 32) {
+                        const int r = i >> 3;
+                        if ((r / (2 * kBoxT)) * kBoxT + r % kBoxT >= keys) vt[i] = make_uint4(0, 0, 0, 0);
+                    }
                     // generic writes the tensor core reads next
                     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                     __syncwarp();
@@ -501,14 +509,17 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 // the buffer), 4 with P_lo (columns 32..63), both dim halves per step
                 const uint64_t dv = dv0 + (uint64_t)((st * kTensorTileBytes) >> 4);
                 if (elect_one()) {
+                    // keys 16kk..16kk+15: rows (16kk) % kBoxT.. of page piece 16kk / kBoxT
 #pragma unroll
-                    for (int kk = 0; kk < kTileT / 16; ++kk)
-                        tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + kk * 8, dv + (uint64_t)(kk * ((16 * 128) >> 4)),
-                                  id_o, (first && kk == 0) ? 0u : 1u);
+                    for (int kk = 0; kk < kTileT / 16; ++kk) {
+                        const uint64_t vk = dv + (uint64_t)((((16 * kk) / kBoxT) * kPieceBytes + ((16 * kk) % kBoxT) * 128) >> 4);
+                        tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + kk * 8, vk, id_o, (first && kk == 0) ? 0u : 1u);
+                    }
 #pragma unroll
-                    for (int kk = 0; kk < kTileT / 16; ++kk)
-                        tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + 32 + kk * 8,
-                                  dv + (uint64_t)(kk * ((16 * 128) >> 4)), id_o, 1u);
+                    for (int kk = 0; kk < kTileT / 16; ++kk) {
+                        const uint64_t vk = dv + (uint64_t)((((16 * kk) / kBoxT) * kPieceBytes + ((16 * kk) % kBoxT) * 128) >> 4);
+                        tc_mma_ts(tmem + kTcOCol, tmem + sb * 64 + 32 + kk * 8, vk, id_o, 1u);
+                    }
                     tc_commit(&o_ready[sb]);
                     tc_commit(&vempty[st]);
                 }
