@@ -6,36 +6,42 @@
 // the other form run out of tensor throughput (with fewer rows the M = 128
 // padding of every MMA costs more than it saves).  Same persistent schedule
 // (equal contiguous tile ranges, spans, two partial slots per CTA, merge
-// kernel), one CTA per SM, warp roles:
+// kernel), one CTA per SM, twelve warps (each SMSP, warp % 4, runs one role
+// warp and two softmax warps):
 //   warp 0  K producer: the span's query rows (one 4-D box per dim half into
 //           one buffer, refilled once the previous span's rows have been
 //           copied into tensor memory; each half as many 128-byte rows as
 //           the span has: the MMA's 128-row window runs on into whatever
 //           follows, which only feeds padded rows) and the K tiles of the
-//           range through the K ring, one box per page piece and dim half, so
-//           a tile lands as [dim half][64 keys][128 B], 128-byte swizzle;
+//           range through the K ring, one box per page piece with both dim
+//           halves (contiguous 256-byte rows: a per-half box of 128-byte rows
+//           kept the SM's copy engine saturated at two thirds of the
+//           bandwidth), so a tile lands as [piece][dim half][keys][128 B],
+//           128-byte swizzle;
 //           beside each stage it leaves whether the tile opens or closes a
 //           piece;
-//   warp 13 V producer: the V tiles through the V ring, the same way.  The
+//   warp 1  V producer: the V tiles through the V ring, the same way.  The
 //           two rings share the 16 KB stages that shared memory holds beside
 //           the query buffer (a third for K, which is released as soon as
 //           its QK is done; the rest for V, held until its PV is done), so
 //           each side runs ahead as far as its own consumer allows;
-//   warp 1  QK issuer (the whole warp waits, one elected lane issues): at
+//   warp 2  QK issuer (the whole warp waits, one elected lane issues): at
 //           a piece's start the query rows from shared into tensor memory
 //           (tcgen05.cp, one buffer per span parity), then per tile
-//           S_t = Q K_t^T into tensor memory (M = 128 padded rows, N = 64
-//           keys, Q from tensor memory, K a K-major shared-memory operand,
-//           8 steps of 16 dims) as soon as K_t has landed and one of four S
-//           buffers is free -- up to four tiles ahead of the softmax;
-//   warp 12 PV issuer: O += P_t V_t (N = 128 dims, 8 steps of 16 keys: 4
+//           S_t = Q K_t^T into tensor memory (M = 128 padded rows, per page
+//           piece N = its keys, Q from tensor memory, K a K-major
+//           shared-memory operand, 8 steps of 16 dims) as soon as K_t has
+//           landed and one of four S buffers is free -- up to four tiles
+//           ahead of the softmax.  It also allocates the tensor memory (512
+//           columns: four S/P buffers of 64, O in 128, two query buffers of
+//           64);
+//   warp 3  PV issuer: O += P_t V_t (N = 128 dims, 8 steps of 16 keys: 4
 //           with P_hi, 4 with P_lo) as soon as the softmax releases P_t and
 //           V_t has landed, with P read from tensor memory and V, as stored
-//           in bf16, an MN-major operand whose two dim halves lie one leading
-//           offset apart; in a span's last tile it first zeroes the V rows
-//           past L_b (their slots may hold any bits);
-//   warp 2  tensor-memory allocation (512 columns: four S/P buffers of 64,
-//           O in 128, two query buffers of 64);
+//           in bf16, an MN-major operand (per 16 keys, the rows of one page
+//           piece) whose two dim halves lie one piece half apart; in a span's
+//           last tile it first zeroes the V rows past L_b (their slots may
+//           hold any bits);
 //   warps 4-11 softmax and epilogue, two warps per query row (one row per
 //           lane; warps 4+q and 8+q own tensor-memory lanes 32q..32q+31 and
 //           take keys 0..31 and 32..63 of every tile): mask, running max
@@ -53,9 +59,10 @@
 
 constexpr int kTcMaxK = 6;                         // K ring depth, at most
 constexpr int kTcMaxV = 10;                        // V ring depth, at most
-constexpr int kTcThreads = 448;                    // 14 warps
-constexpr int kTcPvWarp = 12;                      // the PV issuer
-constexpr int kTcVWarp = 13;                       // the V producer
+constexpr int kTcThreads = 384;                    // 12 warps: 4 roles, 8 softmax (three warps per SMSP)
+constexpr int kTcVWarp = 1;                        // the V producer
+constexpr int kTcQkWarp = 2;                       // the QK issuer (and tensor-memory allocator)
+constexpr int kTcPvWarp = 3;                       // the PV issuer
 constexpr int kTcRows = 128;                       // MMA M: query rows, padded
 constexpr int kTcMinRows = 48;                     // fewer query rows take the mma.sync form
 constexpr int kTcSBuf = 4;                         // S/P buffers in tensor memory
@@ -245,7 +252,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         for (long long i = (long long)blockIdx.x * 32 + lane; i < lines; i += (long long)gridDim.x * 32)
             asm volatile("prefetch.global.L2 [%0];" ::"l"(tab + i * 128));
     }
-    if (warp == 2) {
+    if (warp == kTcQkWarp) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s_tmem)),
                      "n"(kTcTmemCols)
                      : "memory");
@@ -399,7 +406,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         if (lane == 0)
             for (int j = jt > S ? jt - S : 0; j < jt; ++j)
                 if (!mbar_wait_bounded(&fullb[j % S], (uint32_t)(j / S) & 1)) atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-    } else if ((warp == 1 || warp == kTcPvWarp) && n_tiles > 0) {
+    } else if ((warp == kTcQkWarp || warp == kTcPvWarp) && n_tiles > 0) {
         // ---------------------------------------------------------- MMA
         // Two issuing warps, each running its loop with all lanes (the waits)
         // and one elected lane issuing (a lone lane beside 31 parked at the
@@ -416,7 +423,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // yet), so a parity wait is exact.  Descriptors advance by constant
         // offsets (addresses stay below 256 KB: the 14-bit start field cannot
         // carry).
-        const bool qk_warp = warp == 1;
+        const bool qk_warp = warp == kTcQkWarp;
         // QK and PV both bf16: P enters as two bf16 terms (hi + lo) against V as stored
         constexpr uint32_t id_s = tc_idesc(kBoxT, false, false), id_o = tc_idesc(kD, true, false);
         const uint64_t dq0 = tc_sw128_desc(smem_u32(sq));
@@ -736,6 +743,6 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 2)
+    if (warp == kTcQkWarp)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "n"(kTcTmemCols) : "memory");
 }
