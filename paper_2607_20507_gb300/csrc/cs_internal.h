@@ -29,7 +29,7 @@ struct AttnPlan {
     int split;        // consumer groups sharing each tile's keys (1 or 2)
     bool tc;          // the tcgen05 kernel (33..128 rows, one row block)
     int grid;         // persistent CTAs (resident capacity of the device)
-    size_t off_part_o, off_part_ml, bytes;   // workspace layout (status word at 0)
+    size_t off_part_o, off_part_ml, off_part_span, bytes;   // workspace layout (status word at 0)
 };
 AttnPlan plan_verify_attention(const cs_attn_dims& d, int n_draft, int sm_count);
 AttnPlan plan_tree_attention(const cs_attn_dims& d, int n_nodes, int sm_count);

@@ -80,6 +80,7 @@ struct AttnParams {
     const int32_t* parents;      // [B, R] tree parents (tree kernel only)
     float* part_o;               // [2 * grid, n_rows, D]
     float2* part_ml;             // [2 * grid, n_rows]  (m in log2 units, l)
+    int* part_span;              // [2 * grid] span (b * n_vh + h) of each partial slot, -1 if unused
     int* status;
     int Hq, Hkv, G, R, n_rows, ps, box_t, max_pages, row_warps;
     int n_rb;                    // row blocks per KV head (n_rows rows each)
@@ -251,6 +252,12 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
     const long long g_need = (W + kMinTilesPerCta - 1) / kMinTilesPerCta;
     const int Gc = (int)(g_need < (long long)gridDim.x ? (g_need > 0 ? g_need : 1) : gridDim.x);
     const int cta = blockIdx.x;
+    // this CTA's two partial slots start unused (thread 0 -- row warp 0,
+    // lane 0 -- is also the one that records a partial's span below)
+    if (threadIdx.x == 0) {
+        p.part_span[2 * cta] = -1;
+        p.part_span[2 * cta + 1] = -1;
+    }
     if (cta >= Gc) return;
     const long long f0 = (long long)cta * W / Gc, f1 = (long long)(cta + 1) * W / Gc;
     if (f0 >= f1) return;
@@ -637,6 +644,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
                     p.part_ml[slot * p.n_rows + row] =
                         make_float2(m_raw[rh] == kNegInf ? kNegInf : m_raw[rh] * c, lt[rh]);
             }
+            if (threadIdx.x == 0) p.part_span[slot] = cur.b * p.n_vh + cur.h;
         }
         if (j + 1 < n_tiles) {
             advance(cur, s_len, nb, p.n_vh);
@@ -648,31 +656,96 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 }
 
 // ---------------------------------------------------------------------------
-// Merge of split spans.  Every CTA recomputes the schedule of the main kernel
-// from the context lengths, so it knows which CTAs cut its span (b, h) and in
-// which slots their pieces are; a span with a single piece was written by the
-// main kernel and is skipped.  Each piece left its own normalised output and
-// (m, l); the pieces are combined with log-sum-exp weights normalised to sum
-// to one (a convex combination: no value can overflow): one warp per query
-// row (a CTA holds 8 rows of one span, so all rows of a span merge at once),
-// lanes across the 128 dims (one coalesced 512-byte read per piece), eight
-// pieces' loads issued before any is used.
+// Merge of split spans.  Each piece of a cut span left its own normalised
+// output o_q and (m_q, l_q); the span's output is sum_q w_q o_q with
+// w_q = l_q 2^(m_q - M) / sum_r l_r 2^(m_r - M), a convex combination (no
+// value can overflow).  One warp per query row: pass 1 (lanes across the
+// pieces) finds M and the total weight, pass 2 (lanes across the 128 dims,
+// one coalesced 512-byte read per piece, eight pieces in flight) the sum.
+// A CTA holds 8 rows of one span.  Two ways to find a span's pieces, the
+// launch taking the one with the smaller grid:
+//  * per span: every CTA recomputes the main kernel's schedule from the
+//    context lengths (cheap for few requests) and finds the CTAs that cut
+//    its span; a span with a single piece was written whole and is skipped;
+//  * per partial slot: the main kernel records the span of each partial slot
+//    (-1 when unused).  In slot order (CTA c's first piece 2c, its last 2c+1)
+//    a cut span's pieces are consecutive, unused slots aside, so the CTA of
+//    a span's first slot gathers them from a window of the list read into
+//    shared memory.  The grid no longer grows with the number of spans.
 // ---------------------------------------------------------------------------
 constexpr int kMergeThreads = 256;
 constexpr int kMergeRows = kMergeThreads / 32;   // query rows per merge CTA
 constexpr int kMergePieces = 8;   // pieces in flight per row
+constexpr int kMergeBack = 32, kMergeAhead = 96;   // slot-list window around a CTA's own slot
 
+// the convex combination of one row's pieces (slots[0..n_p)), by one warp
+__device__ __forceinline__ void merge_row(const AttnParams& p, const int* slots, int n_p, int bl, int h, int row,
+                                          int lane) {
+    const int bg = p.b_base + bl;
+    const int head = h / p.n_rb, rbase = (h - head * p.n_rb) * p.n_rows;
+    if (row >= p.n_rows || rbase + row >= p.n_rows_all) return;
+    float M = kNegInf;
+    for (int q = lane; q < n_p; q += 32) M = fmaxf(M, __ldcg(&p.part_ml[(size_t)slots[q] * p.n_rows + row]).x);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    float lsum = 0.f;
+    if (M != kNegInf)
+        for (int q = lane; q < n_p; q += 32) {
+            const float2 ml = __ldcg(&p.part_ml[(size_t)slots[q] * p.n_rows + row]);
+            if (ml.x != kNegInf) lsum = fmaf(ml.y, ex2(ml.x - M), lsum);
+        }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+    const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int q0 = 0; q0 < n_p && inv > 0.f; q0 += 32) {
+        float wq = 0.f;   // the weight of piece q0 + lane
+        if (q0 + lane < n_p) {
+            const float2 ml = __ldcg(&p.part_ml[(size_t)slots[q0 + lane] * p.n_rows + row]);
+            wq = ml.x == kNegInf ? 0.f : ml.y * ex2(ml.x - M) * inv;
+        }
+        const int nq = min(32, n_p - q0);
+        for (int qq = 0; qq < nq; qq += kMergePieces) {
+            float4 v[kMergePieces];
+            float wgt[kMergePieces];
+#pragma unroll
+            for (int j = 0; j < kMergePieces; ++j) {
+                const bool ok = qq + j < nq;
+                wgt[j] = __shfl_sync(0xffffffffu, wq, (qq + j) & 31);
+                const size_t sl = (size_t)slots[q0 + (ok ? qq + j : 0)];
+                v[j] = ok ? __ldcg(reinterpret_cast<const float4*>(p.part_o + (sl * p.n_rows + row) * kD + lane * 4))
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+                if (!ok) wgt[j] = 0.f;
+            }
+#pragma unroll
+            for (int j = 0; j < kMergePieces; ++j) {
+                acc.x = fmaf(wgt[j], v[j].x, acc.x);
+                acc.y = fmaf(wgt[j], v[j].y, acc.y);
+                acc.z = fmaf(wgt[j], v[j].z, acc.z);
+                acc.w = fmaf(wgt[j], v[j].w, acc.w);
+            }
+        }
+    }
+    const int i = (rbase + row) / p.G, gi = (rbase + row) % p.G;
+    __nv_bfloat16* dst = p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + lane * 4;
+    uint2 pk;
+    pk.x = pack_bf16x2(acc.x, acc.y);
+    pk.y = pack_bf16x2(acc.z, acc.w);
+    *reinterpret_cast<uint2*>(dst) = pk;
+}
+
+// grid (span h, request bl, 8-row chunk)
 __global__ void __launch_bounds__(kMergeThreads)
 verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     __shared__ long long s_red[2][kMergeThreads / 32];
-    __shared__ int s_slots[kMaxGrid];
+    __shared__ int s_slots[2 * kMaxGrid];
     __shared__ int s_np;
     const int h = blockIdx.x, bl = blockIdx.y;
     const int nb = p.n_batch;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int l_cap = p.max_pages * p.ps;
 
-    // tiles before request bl, and in total (x heads)
+    // tiles before request bl, and in total (x spans)
     long long before = 0, total = 0;
     for (int b = threadIdx.x; b < nb; b += kMergeThreads) {
         int L = __ldg(p.ctx_lens + p.b_base + b);
@@ -707,7 +780,7 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
         const int c_last = owner_of(span0 + T - 1, W, Gc);
         int n_p = 0;
         long long start_c = (long long)c_first * W / Gc;
-        for (int cc = c_first; cc <= c_last && n_p < kMaxGrid; ++cc) {
+        for (int cc = c_first; cc <= c_last && n_p < 2 * kMaxGrid; ++cc) {
             const long long start_n = (long long)(cc + 1) * W / Gc;
             if (start_n > start_c) s_slots[n_p++] = 2 * cc + ((cc == c_first && span0 > start_c) ? 1 : 0);
             start_c = start_n;
@@ -724,65 +797,50 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (n_p <= 1) return;   // written whole by the main kernel
+    merge_row(p, s_slots, n_p, bl, h, blockIdx.z * kMergeRows + warp, lane);
+}
 
-    const int bg = p.b_base + bl;
-    const int head = h / p.n_rb, rbase = (h - head * p.n_rb) * p.n_rows;
-    const int row = blockIdx.z * kMergeRows + warp;
-    if (row < p.n_rows && rbase + row < p.n_rows_all) {
-        // Every piece left its own normalised output o_q and (m_q, l_q); the
-        // row's output is sum_q w_q o_q with w_q = l_q 2^(m_q - M) / sum_r
-        // l_r 2^(m_r - M), a convex combination.  Pass 1 (lanes across the
-        // pieces): M and the total weight.  Pass 2 (lanes across the 128
-        // dims, one 512-byte read per piece, eight pieces in flight): the sum.
-        float M = kNegInf;
-        for (int q = lane; q < n_p; q += 32) M = fmaxf(M, __ldcg(&p.part_ml[(size_t)s_slots[q] * p.n_rows + row]).x);
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-        float lsum = 0.f;
-        if (M != kNegInf)
-            for (int q = lane; q < n_p; q += 32) {
-                const float2 ml = __ldcg(&p.part_ml[(size_t)s_slots[q] * p.n_rows + row]);
-                if (ml.x != kNegInf) lsum = fmaf(ml.y, ex2(ml.x - M), lsum);
-            }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
-        const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int q0 = 0; q0 < n_p && inv > 0.f; q0 += 32) {
-            float wq = 0.f;   // the weight of piece q0 + lane
-            if (q0 + lane < n_p) {
-                const float2 ml = __ldcg(&p.part_ml[(size_t)s_slots[q0 + lane] * p.n_rows + row]);
-                wq = ml.x == kNegInf ? 0.f : ml.y * ex2(ml.x - M) * inv;
-            }
-            const int nq = min(32, n_p - q0);
-            for (int qq = 0; qq < nq; qq += kMergePieces) {
-                float4 v[kMergePieces];
-                float wgt[kMergePieces];
-#pragma unroll
-                for (int j = 0; j < kMergePieces; ++j) {
-                    const bool ok = qq + j < nq;
-                    wgt[j] = __shfl_sync(0xffffffffu, wq, (qq + j) & 31);
-                    const size_t sl = (size_t)s_slots[q0 + (ok ? qq + j : 0)];
-                    v[j] = ok ? __ldcg(reinterpret_cast<const float4*>(p.part_o + (sl * p.n_rows + row) * kD + lane * 4))
-                              : make_float4(0.f, 0.f, 0.f, 0.f);
-                    if (!ok) wgt[j] = 0.f;
-                }
-#pragma unroll
-                for (int j = 0; j < kMergePieces; ++j) {
-                    acc.x = fmaf(wgt[j], v[j].x, acc.x);
-                    acc.y = fmaf(wgt[j], v[j].y, acc.y);
-                    acc.z = fmaf(wgt[j], v[j].z, acc.z);
-                    acc.w = fmaf(wgt[j], v[j].w, acc.w);
-                }
+// grid (partial slot, 8-row chunk)
+__global__ void __launch_bounds__(kMergeThreads)
+verify_attention_merge_slots_kernel(const AttnParams p, int n_slots) {
+    __shared__ int s_slots[2 * kMaxGrid];
+    __shared__ int s_win[kMergeBack + kMergeAhead];
+    __shared__ int s_np;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    // the slot list is the main kernel's output (see the other form on why
+    // every CTA waits)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const int s0 = blockIdx.x;
+    const int w0 = s0 - kMergeBack;
+    if (threadIdx.x < kMergeBack + kMergeAhead) {
+        const int r = w0 + (int)threadIdx.x;
+        s_win[threadIdx.x] = r >= 0 && r < n_slots ? __ldcg(&p.part_span[r]) : -1;
+    }
+    __syncthreads();
+    const int id = s_win[kMergeBack];
+    if (id < 0) return;
+    auto span_of = [&](int r) {
+        return r >= w0 && r - w0 < kMergeBack + kMergeAhead ? s_win[r - w0] : __ldcg(&p.part_span[r]);
+    };
+    if (threadIdx.x == 0) {
+        // the first piece: the used slot before s0 belongs to another span
+        int q = s0 - 1;
+        while (q >= 0 && span_of(q) < 0) --q;
+        int n_p = 0;
+        if (q < 0 || span_of(q) != id) {
+            for (int r = s0; r < n_slots && n_p < 2 * kMaxGrid; ++r) {
+                const int v = span_of(r);
+                if (v == id) s_slots[n_p++] = r;
+                else if (v >= 0) break;
             }
         }
-        const int i = (rbase + row) / p.G, gi = (rbase + row) % p.G;
-        __nv_bfloat16* dst = p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + lane * 4;
-        uint2 pk;
-        pk.x = pack_bf16x2(acc.x, acc.y);
-        pk.y = pack_bf16x2(acc.z, acc.w);
-        *reinterpret_cast<uint2*>(dst) = pk;
+        s_np = n_p;
     }
+    __syncthreads();
+    const int n_p = s_np;
+    if (n_p == 0) return;   // not a first piece
+    merge_row(p, s_slots, n_p, id / p.n_vh, id % p.n_vh, blockIdx.y * kMergeRows + warp, lane);
 }
 
 #include "verify_attention_tc.cuh"
@@ -883,17 +941,24 @@ cudaError_t launch_dependent(void (*kern)(Params...), dim3 grid, dim3 block, siz
 
 // The split merge as a programmatic dependent of the main kernel: it may
 // start early and waits (griddepcontrol.wait) before it reads the partials.
+// The form with the smaller grid: per span (n_vh x requests) or per partial
+// slot (2 x the main grid).
 cudaError_t launch_merge(const AttnParams& p, const AttnPlan& pl, cudaStream_t stream) {
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr.val.programmaticStreamSerializationAllowed = 1;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(p.n_vh, p.n_batch, (pl.n_rows + kMergeRows - 1) / kMergeRows);
+    const unsigned chunks = (unsigned)((pl.n_rows + kMergeRows - 1) / kMergeRows);
     cfg.blockDim = dim3(kMergeThreads, 1, 1);
     cfg.stream = stream;
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, verify_attention_merge_kernel, p, (int)pl.grid);
+    if ((long long)p.n_vh * p.n_batch <= 2LL * pl.grid) {
+        cfg.gridDim = dim3(p.n_vh, p.n_batch, chunks);
+        return cudaLaunchKernelEx(&cfg, verify_attention_merge_kernel, p, (int)pl.grid);
+    }
+    cfg.gridDim = dim3(2 * pl.grid, chunks, 1);
+    return cudaLaunchKernelEx(&cfg, verify_attention_merge_slots_kernel, p, 2 * (int)pl.grid);
 }
 
 // Resident CTAs per SM of the kernel at a given block size (cached per device).
@@ -960,6 +1025,8 @@ AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count
     off = align_up(off + sizeof(float) * 2 * (size_t)2 * pl.grid * pl.n_rows, 256);
     pl.off_part_o = off;
     off = align_up(off + sizeof(float) * kD * (size_t)2 * pl.grid * pl.n_rows, 256);
+    pl.off_part_span = off;
+    off = align_up(off + sizeof(int) * (size_t)2 * pl.grid, 256);
     pl.bytes = off;
     return pl;
 }
@@ -996,6 +1063,7 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     p.status = reinterpret_cast<int*>(ws);
     p.part_ml = reinterpret_cast<float2*>(ws + pl.off_part_ml);
     p.part_o = reinterpret_cast<float*>(ws + pl.off_part_o);
+    p.part_span = reinterpret_cast<int*>(ws + pl.off_part_span);
     p.Hq = d.n_q_heads;
     p.Hkv = d.n_kv_heads;
     p.G = pl.group;
@@ -1020,6 +1088,7 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
         if (alt.grid > pl.grid) alt.grid = pl.grid;
         alt.off_part_ml = pl.off_part_ml;
         alt.off_part_o = pl.off_part_o;
+        alt.off_part_span = pl.off_part_span;
         alt.bytes = pl.bytes;
         return launch_verify_attention(d, alt, q, k_pages, v_pages, page_table, ctx_lens, parents, out, workspace,
                                        stream);

@@ -312,7 +312,12 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         if (threadIdx.x == kTcThreads - 1) s_carry = before + inc;
         __syncthreads();
     }
-    if (threadIdx.x == 0) s_prefix[nb] = s_carry;
+    if (threadIdx.x == 0) {
+        s_prefix[nb] = s_carry;
+        // this CTA's two partial slots start unused
+        p.part_span[2 * blockIdx.x] = -1;
+        p.part_span[2 * blockIdx.x + 1] = -1;
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -729,6 +734,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             }
             if (live_row && !complete && half == 0)
                 p.part_ml[slot * p.n_rows + row] = make_float2(m_run == kNegInf ? kNegInf : m_run * c, l_run);
+            if (!complete && threadIdx.x == 128) p.part_span[slot] = cur.b * p.n_vh + cur.h;
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(o_free);
