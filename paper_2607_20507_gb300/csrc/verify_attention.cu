@@ -1004,8 +1004,8 @@ AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count
     pl.row_warps = (pl.n_rows + 15) / 16;
     // few rows: two consumer groups share each tile's keys
     pl.split = pl.row_warps <= kMaxSplitRowWarps ? 2 : 1;
-    // 49..128 rows (one row block) on pages of 16+ tokens: the tcgen05 kernel
-    // (with fewer rows its M = 128 padding costs more than the mma.sync form)
+    // 33..128 rows (one row block) on pages of 16+ tokens: the tcgen05 kernel
+    // (up to 32 rows the key-split mma.sync form streams faster)
     pl.tc = pl.n_rb == 1 && pl.n_rows_all > kTcMinRows && pl.n_rows_all <= kTcRows &&
             d.page_size >= 16 && rows <= 256 && pl.group <= 256 && tc_resident_per_sm() >= 1;
     if (pl.tc) {

@@ -2,13 +2,16 @@
 // (included by verify_attention.cu inside its anonymous namespace, so that it
 // shares the schedule, the parameter block, the tensor maps and the merge).
 //
-// Used for 49..128 query rows per KV head, where the mma.sync consumers of
-// the other form run out of tensor throughput (with fewer rows the M = 128
-// padding of every MMA costs more than it saves).  Same persistent schedule
-// (equal contiguous tile ranges, spans, two partial slots per CTA, merge
-// kernel), one CTA per SM, twelve warps (each SMSP, warp % 4, runs one role
-// warp and two softmax warps):
-//   warp 0  K producer: the span's query rows (one 4-D box per dim half into
+// Used for 33..128 query rows per KV head, where the mma.sync consumers of
+// the other form run out of tensor throughput (up to 32 rows the key-split
+// mma.sync form streams faster than this one with its M = 128 padding).
+// Same persistent schedule (equal contiguous tile ranges, spans, two partial
+// slots per CTA, merge kernel), one CTA per SM, twelve warps.  Each SMSP
+// (warp % 4) runs one role warp and up to two softmax warps; the live
+// softmax warps fill SMSPs 0 and 1 first, so the two producers sit on SMSPs
+// 2 and 3, where they share the issue slots with the fewest softmax warps
+// (with them on SMSPs 0 and 1 the kernel ran 7-15% slower):
+//   warp 2  K producer: the span's query rows (one 4-D box per dim half into
 //           one buffer, refilled once the previous span's rows have been
 //           copied into tensor memory; each half as many 128-byte rows as
 //           the span has: the MMA's 128-row window runs on into whatever
@@ -20,12 +23,12 @@
 //           128-byte swizzle;
 //           beside each stage it leaves whether the tile opens or closes a
 //           piece;
-//   warp 1  V producer: the V tiles through the V ring, the same way.  The
+//   warp 3  V producer: the V tiles through the V ring, the same way.  The
 //           two rings share the 16 KB stages that shared memory holds beside
 //           the query buffer (a third for K, which is released as soon as
 //           its QK is done; the rest for V, held until its PV is done), so
 //           each side runs ahead as far as its own consumer allows;
-//   warp 2  QK issuer (the whole warp waits, one elected lane issues): at
+//   warp 0  QK issuer (the whole warp waits, one elected lane issues): at
 //           a piece's start the query rows from shared into tensor memory
 //           (tcgen05.cp, one buffer per span parity), then per tile
 //           S_t = Q K_t^T into tensor memory (M = 128 padded rows, per page
@@ -35,36 +38,40 @@
 //           ahead of the softmax.  It also allocates the tensor memory (512
 //           columns: four S/P buffers of 64, O in 128, two query buffers of
 //           64);
-//   warp 3  PV issuer: O += P_t V_t (N = 128 dims, 8 steps of 16 keys: 4
+//   warp 1  PV issuer: O += P_t V_t (N = 128 dims, 8 steps of 16 keys: 4
 //           with P_hi, 4 with P_lo) as soon as the softmax releases P_t and
 //           V_t has landed, with P read from tensor memory and V, as stored
 //           in bf16, an MN-major operand (per 16 keys, the rows of one page
 //           piece) whose two dim halves lie one piece half apart; in a span's
 //           last tile it first zeroes the V rows past L_b (their slots may
 //           hold any bits);
-//   warps 4-11 softmax and epilogue, two warps per query row (one row per
-//           lane; warps 4+q and 8+q own tensor-memory lanes 32q..32q+31 and
-//           take keys 0..31 and 32..63 of every tile): mask, running max
-//           (the two halves' maxima swapped through shared memory), exp2,
-//           row sum, P written back over S as two bf16 terms, hi and lo
-//           (bf16 P alone can exceed the output tolerance on rows whose terms
-//           cancel), formed as P * 2^-64 so that no partial sum of P.V
-//           overflows fp32 for any finite bf16 V; O is rescaled in tensor
-//           memory only when the running max grows by more than 2^8 (the
-//           stale max keeps every P below 256); at a span piece's end the row
-//           is normalised and written (bf16) or left as a partial, 64 dims by
-//           each warp of the pair.
+//   warps 4-11 softmax and epilogue, one warp per 16 tensor-memory lanes
+//           (query rows; warp 4+q lanes 32q..32q+15, warp 8+q lanes
+//           32q+16..32q+31; a warp whose lanes hold no query row idles):
+//           threads t and t+16 share the row of lane t % 16 and take keys
+//           0..31 and 32..63 of every tile (16-lane tensor-memory access),
+//           so a row's maximum and sum meet in one shuffle.  Mask, running
+//           max, exp2, row sum, P written back over S as two bf16 terms, hi
+//           and lo (bf16 P alone can exceed the output tolerance on rows
+//           whose terms cancel), formed as P * 2^-64 so that no partial sum
+//           of P.V overflows fp32 for any finite bf16 V; pairs of keys in
+//           packed fp32 arithmetic.  O is rescaled in tensor memory only
+//           when the running max grows by more than 2^8 (the stale max keeps
+//           every P below 256); at a span piece's end the row is normalised
+//           and written (bf16) or left as a partial, dims 0..63 by thread t
+//           and 64..127 by thread t+16.
 // Every mbarrier wait is bounded; a wait that gives up sets the status word
 // and a shared flag that ends every warp's loop.
 
 constexpr int kTcMaxK = 6;                         // K ring depth, at most
 constexpr int kTcMaxV = 10;                        // V ring depth, at most
 constexpr int kTcThreads = 384;                    // 12 warps: 4 roles, 8 softmax (three warps per SMSP)
-constexpr int kTcVWarp = 1;                        // the V producer
-constexpr int kTcQkWarp = 2;                       // the QK issuer (and tensor-memory allocator)
-constexpr int kTcPvWarp = 3;                       // the PV issuer
+constexpr int kTcKWarp = 2;                        // the K producer (and the query rows)
+constexpr int kTcVWarp = 3;                        // the V producer
+constexpr int kTcQkWarp = 0;                       // the QK issuer (and tensor-memory allocator)
+constexpr int kTcPvWarp = 1;                       // the PV issuer
 constexpr int kTcRows = 128;                       // MMA M: query rows, padded
-constexpr int kTcMinRows = 48;                     // fewer query rows take the mma.sync form
+constexpr int kTcMinRows = 32;                     // fewer query rows take the key-split mma.sync form
 constexpr int kTcSBuf = 4;                         // S/P buffers in tensor memory
 constexpr int kTcOCol = kTcSBuf * 64;              // first column of O
 constexpr int kTcQCol = kTcOCol + 128;             // first column of the two query buffers (64 each)
@@ -93,7 +100,7 @@ __host__ __device__ constexpr int tc_smem_bytes(int rows) {
     return 2 * tc_q_half_bytes(rows) + (tc_k_stages(rows) + tc_v_stages(rows)) * kTensorTileBytes + kTcFixedSmem;
 }
 static_assert(tc_k_stages(kTcRows) >= 2 && tc_v_stages(kTcRows) >= 4, "rings too shallow for 128 query rows");
-static_assert((2 * kTcMaxK + 2 * kTcMaxV + 5 + 3 * 4 + 1 + 4) * 8 <= kTcBarBytes, "barrier block too small");
+static_assert((2 * kTcMaxK + 2 * kTcMaxV + 4 + 3 * kTcSBuf + 1) * 8 <= kTcBarBytes, "barrier block too small");
 constexpr float kTcRescale = 8.f;                  // log2 growth of the max that forces a rescale of O
 
 __device__ __forceinline__ uint64_t tc_sw128_desc(uint32_t addr) {
@@ -190,6 +197,77 @@ __device__ __forceinline__ void tc_st16(uint32_t addr, const uint32_t (&r)[16]) 
         : "memory");
 }
 
+// 16 lanes x 32 columns, twice: threads 0..15 read lanes base..base+15 at
+// columns col..col+31, threads 16..31 the same lanes at col + split..  (each
+// thread one lane, 32 consecutive columns)
+template <int kSplitOff>
+__device__ __forceinline__ void tc_ld16x2_32(uint32_t addr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], %33;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+          "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+          "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(addr), "n"(kSplitOff));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+template <int kSplitOff>
+__device__ __forceinline__ void tc_st16x2_32(uint32_t addr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.16x32bx2.x32.b32 [%0], %1, {%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33};" ::"r"(addr),
+        "n"(kSplitOff), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]),
+        "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]),
+        "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+
+template <int kSplitOff>
+__device__ __forceinline__ void tc_st16x2_16(uint32_t addr, const uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.16x32bx2.x16.b32 [%0], %1, {%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+        "%17};" ::"r"(addr),
+        "n"(kSplitOff), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+}
+
+// Packed fp32 pairs (one instruction for both lanes of a pair)
+__device__ __forceinline__ uint64_t f2_pack(float a, float b) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& a, float& b) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ uint64_t f2_sub(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 __device__ __forceinline__ void tc_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -228,10 +306,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     uint64_t* q_cp = q_full + 1;                            // ... and were copied into tensor memory
     uint64_t* q_free = q_cp + 1;                            // [2] last QK of a span done (tensor-memory buffer)
     uint64_t* s_full = q_free + 2;                          // [kTcSBuf] S_t in tensor memory
-    uint64_t* p_full = s_full + kTcSBuf;                    // [kTcSBuf] P_t written (count 8 warps)
+    uint64_t* p_full = s_full + kTcSBuf;                    // [kTcSBuf] P_t written (count: live softmax warps)
     uint64_t* o_ready = p_full + kTcSBuf;                   // [kTcSBuf] PV_t done (S buffer free again)
-    uint64_t* o_free = o_ready + kTcSBuf;                   // O read out by the epilogue (count 8 warps)
-    uint64_t* pair_bar = o_free + 1;                        // [4] a softmax warp pair swapped values
+    uint64_t* o_free = o_ready + kTcSBuf;                   // O read out by the epilogue (count: live softmax warps)
     long long* s_prefix = reinterpret_cast<long long*>(reinterpret_cast<uint8_t*>(bars) + kTcBarBytes);
     int* s_len = reinterpret_cast<int*>(s_prefix + kMaxBatchPerLaunch + 1);
     __shared__ long long s_wtot[kTcThreads / 32];
@@ -240,12 +317,14 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     __shared__ volatile int s_dead;
     __shared__ int s_keys[kTcMaxV];   // keys of the tile in each V stage (V rows past are zeroed)
     __shared__ int s_info[kTcMaxK];   // per K stage, bit 0: the tile opens a span piece, bit 1: ends one
-    __shared__ float s_xch[4 * 2 * 2 * 32];   // softmax pair swaps: [pair][slot][half][lane]
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nb = p.n_batch;
+    // softmax warps with a live query row: 16-lane group g (lanes 16g..16g+15)
+    // belongs to warp 4 + g / 2 + 4 (g % 2); groups past the span's rows idle
+    const int n_live = min(8, (p.n_rows_all + 15) / 16);
 
-    if (warp == 0) {
+    if (warp == kTcKWarp) {
         // the page table of this launch into L2 while the schedule is computed
         const char* tab = reinterpret_cast<const char*>(p.page_table + (size_t)p.b_base * p.max_pages);
         const long long lines = ((long long)nb * p.max_pages * 4 + 127) / 128;
@@ -274,11 +353,10 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         for (int i = 0; i < 2; ++i) mbar_init(&q_free[i], 1);
         for (int i = 0; i < kTcSBuf; ++i) {
             mbar_init(&s_full[i], 1);
-            mbar_init(&p_full[i], 8);
+            mbar_init(&p_full[i], n_live);
             mbar_init(&o_ready[i], 1);
         }
-        mbar_init(o_free, 8);
-        for (int i = 0; i < 4; ++i) mbar_init(&pair_bar[i], 2);
+        mbar_init(o_free, n_live);
         fence_barrier_init();
     }
     // a programmatic dependent of the kernel before it (inputs are read
@@ -332,12 +410,12 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     const int n_tiles = (int)(f1 - f0);
     const uint32_t qrow_bytes = (uint32_t)(p.R * p.G) * 128u;   // one dim half of a span's rows
 
-    if ((warp == 0 || warp == kTcVWarp) && n_tiles > 0) {
+    if ((warp == kTcKWarp || warp == kTcVWarp) && n_tiles > 0) {
         // --------------------------------------------------------- producers
-        // warp 0: the K tiles (and, opening a piece, the query rows) through
+        // warp kTcKWarp: the K tiles (and, opening a piece, the query rows) through
         // the K ring; warp kTcVWarp: the V tiles through the V ring.  Each
         // runs ahead as far as its own ring allows.
-        const bool k_side = warp == 0;
+        const bool k_side = warp == kTcKWarp;
         const int S = k_side ? SK : SV;
         uint8_t* const ring = k_side ? sk : sv;
         uint64_t* const fullb = k_side ? kfull : vfull;
@@ -418,7 +496,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // block barrier pays hundreds of cycles per barrier probe and per
         // tcgen05 instruction).  Each commit tracks the MMAs of its own
         // thread only, and the two streams meet only through barriers:
-        //   warp 1 (QK): S_t = Q K_t^T as soon as K_t has landed and S buffer
+        //   warp kTcQkWarp (QK): S_t = Q K_t^T as soon as K_t has landed and S buffer
         //     t % 4 is free (PV_{t-4} done) -- up to four tiles ahead of the
         //     softmax, whatever the PV stream is doing;
         //   warp kTcPvWarp (PV): O += P_t V_t as soon as the softmax has
@@ -543,44 +621,30 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // every MMA of this warp completes before tensor memory is freed
         if (last_bar != nullptr && !mbar_wait_bounded(last_bar, last_par) && lane == 0)
             atomicOr(p.status, CS_DEVICE_WAIT_TIMEOUT);
-    } else if (warp >= 4 && warp < 12 && n_tiles > 0) {
+    } else if (warp >= 4 && warp < 12 && n_tiles > 0 && ((warp & 3) * 2 + (warp >> 3)) < n_live) {
         // ---------------------------------------------------- softmax, epilogue
-        // Two warps per tensor-memory lane quarter: warp 4+q (half 0) takes
-        // keys 0..31 of every tile, warp 8+q (half 1) keys 32..63, both for
-        // the query rows 32q..32q+31 (one per lane).  They swap their partial
-        // maxima of each tile (and their row sums at a piece's end) through
-        // shared memory, so both hold the same running max and make the same
-        // rescale decisions; each writes its half of P, rescales and writes
-        // its half of O, and keeps its half of the row sum.
-        const int sub = warp & 3, half = warp >= 8 ? 1 : 0;
-        const int kb = half * 32;                              // this warp's first key of a tile
-        const int row = sub * 32 + lane;                       // query row of the span = tensor-memory lane
-        const uint32_t t_row = tmem + ((uint32_t)(sub * 32) << 16);
+        // Two warps per tensor-memory lane quarter q: warp 4+q takes lanes
+        // 32q..32q+15, warp 8+q lanes 32q+16..32q+31 (one query row per lane).
+        // In a warp, threads t and t+16 share the row of lane t % 16: the
+        // first takes keys 0..31 of every tile, the second keys 32..63 (the
+        // 16x32bx2 access shape), so a row's max and sum meet in one shuffle.
+        const int sub = warp & 3, hw = warp >> 3;
+        const int kh = lane >> 4;                              // key half of this thread
+        const int kb = kh * 32;                                // its first key of a tile
+        const int lane0 = sub * 32 + hw * 16;                  // the warp's first tensor-memory lane
+        const int row = lane0 + (lane & 15);                   // query row of the span = tensor-memory lane
+        const uint32_t t_row = tmem + ((uint32_t)lane0 << 16);
         const float c = p.scale_log2;
-        uint32_t n_x = 0;                                      // swaps so far (the same count in both warps)
-        // the partner's value for this lane; false once a wait gave up
-        auto swap = [&](float mine, float& other) -> bool {
-            const int slot = (int)(n_x & 1);
-            s_xch[((sub * 2 + slot) * 2 + half) * 32 + lane] = mine;
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&pair_bar[sub]);
-            const bool ok = __all_sync(0xffffffffu, tc_wait(&pair_bar[sub], n_x & 1, &s_dead, p.status));
-            tc_fence_after();
-            ++n_x;
-            other = s_xch[((sub * 2 + slot) * 2 + (half ^ 1)) * 32 + lane];
-            return ok;
-        };
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
         int seg_t0 = cur.t;
         bool first_seg = true;
-        float m_run = kNegInf, l_half = 0.f;
+        float m_run = kNegInf, l_part = 0.f;
         int lim = 0, tree_base = 0, span_L = 0;
         uint64_t anc = ~0ull;
         auto begin_span = [&](const Cursor& cc) {
             const int L = s_len[cc.b];
             m_run = kNegInf;
-            l_half = 0.f;
+            l_part = 0.f;
             if (kTree) {
                 uint64_t ma, mb;
                 tree_ancestor_masks(p.parents + (size_t)(p.b_base + cc.b) * p.R, p.R, lane, ma, mb);
@@ -601,10 +665,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             if (!tc_wait(&s_full[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) break;
             tc_fence_after();
             float s[32];
-            tc_ld32(t_row + sb * 64 + kb, s);
+            tc_ld16x2_32<32>(t_row + sb * 64, s);
             // ---- mask (tree ancestors or the causal chain, and the context end);
             // padded rows see nothing
-            float mh = kNegInf;
             if (row >= p.n_rows_all) {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) s[e] = kNegInf;
@@ -615,10 +678,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 const uint64_t tr = d >= 64 ? 0ull : (d >= 0 ? anc >> d : (d <= -64 ? 0ull : anc << -d));
                 const uint32_t vis = (uint32_t)(((pre | tr) & live) >> kb);
 #pragma unroll
-                for (int e = 0; e < 32; ++e) {
+                for (int e = 0; e < 32; ++e)
                     if (!((vis >> e) & 1u)) s[e] = kNegInf;
-                    mh = fmaxf(mh, s[e]);
-                }
             } else {
                 const int lim_t = lim - ts - kb;   // keys e < lim_t of this half are visible
                 if (lim_t < 32) {
@@ -626,18 +687,19 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                     for (int e = 0; e < 32; ++e)
                         if (e >= lim_t) s[e] = kNegInf;
                 }
-                // eight independent chains: the maximum is exact in any order
-                float m8[8];
-#pragma unroll
-                for (int j = 0; j < 8; ++j) m8[j] = fmaxf(s[j], s[j + 8]);
-#pragma unroll
-                for (int e = 16; e < 32; ++e) m8[e & 7] = fmaxf(m8[e & 7], s[e]);
-                mh = fmaxf(fmaxf(fmaxf(m8[0], m8[1]), fmaxf(m8[2], m8[3])),
-                           fmaxf(fmaxf(m8[4], m8[5]), fmaxf(m8[6], m8[7])));
             }
-            float mo;
-            if (!swap(mh, mo)) break;
-            const float mt = fmaxf(mh, mo);   // the tile's row maximum, the same in both warps
+            // three-input maxima in independent chains: exact in any order
+            float m4[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) m4[j] = fmax3(s[j], s[j + 4], s[j + 8]);
+#pragma unroll
+            for (int e = 12; e < 28; e += 8)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) m4[j] = fmax3(m4[j], s[e + j], s[e + 4 + j]);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) m4[j] = fmaxf(m4[j], s[28 + j]);
+            const float mh = fmaxf(fmax3(m4[0], m4[1], m4[2]), m4[3]);
+            const float mt = fmaxf(mh, __shfl_xor_sync(0xffffffffu, mh, 16));   // the tile's row maximum
             // ---- running max, lazily: O is rescaled only for a growth > 2^8
             float alpha = 1.f;
             if (mt != kNegInf && (m_run == kNegInf || (mt - m_run) * c > kTcRescale)) {
@@ -645,42 +707,55 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 m_run = mt;
             }
             // ---- P = 2^((s - m) c - 64) (the row sum carries the same 2^-64),
-            // as the sum of two bf16 terms
+            // as the sum of two bf16 terms; pairs of keys in packed fp32
             const float neg = m_run == kNegInf ? 0.f : -m_run * c - kPShift;
-            float r4[4] = {0.f, 0.f, 0.f, 0.f};
+            const uint64_t c2 = f2_pack(c, c), n2 = f2_pack(neg, neg);
+            uint64_t r2[4] = {0ull, 0ull, 0ull, 0ull};   // +0.0f pairs
             uint32_t ph[16], pl[16];
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
-                const float p0 = ex2(fmaf(s[2 * e], c, neg)), p1 = ex2(fmaf(s[2 * e + 1], c, neg));
-                r4[e & 3] += p0 + p1;
-                split_bf16x2(p0, p1, ph[e], pl[e]);
+                float x0, x1;
+                f2_unpack(f2_fma(f2_pack(s[2 * e], s[2 * e + 1]), c2, n2), x0, x1);
+                const float p0 = ex2(x0), p1 = ex2(x1);
+                const uint64_t pp = f2_pack(p0, p1);
+                r2[e & 3] = f2_add(r2[e & 3], pp);
+                const uint32_t hi = pack_bf16x2(p0, p1);
+                float d0, d1;
+                f2_unpack(f2_sub(pp, f2_pack(__uint_as_float(hi << 16), __uint_as_float(hi & 0xffff0000u))), d0, d1);
+                ph[e] = hi;
+                pl[e] = pack_bf16x2(d0, d1);
             }
-            l_half = l_half * alpha + ((r4[0] + r4[1]) + (r4[2] + r4[3]));
-            // ---- a rescale of O (this warp's 64 dims) waits for PV_{t-1}; the
-            // first tile of a piece needs none (its PV overwrites O).
-            // o_ready[b] completes once per tile of S buffer b: PV_{t-5} is
-            // complete (QK_t waited for PV_{t-4}) and PV_{t+3} is not issued,
-            // so the parity of PV_{t-1}'s phase is unambiguous.
+            {
+                float a0, a1, b0, b1;
+                f2_unpack(f2_add(r2[0], r2[1]), a0, a1);
+                f2_unpack(f2_add(r2[2], r2[3]), b0, b1);
+                l_part = l_part * alpha + ((a0 + a1) + (b0 + b1));
+            }
+            // ---- a rescale of O (this warp's 16 rows, all 128 dims) waits for
+            // PV_{t-1}; the first tile of a piece needs none (its PV
+            // overwrites O).  o_ready[b] completes once per tile of S buffer
+            // b: PV_{t-5} is complete (QK_t waited for PV_{t-4}) and PV_{t+3}
+            // is not issued, so the parity of PV_{t-1}'s phase is unambiguous.
             const unsigned need = __ballot_sync(0xffffffffu, alpha != 1.f && cur.t != seg_t0);
             if (need) {
                 const int tp = t - 1;
                 if (!tc_wait(&o_ready[tp % kTcSBuf], (uint32_t)(tp / kTcSBuf) & 1, &s_dead, p.status)) break;
                 tc_fence_after();
 #pragma unroll 1
-                for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
+                for (int c0 = 0; c0 < 64; c0 += 32) {
                     float o[32];
-                    tc_ld32(t_row + kTcOCol + c0, o);
+                    tc_ld16x2_32<64>(t_row + kTcOCol + c0, o);
                     uint32_t r[32];
 #pragma unroll
                     for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(o[i] * alpha);
-                    tc_st32(t_row + kTcOCol + c0, r);
+                    tc_st16x2_32<64>(t_row + kTcOCol + c0, r);
                 }
             }
-            // P as bf16 pairs: keys kb..kb+31 are columns kb/2 .. kb/2+15 of the
-            // buffer (hi) and 32 + kb/2 .. (lo); the S columns there were loaded
-            // by both warps of the pair before the swap
-            tc_st16(t_row + sb * 64 + half * 16, ph);
-            tc_st16(t_row + sb * 64 + 32 + half * 16, pl);
+            // P as bf16 pairs: keys kb..kb+31 are columns kb/2 .. kb/2+15 of
+            // the buffer (hi) and 32 + kb/2 .. (lo); the S columns there were
+            // loaded by this warp (the same lanes) before
+            tc_st16x2_16<16>(t_row + sb * 64, ph);
+            tc_st16x2_16<16>(t_row + sb * 64 + 32, pl);
             tc_wait_st();
             tc_fence_before();
             __syncwarp();
@@ -691,14 +766,12 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 continue;
             }
             // ---- end of a span piece: O after its last PV (every earlier MMA
-            // completes before that commit), then written, each warp its 64
-            // dims; the row sum is the two halves' sum, added in the same
-            // order in both warps
+            // completes before that commit), then written: thread t dims
+            // 0..63 of its row, thread t+16 dims 64..127; the row sum is the
+            // two threads' sum (the same in both: addition commutes)
             if (!tc_wait(&o_ready[sb], (uint32_t)(t / kTcSBuf) & 1, &s_dead, p.status)) break;
             tc_fence_after();
-            float lo;
-            if (!swap(l_half, lo)) break;
-            const float l_run = half == 0 ? l_half + lo : lo + l_half;
+            const float l_run = l_part + __shfl_xor_sync(0xffffffffu, l_part, 16);
             const int bg = p.b_base + cur.b;
             const int head = cur.h / p.n_rb;
             const bool complete = seg_t0 == 0 && cur.t + 1 == cur.T;
@@ -708,13 +781,15 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             // (the merge takes a convex combination)
             const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
 #pragma unroll 1
-            for (int c0 = half * 64; c0 < half * 64 + 64; c0 += 32) {
+            for (int c0 = 0; c0 < 64; c0 += 32) {
                 float o[32];
-                tc_ld32(t_row + kTcOCol + c0, o);
+                tc_ld16x2_32<64>(t_row + kTcOCol + c0, o);
                 if (!live_row) continue;
+                const int dim0 = kh * 64 + c0;
                 if (complete) {
                     const int i = row / p.G, gi = row % p.G;
-                    __nv_bfloat16* dst = p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + c0;
+                    __nv_bfloat16* dst =
+                        p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + dim0;
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
                         uint4 v;
@@ -725,14 +800,14 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                         *reinterpret_cast<uint4*>(dst + 8 * q) = v;
                     }
                 } else {
-                    float* dst = p.part_o + (slot * p.n_rows + row) * kD + c0;
+                    float* dst = p.part_o + (slot * p.n_rows + row) * kD + dim0;
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
                         *reinterpret_cast<float4*>(dst + 4 * q) =
                             make_float4(o[4 * q] * inv, o[4 * q + 1] * inv, o[4 * q + 2] * inv, o[4 * q + 3] * inv);
                 }
             }
-            if (live_row && !complete && half == 0)
+            if (live_row && !complete && kh == 0)
                 p.part_ml[slot * p.n_rows + row] = make_float2(m_run == kNegInf ? kNegInf : m_run * c, l_run);
             if (!complete && threadIdx.x == 128) p.part_span[slot] = cur.b * p.n_vh + cur.h;
             tc_fence_before();

@@ -209,13 +209,23 @@ def test_empty_batch():
     assert out.shape[0] == 0
 
 
-# ---- the tcgen05 form (49..128 query rows per KV head, pages of 16+ tokens)
+# ---- the tcgen05 form (33..128 query rows per KV head, pages of 16+ tokens)
 @pytest.mark.parametrize("k,Hq,Hkv,ps", [(8, 64, 8, 16), (8, 64, 8, 32), (8, 64, 8, 64), (8, 64, 8, 128),
-                                         (8, 64, 8, 256), (6, 28, 4, 16), (15, 64, 8, 32), (16, 32, 8, 16)])
+                                         (8, 64, 8, 256), (6, 28, 4, 16), (15, 64, 8, 32), (16, 32, 8, 16),
+                                         (10, 24, 8, 16), (4, 28, 4, 16), (7, 48, 8, 32)])
 def test_tcgen05_row_counts_and_page_sizes(k, Hq, Hkv, ps):
-    """Boundary row counts (49, 128), every page size the form takes."""
+    """Boundary row counts (33, 128), the 33-48 band (33, 35, 48 rows), and
+    every page size the form takes."""
     inp = W.attention_inputs(small(B=3, k=k, Hq=Hq, Hkv=Hkv, ps=ps, lo=k + 1, hi=900, cell=7000 + k * 10 + ps), DEV)
     assert_parity(gpu(inp), ref(inp), f"tc k={k} G={Hq // Hkv} ps={ps}")
+
+
+@pytest.mark.parametrize("k,Hq,Hkv", [(4, 28, 4), (10, 24, 8), (7, 48, 8)])
+def test_mma_sync_33_to_48_rows_on_8_token_pages(k, Hq, Hkv):
+    """33-48 query rows on pages of 8 tokens take the mma.sync form without
+    the key split (the tcgen05 form needs pages of 16+ tokens)."""
+    inp = W.attention_inputs(small(B=3, k=k, Hq=Hq, Hkv=Hkv, ps=8, lo=k + 1, hi=800, cell=7300 + k * 10 + Hq), DEV)
+    assert_parity(gpu(inp), ref(inp), f"mma.sync k={k} G={Hq // Hkv} ps=8")
 
 
 def test_tcgen05_span_pieces_and_repeat_calls():

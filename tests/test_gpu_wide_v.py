@@ -1,15 +1,14 @@
-"""Verify attention with V entries beyond fp16's range, against the fp64 oracle.
+"""Verify attention with V entries of any finite bf16 magnitude, against the
+fp64 oracle.
 
-The kernels take P.V in fp16 (P rounded to fp16, V converted from bf16,
-exact for |v| <= 65280).  A span piece whose V holds an entry fp16 cannot
-represent (|v| >= 65536, up to bf16's largest, ~3.39e38) switches, from that
-tile on, to bf16 P scaled by 2^-64 against bf16 V, so that no partial sum
-overflows fp32.  These tests plant such entries in the middle of contexts
-(so that a piece enters the wide mode after normal tiles), in draft rows
-(seen by later rows only) and in spans that are cut across CTAs (split
-partials and the merge), for each kernel form: key-split mma.sync (<= 32
-query rows per KV head), producer-converted mma.sync (33-48 rows and row
-blocks of trees), and tcgen05 (49-128 rows).  Outputs are compared element by
+Every kernel form takes P.V on bf16 tensor cores with V as stored and P as
+two bf16 terms (hi + lo), formed as P * 2^-64 (the row sum carries the same
+factor): no partial sum can overflow fp32 for any finite bf16 V, and split
+partials are stored normalised, so the merge cannot overflow either.  These
+tests plant entries far beyond fp16's range (up to ~3.3e38, near bf16's
+largest) in the middle of contexts, in draft rows (seen by later rows only)
+and in spans that are cut across CTAs (split partials and the merge), for
+each kernel form and for tree attention.  Outputs are compared element by
 element with |gpu - oracle| <= 2e-3 + 1e-2 |oracle|.
 """
 import dataclasses
@@ -74,10 +73,11 @@ def small(B, k, Hq, Hkv, ps, lo, hi, cell):
 @pytest.mark.parametrize("k,Hq,Hkv,ps,form", [
     (5, 32, 8, 16, "key-split mma.sync (24 rows)"),
     (1, 32, 8, 16, "key-split mma.sync (8 rows)"),
-    (4, 28, 4, 16, "producer-converted mma.sync (35 rows)"),
+    (4, 28, 4, 16, "tcgen05 (35 rows)"),
+    (4, 28, 4, 8, "mma.sync without key split (35 rows, 8-token pages)"),
     (8, 64, 8, 32, "tcgen05 (72 rows)"),
     (15, 64, 8, 16, "tcgen05 (128 rows)"),
-    (16, 64, 8, 16, "producer-converted mma.sync (136 rows)"),
+    (16, 64, 8, 16, "mma.sync row blocks (136 rows)"),
 ])
 def test_wide_v_matches_oracle(k, Hq, Hkv, ps, form):
     rng = np.random.default_rng(k * 100 + Hq)
@@ -126,8 +126,9 @@ def test_wide_v_tree_attention():
     check(out, expect, "tree")
 
 
-def test_largest_fp16_value_stays_on_the_fp16_path():
-    """65280, the largest bf16 value that fp16 holds, stays on the fp16 path."""
+def test_values_at_the_edge_of_fp16():
+    """65280 (the largest bf16 value fp16 holds) and its negative: the edge
+    where an fp16 P.V product would begin to overflow."""
     inp = W.attention_inputs(small(2, 5, 32, 8, 16, 300, 900, cell=9), DEV)
     rng = np.random.default_rng(3)
     plant(inp, rng, [65280.0, -65280.0])
