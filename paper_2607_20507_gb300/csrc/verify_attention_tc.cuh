@@ -437,53 +437,68 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         Cursor cur = locate(f0, s_prefix, s_len, nb, p.n_vh);
         int pg_cur = batch_pages(0);
         int pg_next = per_batch < n_tiles ? batch_pages(per_batch) : -1;
+        // The next tile's page, position and flags are worked out while the
+        // current one waits for its stage (the cursor walk, the page-id
+        // batches and their lookups stay off the path from a free stage to
+        // its copy).
+        struct Next {
+            int page, L, ts, h, b, valid;
+            bool first, last;
+        } nx;
+        auto prepare = [&](int jt) {
+            const int jb = jt % per_batch;
+            if (jt > 0 && jb == 0) {
+                pg_cur = pg_next;
+                pg_next = jt + per_batch < n_tiles ? batch_pages(jt + per_batch) : -1;
+            }
+            nx.page = __shfl_sync(0xffffffffu, pg_cur, jb * kPieces + lane % kPieces);
+            nx.first = jt == 0 || cur.t == 0;
+            nx.last = jt + 1 == n_tiles || cur.t + 1 == cur.T;
+            nx.L = s_len[cur.b];
+            nx.ts = cur.t * kTileT;
+            nx.h = cur.h / p.n_rb;
+            nx.b = cur.b;
+            advance(cur, s_len, nb, p.n_vh);
+            nx.valid = 0;
+            for (int pc = 0; pc < kPieces; ++pc)
+                if (nx.ts + pc * kBoxT < nx.L) ++nx.valid;
+        };
+        prepare(0);
         int span = -1;
         // tile jt goes out once its stage is free and, K side opening a
         // piece, once the query buffer is free
         int jt = 0;
         for (; jt < n_tiles; ++jt) {
             const int st = jt % S;
-            const bool first = jt == 0 || cur.t == 0;
-            const bool last = jt + 1 == n_tiles || cur.t + 1 == cur.T;
-            if (first) ++span;
+            const Next c = nx;
+            if (c.first) ++span;
             bool go = jt < S || tc_wait(&emptyb[st], (uint32_t)(jt / S - 1) & 1, &s_dead, p.status);
             // the query buffer is free once the previous span's rows are in tensor memory
-            if (go && k_side && first && span >= 1)
+            if (go && k_side && c.first && span >= 1)
                 go = tc_wait(q_cp, (uint32_t)(span - 1) & 1, &s_dead, p.status);
             if (!__all_sync(0xffffffffu, go)) break;
-            const int jb = jt % per_batch;
-            if (jt > 0 && jb == 0) {
-                pg_cur = pg_next;
-                pg_next = jt + per_batch < n_tiles ? batch_pages(jt + per_batch) : -1;
-            }
-            const int page = __shfl_sync(0xffffffffu, pg_cur, jb * kPieces + lane % kPieces);
-            const int L = s_len[cur.b];
-            const int ts = cur.t * kTileT;
-            const int h_cur = cur.h / p.n_rb;
-            if (k_side && first && lane == 0) {
+            if (k_side && c.first && lane == 0) {
                 // a new span piece: its query rows into the query buffer
                 mbar_arrive_expect_tx(q_full, 2 * qrow_bytes);
                 const uint32_t qdst = smem_u32(sq);
 #pragma unroll
                 for (int hh = 0; hh < 2; ++hh)
-                    tma_load_4d(qdst + hh * qh, &tmap_q, q_full, hh * 64, h_cur * p.G, 0, p.b_base + cur.b);
+                    tma_load_4d(qdst + hh * qh, &tmap_q, q_full, hh * 64, c.h * p.G, 0, p.b_base + c.b);
             }
-            advance(cur, s_len, nb, p.n_vh);
-            int valid = 0;
-            for (int pc = 0; pc < kPieces; ++pc)
-                if (ts + pc * kBoxT < L) ++valid;
             if (lane == 0) {
-                if (k_side) s_info[st] = (first ? 1 : 0) | (last ? 2 : 0);
-                else s_keys[st] = max(0, min(kTileT, L - ts));
-                mbar_arrive_expect_tx(&fullb[st], (uint32_t)valid * kPieceBytes);
+                if (k_side) s_info[st] = (c.first ? 1 : 0) | (c.last ? 2 : 0);
+                else s_keys[st] = max(0, min(kTileT, c.L - c.ts));
+                mbar_arrive_expect_tx(&fullb[st], (uint32_t)c.valid * kPieceBytes);
             }
             __syncwarp();
-            if (lane < valid) {
+            if (lane < c.valid) {
                 // one box per page piece, both dim halves: [half][kBoxT keys][128 B]
+                // (page sizes are powers of two)
                 const uint32_t dst = smem_u32(ring + st * kTensorTileBytes) + (uint32_t)lane * kPieceBytes;
-                const int slot = (ts + lane * kBoxT) % p.ps;
-                tma_load_5d(dst, tmap, &fullb[st], 0, slot, 0, h_cur, page);
+                const int slot = (c.ts + lane * kBoxT) & (p.ps - 1);
+                tma_load_5d(dst, tmap, &fullb[st], 0, slot, 0, c.h, c.page);
             }
+            if (jt + 1 < n_tiles) prepare(jt + 1);
         }
         // no copy in flight at exit: every issued tile has landed
         if (lane == 0)
