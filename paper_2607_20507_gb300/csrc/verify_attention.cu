@@ -678,51 +678,88 @@ constexpr int kMergeRows = kMergeThreads / 32;   // query rows per merge CTA
 constexpr int kMergePieces = 8;   // pieces in flight per row
 constexpr int kMergeBack = 32, kMergeAhead = 96;   // slot-list window around a CTA's own slot
 
-// the convex combination of one row's pieces (slots[0..n_p)), by one warp
+// the convex combination of one row's pieces (slots[0..n_p)), by one warp.
+// Up to kMergePieces pieces (the usual case) take one round trip: every
+// piece's (m, l) and this lane's four output columns of every piece are
+// requested together; more pieces go through the general loop.
 __device__ __forceinline__ void merge_row(const AttnParams& p, const int* slots, int n_p, int bl, int h, int row,
                                           int lane) {
     const int bg = p.b_base + bl;
     const int head = h / p.n_rb, rbase = (h - head * p.n_rb) * p.n_rows;
     if (row >= p.n_rows || rbase + row >= p.n_rows_all) return;
-    float M = kNegInf;
-    for (int q = lane; q < n_p; q += 32) M = fmaxf(M, __ldcg(&p.part_ml[(size_t)slots[q] * p.n_rows + row]).x);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    float lsum = 0.f;
-    if (M != kNegInf)
-        for (int q = lane; q < n_p; q += 32) {
-            const float2 ml = __ldcg(&p.part_ml[(size_t)slots[q] * p.n_rows + row]);
-            if (ml.x != kNegInf) lsum = fmaf(ml.y, ex2(ml.x - M), lsum);
-        }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
-    const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int q0 = 0; q0 < n_p && inv > 0.f; q0 += 32) {
-        float wq = 0.f;   // the weight of piece q0 + lane
-        if (q0 + lane < n_p) {
-            const float2 ml = __ldcg(&p.part_ml[(size_t)slots[q0 + lane] * p.n_rows + row]);
-            wq = ml.x == kNegInf ? 0.f : ml.y * ex2(ml.x - M) * inv;
-        }
-        const int nq = min(32, n_p - q0);
-        for (int qq = 0; qq < nq; qq += kMergePieces) {
-            float4 v[kMergePieces];
-            float wgt[kMergePieces];
+    if (n_p <= kMergePieces) {
+        float4 v[kMergePieces];
+        float2 ml = make_float2(kNegInf, 0.f);   // lane q < n_p: piece q
+        if (lane < n_p) ml = __ldcg(&p.part_ml[(size_t)slots[lane] * p.n_rows + row]);
 #pragma unroll
-            for (int j = 0; j < kMergePieces; ++j) {
-                const bool ok = qq + j < nq;
-                wgt[j] = __shfl_sync(0xffffffffu, wq, (qq + j) & 31);
-                const size_t sl = (size_t)slots[q0 + (ok ? qq + j : 0)];
-                v[j] = ok ? __ldcg(reinterpret_cast<const float4*>(p.part_o + (sl * p.n_rows + row) * kD + lane * 4))
-                          : make_float4(0.f, 0.f, 0.f, 0.f);
-                if (!ok) wgt[j] = 0.f;
+        for (int j = 0; j < kMergePieces; ++j) {
+            v[j] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (j < n_p)
+                v[j] = __ldcg(reinterpret_cast<const float4*>(p.part_o + ((size_t)slots[j] * p.n_rows + row) * kD +
+                                                              lane * 4));
+        }
+        float M = ml.x;
+#pragma unroll
+        for (int off = 4; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+        M = __shfl_sync(0xffffffffu, M, 0);
+        float wq = (M == kNegInf || ml.x == kNegInf) ? 0.f : ml.y * ex2(ml.x - M);
+        float lsum = wq;
+#pragma unroll
+        for (int off = 4; off > 0; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+        lsum = __shfl_sync(0xffffffffu, lsum, 0);
+        const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+        wq *= inv;
+#pragma unroll
+        for (int j = 0; j < kMergePieces; ++j) {
+            const float wgt = __shfl_sync(0xffffffffu, wq, j);
+            if (j < n_p) {
+                acc.x = fmaf(wgt, v[j].x, acc.x);
+                acc.y = fmaf(wgt, v[j].y, acc.y);
+                acc.z = fmaf(wgt, v[j].z, acc.z);
+                acc.w = fmaf(wgt, v[j].w, acc.w);
+            }
+        }
+    } else {
+        float M = kNegInf;
+        for (int q = lane; q < n_p; q += 32) M = fmaxf(M, __ldcg(&p.part_ml[(size_t)slots[q] * p.n_rows + row]).x);
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+        float lsum = 0.f;
+        if (M != kNegInf)
+            for (int q = lane; q < n_p; q += 32) {
+                const float2 ml = __ldcg(&p.part_ml[(size_t)slots[q] * p.n_rows + row]);
+                if (ml.x != kNegInf) lsum = fmaf(ml.y, ex2(ml.x - M), lsum);
             }
 #pragma unroll
-            for (int j = 0; j < kMergePieces; ++j) {
-                acc.x = fmaf(wgt[j], v[j].x, acc.x);
-                acc.y = fmaf(wgt[j], v[j].y, acc.y);
-                acc.z = fmaf(wgt[j], v[j].z, acc.z);
-                acc.w = fmaf(wgt[j], v[j].w, acc.w);
+        for (int off = 16; off > 0; off >>= 1) lsum += __shfl_xor_sync(0xffffffffu, lsum, off);
+        const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
+        for (int q0 = 0; q0 < n_p && inv > 0.f; q0 += 32) {
+            float wq = 0.f;   // the weight of piece q0 + lane
+            if (q0 + lane < n_p) {
+                const float2 ml = __ldcg(&p.part_ml[(size_t)slots[q0 + lane] * p.n_rows + row]);
+                wq = ml.x == kNegInf ? 0.f : ml.y * ex2(ml.x - M) * inv;
+            }
+            const int nq = min(32, n_p - q0);
+            for (int qq = 0; qq < nq; qq += kMergePieces) {
+                float4 v[kMergePieces];
+                float wgt[kMergePieces];
+#pragma unroll
+                for (int j = 0; j < kMergePieces; ++j) {
+                    const bool ok = qq + j < nq;
+                    wgt[j] = __shfl_sync(0xffffffffu, wq, (qq + j) & 31);
+                    const size_t sl = (size_t)slots[q0 + (ok ? qq + j : 0)];
+                    v[j] = ok ? __ldcg(reinterpret_cast<const float4*>(p.part_o + (sl * p.n_rows + row) * kD + lane * 4))
+                              : make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (!ok) wgt[j] = 0.f;
+                }
+#pragma unroll
+                for (int j = 0; j < kMergePieces; ++j) {
+                    acc.x = fmaf(wgt[j], v[j].x, acc.x);
+                    acc.y = fmaf(wgt[j], v[j].y, acc.y);
+                    acc.z = fmaf(wgt[j], v[j].z, acc.z);
+                    acc.w = fmaf(wgt[j], v[j].w, acc.w);
+                }
             }
         }
     }
