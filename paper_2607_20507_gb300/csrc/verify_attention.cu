@@ -916,17 +916,18 @@ cs_status encode_pool_map(CUtensorMap* map, const void* pool, const cs_attn_dims
     return CS_OK;
 }
 
-// The query rows of one KV head of one request as one box per dim half: q
-// [B, R, Hq, D] seen as (D, Hq, R, B), box (64, G, R, 1), landing as
-// [draft row][group head][64 dims] = query row i*G + g.
-cs_status encode_q_map(CUtensorMap* map, const void* q, const cs_attn_dims& d, int rows) {
+// The query rows of one KV head of one request (or of one row block of
+// them) as one box per dim half: q [B, R, Hq, D] seen as (D, Hq, R, B), box
+// (64, G, box_rows, 1), landing as [draft row][group head][64 dims] = query
+// row i*G + g of the block.  A block that runs past row R reads zeros there.
+cs_status encode_q_map(CUtensorMap* map, const void* q, const cs_attn_dims& d, int rows, int box_rows) {
     auto enc = tensor_map_encoder();
     if (!enc) return fail(CS_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
     const int G = d.n_q_heads / d.n_kv_heads;
     const cuuint64_t dims[4] = {(cuuint64_t)d.head_dim, (cuuint64_t)d.n_q_heads, (cuuint64_t)rows, (cuuint64_t)d.batch};
     const cuuint64_t row = (cuuint64_t)d.head_dim * 2;
     const cuuint64_t strides[3] = {row, row * d.n_q_heads, row * d.n_q_heads * rows};
-    const cuuint32_t box[4] = {64, (cuuint32_t)G, (cuuint32_t)rows, 1};
+    const cuuint32_t box[4] = {64, (cuuint32_t)G, (cuuint32_t)box_rows, 1};
     const cuuint32_t estr[4] = {1, 1, 1, 1};
     const CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(q), dims, strides, box, estr,
                            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -1027,7 +1028,23 @@ int resident_per_sm(int threads) {
 
 }  // namespace
 
-AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count) {
+// Workspace layout of a plan: the status word (256 B), then the split
+// partials (m, l) [2 grid, rows], O [2 grid, rows, D] and the span of each
+// partial slot [2 grid].
+void attn_layout(AttnPlan& pl) {
+    size_t off = 256;
+    pl.off_part_ml = off;
+    off = align_up(off + sizeof(float) * 2 * (size_t)2 * pl.grid * pl.n_rows, 256);
+    pl.off_part_o = off;
+    off = align_up(off + sizeof(float) * kD * (size_t)2 * pl.grid * pl.n_rows, 256);
+    pl.off_part_span = off;
+    off = align_up(off + sizeof(int) * (size_t)2 * pl.grid, 256);
+    pl.bytes = off;
+}
+
+// allow_tc: whether the tcgen05 form may be chosen (the mma.sync form's own
+// plan otherwise)
+AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count, bool allow_tc = true) {
     AttnPlan pl{};
     pl.group = d.n_q_heads / d.n_kv_heads;
     pl.rows = rows;
@@ -1041,11 +1058,23 @@ AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count
     pl.row_warps = (pl.n_rows + 15) / 16;
     // few rows: two consumer groups share each tile's keys
     pl.split = pl.row_warps <= kMaxSplitRowWarps ? 2 : 1;
-    // 33..128 rows (one row block) on pages of 16+ tokens: the tcgen05 kernel
-    // (up to 32 rows the key-split mma.sync form streams faster)
-    pl.tc = pl.n_rb == 1 && pl.n_rows_all > kTcMinRows && pl.n_rows_all <= kTcRows &&
-            d.page_size >= 16 && rows <= 256 && pl.group <= 256 && tc_resident_per_sm() >= 1;
+    // more than 32 rows on pages of 16+ tokens: the tcgen05 kernel (up to 32
+    // rows the key-split mma.sync form streams faster), in one block of up
+    // to 128 rows or -- trees -- in row blocks of whole nodes of at most 128
+    // rows each, every block its own span (its keys are then read once per
+    // block)
+    int tc_rb = 1, tc_rows = pl.n_rows_all;
+    while (tree && tc_rows > kTcRows && tc_rb < rows) {
+        ++tc_rb;
+        tc_rows = ((rows + tc_rb - 1) / tc_rb) * pl.group;
+    }
+    pl.tc = allow_tc && tc_rows > kTcMinRows && tc_rows <= kTcRows && d.page_size >= 16 && rows <= 256 &&
+            pl.group <= 256 &&
+            tc_resident_per_sm() >= 1;
     if (pl.tc) {
+        pl.n_rb = tc_rb;
+        pl.n_rows = tc_rows;
+        pl.row_warps = (pl.n_rows + 15) / 16;
         pl.split = 1;
         pl.grid = (sm_count > 0 ? sm_count : 148) * tc_resident_per_sm();
         if (pl.grid > kMaxGrid) pl.grid = kMaxGrid;
@@ -1057,14 +1086,15 @@ AttnPlan plan_attention(const cs_attn_dims& d, int rows, bool tree, int sm_count
         pl.grid = (sm_count > 0 ? sm_count : 148) * res;
         if (pl.grid > kMaxGrid) pl.grid = kMaxGrid;
     }
-    size_t off = 256;   // status word lives at offset 0
-    pl.off_part_ml = off;
-    off = align_up(off + sizeof(float) * 2 * (size_t)2 * pl.grid * pl.n_rows, 256);
-    pl.off_part_o = off;
-    off = align_up(off + sizeof(float) * kD * (size_t)2 * pl.grid * pl.n_rows, 256);
-    pl.off_part_span = off;
-    off = align_up(off + sizeof(int) * (size_t)2 * pl.grid, 256);
-    pl.bytes = off;
+    attn_layout(pl);
+    if (pl.tc) {
+        // a query buffer TMA cannot read falls back to the mma.sync form on
+        // the same workspace (its grid capped at this one): room for both
+        AttnPlan alt = plan_attention(d, rows, tree, sm_count, false);
+        if (alt.grid > pl.grid) alt.grid = pl.grid;
+        attn_layout(alt);
+        if (alt.bytes > pl.bytes) pl.bytes = alt.bytes;
+    }
     return pl;
 }
 
@@ -1120,19 +1150,15 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
         // the query rows come in by TMA, which needs a 16-byte aligned base:
         // run the mma.sync form on the same workspace (its grid capped at
         // the plan's, so the partial slots fit)
-        AttnPlan alt = plan_attention(d, pl.rows, pl.tree, 0);
-        alt.tc = false;
+        AttnPlan alt = plan_attention(d, pl.rows, pl.tree, 0, false);
         if (alt.grid > pl.grid) alt.grid = pl.grid;
-        alt.off_part_ml = pl.off_part_ml;
-        alt.off_part_o = pl.off_part_o;
-        alt.off_part_span = pl.off_part_span;
-        alt.bytes = pl.bytes;
+        attn_layout(alt);   // fits: the tcgen05 plan's size covers this layout
         return launch_verify_attention(d, alt, q, k_pages, v_pages, page_table, ctx_lens, parents, out, workspace,
                                        stream);
     }
     if (pl.tc) {
         CUtensorMap tq;
-        st = encode_q_map(&tq, q, d, pl.rows);
+        st = encode_q_map(&tq, q, d, pl.rows, pl.n_rows / pl.group);
         if (st != CS_OK) return st;
         // one box per page piece with both dim halves, as for the other form
 
@@ -1144,10 +1170,10 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
              verify_attention_tc_kernel<true, 64>}};
         const int ti = box_t == 16 ? 0 : box_t == 32 ? 1 : 2;
         const TcKern tk_fn = tc_kerns[pl.tree][ti];
-        p.tc_stages = tc_k_stages(pl.n_rows_all);
-        p.tc_vstages = tc_v_stages(pl.n_rows_all);
-        p.tc_q_half = tc_q_half_bytes(pl.n_rows_all);
-        const int smem_bytes = tc_smem_bytes(pl.n_rows_all);
+        p.tc_stages = tc_k_stages(pl.n_rows);
+        p.tc_vstages = tc_v_stages(pl.n_rows);
+        p.tc_q_half = tc_q_half_bytes(pl.n_rows);
+        const int smem_bytes = tc_smem_bytes(pl.n_rows);
         cudaError_t e = cudaFuncSetAttribute(tk_fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
         if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(verify_attention_tc_kernel)");
         for (int b0 = 0; b0 < d.batch; b0 += kMaxBatchPerLaunch) {

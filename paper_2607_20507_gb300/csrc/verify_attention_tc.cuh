@@ -4,7 +4,10 @@
 //
 // Used for 33..128 query rows per KV head, where the mma.sync consumers of
 // the other form run out of tensor throughput (up to 32 rows the key-split
-// mma.sync form streams faster than this one with its M = 128 padding).
+// mma.sync form streams faster than this one with its M = 128 padding).  A
+// token tree with more rows comes in row blocks of whole nodes, at most 128
+// rows each; each block is a span of its own (reading the request's keys
+// again) whose query box starts at the block's first node.
 // Same persistent schedule (equal contiguous tile ranges, spans, two partial
 // slots per CTA, merge kernel), one CTA per SM, twelve warps.  Each SMSP
 // (warp % 4) runs one role warp and up to two softmax warps; the live
@@ -322,7 +325,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     const int nb = p.n_batch;
     // softmax warps with a live query row: 16-lane group g (lanes 16g..16g+15)
     // belongs to warp 4 + g / 2 + 4 (g % 2); groups past the span's rows idle
-    const int n_live = min(8, (p.n_rows_all + 15) / 16);
+    const int n_live = min(8, ((kTree ? p.n_rows : p.n_rows_all) + 15) / 16);
 
     if (warp == kTcKWarp) {
         // the page table of this launch into L2 while the schedule is computed
@@ -408,7 +411,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     long long f0 = (long long)cta * W / Gc, f1 = (long long)(cta + 1) * W / Gc;
     if (cta >= Gc) f0 = f1 = 0;
     const int n_tiles = (int)(f1 - f0);
-    const uint32_t qrow_bytes = (uint32_t)(p.R * p.G) * 128u;   // one dim half of a span's rows
+    // one dim half of a span's rows (trees: of its row block of q_nodes nodes)
+    const uint32_t qrow_bytes = (uint32_t)(kTree ? p.n_rows : p.R * p.G) * 128u;
+    const int q_nodes = p.n_rows / p.G;
 
     if ((warp == kTcKWarp || warp == kTcVWarp) && n_tiles > 0) {
         // --------------------------------------------------------- producers
@@ -442,7 +447,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         // batches and their lookups stay off the path from a free stage to
         // its copy).
         struct Next {
-            int page, L, ts, h, b, valid;
+            int page, L, ts, h, rb, b, valid;
             bool first, last;
         } nx;
         auto prepare = [&](int jt) {
@@ -457,6 +462,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             nx.L = s_len[cur.b];
             nx.ts = cur.t * kTileT;
             nx.h = cur.h / p.n_rb;
+            if (kTree) nx.rb = cur.h - nx.h * p.n_rb;
             nx.b = cur.b;
             advance(cur, s_len, nb, p.n_vh);
             nx.valid = 0;
@@ -483,7 +489,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 const uint32_t qdst = smem_u32(sq);
 #pragma unroll
                 for (int hh = 0; hh < 2; ++hh)
-                    tma_load_4d(qdst + hh * qh, &tmap_q, q_full, hh * 64, c.h * p.G, 0, p.b_base + c.b);
+                    tma_load_4d(qdst + hh * qh, &tmap_q, q_full, hh * 64, c.h * p.G, kTree ? c.rb * q_nodes : 0,
+                                p.b_base + c.b);
             }
             if (lane == 0) {
                 if (k_side) s_info[st] = (c.first ? 1 : 0) | (c.last ? 2 : 0);
@@ -655,17 +662,24 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
         bool first_seg = true;
         float m_run = kNegInf, l_part = 0.f;
         int lim = 0, tree_base = 0, span_L = 0;
+        // trees may come in row blocks: the query row of the request and KV
+        // head is the block's first row + row, and rows past the block's
+        // end are padding; a chain is one block
+        int qrow = row;
+        bool tree_live = false;
         uint64_t anc = ~0ull;
         auto begin_span = [&](const Cursor& cc) {
             const int L = s_len[cc.b];
             m_run = kNegInf;
             l_part = 0.f;
             if (kTree) {
+                qrow = (cc.h % p.n_rb) * p.n_rows + row;
+                tree_live = row < p.n_rows && qrow < p.n_rows_all;
                 uint64_t ma, mb;
                 tree_ancestor_masks(p.parents + (size_t)(p.b_base + cc.b) * p.R, p.R, lane, ma, mb);
-                const int i = row / p.G;
+                const int i = tree_live ? qrow / p.G : 0;
                 const uint64_t x = __shfl_sync(0xffffffffu, ma, i & 31), y = __shfl_sync(0xffffffffu, mb, i & 31);
-                anc = row < p.n_rows_all ? (i >= 32 ? y : x) : ~0ull;
+                anc = tree_live ? (i >= 32 ? y : x) : ~0ull;
                 tree_base = L - p.R;
                 span_L = L;
             } else {
@@ -683,7 +697,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             tc_ld16x2_32<32>(t_row + sb * 64, s);
             // ---- mask (tree ancestors or the causal chain, and the context end);
             // padded rows see nothing
-            if (row >= p.n_rows_all) {
+            if (kTree ? !tree_live : row >= p.n_rows_all) {
 #pragma unroll
                 for (int e = 0; e < 32; ++e) s[e] = kNegInf;
             } else if (kTree) {
@@ -791,7 +805,7 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
             const int head = cur.h / p.n_rb;
             const bool complete = seg_t0 == 0 && cur.t + 1 == cur.T;
             const size_t slot = 2 * (size_t)cta + (first_seg ? 0 : 1);
-            const bool live_row = row < p.n_rows_all;
+            const bool live_row = kTree ? tree_live : row < p.n_rows_all;
             // normalised output; a partial is the piece's own normalised output
             // (the merge takes a convex combination)
             const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
@@ -802,7 +816,8 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
                 if (!live_row) continue;
                 const int dim0 = kh * 64 + c0;
                 if (complete) {
-                    const int i = row / p.G, gi = row % p.G;
+                    const int qr = kTree ? qrow : row;
+                    const int i = qr / p.G, gi = qr % p.G;
                     __nv_bfloat16* dst =
                         p.out + (((size_t)bg * p.R + i) * p.Hq + (size_t)head * p.G + gi) * kD + dim0;
 #pragma unroll
