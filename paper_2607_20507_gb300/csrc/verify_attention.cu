@@ -659,41 +659,49 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 // Merge of split spans.  Each piece of a cut span left its own normalised
 // output o_q and (m_q, l_q); the span's output is sum_q w_q o_q with
 // w_q = l_q 2^(m_q - M) / sum_r l_r 2^(m_r - M), a convex combination (no
-// value can overflow).  One warp per query row: pass 1 (lanes across the
-// pieces) finds M and the total weight, pass 2 (lanes across the 128 dims,
-// one coalesced 512-byte read per piece, eight pieces in flight) the sum.
-// A CTA holds 8 rows of one span.  Two ways to find a span's pieces, the
-// launch taking the one with the smaller grid:
+// value can overflow).  One warp per query row (lanes across the pieces for
+// the weights, across the 128 dims for the sum).
+// Two ways to find a span's pieces, the launch taking the one with the
+// smaller grid:
 //  * per span: every CTA recomputes the main kernel's schedule from the
-//    context lengths (cheap for few requests) and finds the CTAs that cut
-//    its span; a span with a single piece was written whole and is skipped;
-//  * per partial slot: the main kernel records the span of each partial slot
-//    (-1 when unused).  In slot order (CTA c's first piece 2c, its last 2c+1)
-//    a cut span's pieces are consecutive, unused slots aside, so the CTA of
-//    a span's first slot gathers them from a window of the list read into
-//    shared memory.  The grid no longer grows with the number of spans.
+//    context lengths (cheap for few requests, and done while the main
+//    kernel runs) and finds the CTAs that cut its span; a span with a single
+//    piece was written whole and is skipped;
+//  * per main-kernel CTA: the main kernels record the span of each partial
+//    slot (-1 when unused):
+// slot 2c holds CTA c's first piece, 2c + 1 its last one when that is a
+// different piece.  In slot order a cut span's pieces are consecutive,
+// unused slots aside, and at most one cut span starts in each CTA: its last
+// piece, or -- one piece only -- that piece, unless the previous CTA's last
+// piece belongs to the same span.  Merge CTA (c, y) reads the slot list
+// around CTA c once into shared memory, gathers the pieces of the span that
+// starts in CTA c (if any) and merges rows 8y .. 8y + 7 of it.  Six merge
+// CTAs fit an SM, so the whole grid is resident at once in the usual case.
 // ---------------------------------------------------------------------------
 constexpr int kMergeThreads = 256;
 constexpr int kMergeRows = kMergeThreads / 32;   // query rows per merge CTA
-constexpr int kMergePieces = 8;   // pieces in flight per row
-constexpr int kMergeBack = 32, kMergeAhead = 96;   // slot-list window around a CTA's own slot
+constexpr int kMergePerSm = 6;                   // merge CTAs resident per SM (registers capped to fit)
+constexpr int kMergePieces = 8;                  // pieces of a row merged in one round trip (per-span form)
+constexpr int kMergePiecesCut = 4;               // the same for the register-capped per-CTA form
+constexpr int kMergeWin = 64;                    // slots read ahead of CTA c's first slot
 
 // the convex combination of one row's pieces (slots[0..n_p)), by one warp.
-// Up to kMergePieces pieces (the usual case) take one round trip: every
+// Up to kPieces pieces (the usual case) take one round trip: every
 // piece's (m, l) and this lane's four output columns of every piece are
 // requested together; more pieces go through the general loop.
+template <int kPieces>
 __device__ __forceinline__ void merge_row(const AttnParams& p, const int* slots, int n_p, int bl, int h, int row,
                                           int lane) {
     const int bg = p.b_base + bl;
     const int head = h / p.n_rb, rbase = (h - head * p.n_rb) * p.n_rows;
     if (row >= p.n_rows || rbase + row >= p.n_rows_all) return;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (n_p <= kMergePieces) {
-        float4 v[kMergePieces];
+    if (n_p <= kPieces) {
+        float4 v[kPieces];
         float2 ml = make_float2(kNegInf, 0.f);   // lane q < n_p: piece q
         if (lane < n_p) ml = __ldcg(&p.part_ml[(size_t)slots[lane] * p.n_rows + row]);
 #pragma unroll
-        for (int j = 0; j < kMergePieces; ++j) {
+        for (int j = 0; j < kPieces; ++j) {
             v[j] = make_float4(0.f, 0.f, 0.f, 0.f);
             if (j < n_p)
                 v[j] = __ldcg(reinterpret_cast<const float4*>(p.part_o + ((size_t)slots[j] * p.n_rows + row) * kD +
@@ -711,7 +719,7 @@ __device__ __forceinline__ void merge_row(const AttnParams& p, const int* slots,
         const float inv = lsum > 0.f ? 1.f / lsum : 0.f;
         wq *= inv;
 #pragma unroll
-        for (int j = 0; j < kMergePieces; ++j) {
+        for (int j = 0; j < kPieces; ++j) {
             const float wgt = __shfl_sync(0xffffffffu, wq, j);
             if (j < n_p) {
                 acc.x = fmaf(wgt, v[j].x, acc.x);
@@ -741,11 +749,11 @@ __device__ __forceinline__ void merge_row(const AttnParams& p, const int* slots,
                 wq = ml.x == kNegInf ? 0.f : ml.y * ex2(ml.x - M) * inv;
             }
             const int nq = min(32, n_p - q0);
-            for (int qq = 0; qq < nq; qq += kMergePieces) {
-                float4 v[kMergePieces];
-                float wgt[kMergePieces];
+            for (int qq = 0; qq < nq; qq += kPieces) {
+                float4 v[kPieces];
+                float wgt[kPieces];
 #pragma unroll
-                for (int j = 0; j < kMergePieces; ++j) {
+                for (int j = 0; j < kPieces; ++j) {
                     const bool ok = qq + j < nq;
                     wgt[j] = __shfl_sync(0xffffffffu, wq, (qq + j) & 31);
                     const size_t sl = (size_t)slots[q0 + (ok ? qq + j : 0)];
@@ -754,7 +762,7 @@ __device__ __forceinline__ void merge_row(const AttnParams& p, const int* slots,
                     if (!ok) wgt[j] = 0.f;
                 }
 #pragma unroll
-                for (int j = 0; j < kMergePieces; ++j) {
+                for (int j = 0; j < kPieces; ++j) {
                     acc.x = fmaf(wgt[j], v[j].x, acc.x);
                     acc.y = fmaf(wgt[j], v[j].y, acc.y);
                     acc.z = fmaf(wgt[j], v[j].z, acc.z);
@@ -773,7 +781,7 @@ __device__ __forceinline__ void merge_row(const AttnParams& p, const int* slots,
 
 // grid (span h, request bl, 8-row chunk)
 __global__ void __launch_bounds__(kMergeThreads)
-verify_attention_merge_kernel(const AttnParams p, int grid_main) {
+verify_attention_merge_span_kernel(const AttnParams p, int grid_main) {
     __shared__ long long s_red[2][kMergeThreads / 32];
     __shared__ int s_slots[2 * kMaxGrid];
     __shared__ int s_np;
@@ -834,50 +842,62 @@ verify_attention_merge_kernel(const AttnParams p, int grid_main) {
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (n_p <= 1) return;   // written whole by the main kernel
-    merge_row(p, s_slots, n_p, bl, h, blockIdx.z * kMergeRows + warp, lane);
+    merge_row<kMergePieces>(p, s_slots, n_p, bl, h, blockIdx.z * kMergeRows + warp, lane);
 }
 
-// grid (partial slot, 8-row chunk)
-__global__ void __launch_bounds__(kMergeThreads)
-verify_attention_merge_slots_kernel(const AttnParams p, int n_slots) {
+// grid (main-kernel CTA c, 8-row chunk)
+__global__ void __launch_bounds__(kMergeThreads, kMergePerSm)
+verify_attention_merge_cut_kernel(const AttnParams p, int n_slots) {
+    __shared__ int s_win[2 + kMergeWin];   // slots 2c-2 .. 2c+kMergeWin-1
     __shared__ int s_slots[2 * kMaxGrid];
-    __shared__ int s_win[kMergeBack + kMergeAhead];
-    __shared__ int s_np;
+    __shared__ int s_np, s_span;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // the slot list is the main kernel's output (see the other form on why
-    // every CTA waits)
+    // the slot list is the main kernel's output.  Every CTA waits, even one
+    // with nothing to merge, so that this grid never completes before the
+    // main kernel (a programmatic dependent of this kernel may rely on that),
+    // then lets the next kernel of the stream start.
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-    const int s0 = blockIdx.x;
-    const int w0 = s0 - kMergeBack;
-    if (threadIdx.x < kMergeBack + kMergeAhead) {
+    const int c = blockIdx.x, w0 = 2 * c - 2;
+    if (threadIdx.x < 2 + kMergeWin) {
         const int r = w0 + (int)threadIdx.x;
         s_win[threadIdx.x] = r >= 0 && r < n_slots ? __ldcg(&p.part_span[r]) : -1;
     }
     __syncthreads();
-    const int id = s_win[kMergeBack];
-    if (id < 0) return;
-    auto span_of = [&](int r) {
-        return r >= w0 && r - w0 < kMergeBack + kMergeAhead ? s_win[r - w0] : __ldcg(&p.part_span[r]);
-    };
     if (threadIdx.x == 0) {
-        // the first piece: the used slot before s0 belongs to another span
-        int q = s0 - 1;
-        while (q >= 0 && span_of(q) < 0) --q;
+        auto span_at = [&](int r) {
+            return r < 0 || r >= n_slots ? -1 : (r - w0 < 2 + kMergeWin ? s_win[r - w0] : __ldcg(&p.part_span[r]));
+        };
+        const int first = span_at(2 * c), last = span_at(2 * c + 1);
+        // the cut span that starts in CTA c, and its first slot
+        int id = -1, r0 = -1;
+        if (last >= 0) {
+            id = last;
+            r0 = 2 * c + 1;
+        } else if (first >= 0) {
+            const int prev = c > 0 ? (span_at(2 * c - 1) >= 0 ? span_at(2 * c - 1) : span_at(2 * c - 2)) : -1;
+            if (prev != first) {
+                id = first;
+                r0 = 2 * c;
+            }
+        }
         int n_p = 0;
-        if (q < 0 || span_of(q) != id) {
-            for (int r = s0; r < n_slots && n_p < 2 * kMaxGrid; ++r) {
-                const int v = span_of(r);
-                if (v == id) s_slots[n_p++] = r;
-                else if (v >= 0) break;
+        if (id >= 0) {
+            s_slots[n_p++] = r0;
+            // the following CTAs' first pieces, while the span goes on
+            for (int cc = c + 1; 2 * cc < n_slots && n_p < 2 * kMaxGrid; ++cc) {
+                if (span_at(2 * cc) != id) break;
+                s_slots[n_p++] = 2 * cc;
+                if (span_at(2 * cc + 1) >= 0) break;   // CTA cc has a later piece: the span ends here
             }
         }
         s_np = n_p;
+        s_span = id;
     }
     __syncthreads();
-    const int n_p = s_np;
-    if (n_p == 0) return;   // not a first piece
-    merge_row(p, s_slots, n_p, id / p.n_vh, id % p.n_vh, blockIdx.y * kMergeRows + warp, lane);
+    const int n_p = s_np, id = s_span;
+    if (n_p <= 1) return;   // no cut span starts here (a single piece cannot occur)
+    merge_row<kMergePiecesCut>(p, s_slots, n_p, id / p.n_vh, id % p.n_vh, blockIdx.y * kMergeRows + warp, lane);
 }
 
 #include "verify_attention_tc.cuh"
@@ -979,8 +999,8 @@ cudaError_t launch_dependent(void (*kern)(Params...), dim3 grid, dim3 block, siz
 
 // The split merge as a programmatic dependent of the main kernel: it may
 // start early and waits (griddepcontrol.wait) before it reads the partials.
-// The form with the smaller grid: per span (n_vh x requests) or per partial
-// slot (2 x the main grid).
+// The form with the smaller grid: per span (spans x 8-row chunks; few
+// requests) or per main-kernel CTA (main grid x 8-row chunks).
 cudaError_t launch_merge(const AttnParams& p, const AttnPlan& pl, cudaStream_t stream) {
     cudaLaunchAttribute attr;
     attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -991,12 +1011,12 @@ cudaError_t launch_merge(const AttnParams& p, const AttnPlan& pl, cudaStream_t s
     cfg.stream = stream;
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
-    if ((long long)p.n_vh * p.n_batch <= 2LL * pl.grid) {
+    if ((long long)p.n_vh * p.n_batch <= (long long)pl.grid) {
         cfg.gridDim = dim3(p.n_vh, p.n_batch, chunks);
-        return cudaLaunchKernelEx(&cfg, verify_attention_merge_kernel, p, (int)pl.grid);
+        return cudaLaunchKernelEx(&cfg, verify_attention_merge_span_kernel, p, (int)pl.grid);
     }
-    cfg.gridDim = dim3(2 * pl.grid, chunks, 1);
-    return cudaLaunchKernelEx(&cfg, verify_attention_merge_slots_kernel, p, 2 * (int)pl.grid);
+    cfg.gridDim = dim3((unsigned)pl.grid, chunks, 1);
+    return cudaLaunchKernelEx(&cfg, verify_attention_merge_cut_kernel, p, 2 * (int)pl.grid);
 }
 
 // Resident CTAs per SM of the kernel at a given block size (cached per device).
