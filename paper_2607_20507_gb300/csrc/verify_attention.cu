@@ -89,6 +89,7 @@ struct AttnParams {
     int tc_stages, tc_vstages;   // tcgen05 kernel: K and V ring depths
     int tc_q_half;               // tcgen05 kernel: bytes between query dim halves
     int b_base, n_batch;         // requests [b_base, b_base + n_batch) in this launch
+    int span_x;                  // work units charged to each span's start (see tiles_before)
     float scale_log2;            // sm_scale * log2(e)
 };
 
@@ -98,9 +99,42 @@ __device__ __forceinline__ void flag_timeout(int* status) {
 
 __device__ __forceinline__ int tiles_of(int L) { return max(1, (L + kTileT - 1) / kTileT); }
 
-// The CTA whose tile range holds flat tile f (ranges start at floor(c*W/G)).
-__device__ __forceinline__ int owner_of(long long f, long long W, int G) {
-    return (int)(((f + 1) * G + W - 1) / W) - 1;
+// The CTA whose range holds work unit v (ranges start at floor(c*U/G)).
+__device__ __forceinline__ int owner_of(long long v, long long U, int G) {
+    return (int)(((v + 1) * G + U - 1) / U) - 1;
+}
+
+// The work split.  Every span (request, KV head or row block) costs its T
+// tiles plus X units for starting it (query rows, epilogue: a CTA's time
+// grows with the span pieces it holds).  In the sequence of work units --
+// each span's X start units, then its T tiles -- CTA c of G takes units
+// [floor(c U / G), floor((c+1) U / G)) of U = W + X * n_vh * B, i.e. the
+// tiles whose unit index falls there.  tiles_before(v) counts the tiles
+// whose unit index is below v; request b's units start at
+// prefix[b] + X * n_vh * b (prefix: its first tile).
+__device__ __forceinline__ long long tiles_before(long long v, const long long* prefix, const int* lens,
+                                                  int n_batch, int n_vh, int X) {
+    if (v <= 0) return 0;
+    int lo = 0, hi = n_batch - 1;   // largest b whose units start at or below v
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (prefix[mid] + (long long)X * n_vh * mid <= v) lo = mid;
+        else hi = mid - 1;
+    }
+    const int T = tiles_of(lens[lo]);
+    const long long local = v - (prefix[lo] + (long long)X * n_vh * lo);
+    const int S = T + X;
+    // local < (n_vh + 1) * S: one 32-bit division whenever that fits
+    const long long h = local <= 0x7fffffffLL ? (long long)((unsigned)local / (unsigned)S) : local / S;
+    if (h >= n_vh) return prefix[lo] + (long long)n_vh * T;   // past the last unit
+    const long long tv = local - h * S;
+    return prefix[lo] + h * T + (tv > X ? tv - X : 0);
+}
+
+// floor(c * U / G) for the unit range of CTA c
+__device__ __forceinline__ long long unit_start(int c, long long U, int G) {
+    const long long n = (long long)c * U;
+    return n <= 0xffffffffLL ? (long long)((unsigned)n / (unsigned)G) : n / G;
 }
 
 // Position of flat tile f in the schedule: request (launch-local), head, tile.
@@ -259,7 +293,9 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
         p.part_span[2 * cta + 1] = -1;
     }
     if (cta >= Gc) return;
-    const long long f0 = (long long)cta * W / Gc, f1 = (long long)(cta + 1) * W / Gc;
+    const long long U = W + (long long)p.span_x * p.n_vh * nb;
+    const long long f0 = tiles_before(unit_start(cta, U, Gc), s_prefix, s_len, nb, p.n_vh, p.span_x);
+    const long long f1 = tiles_before(unit_start(cta + 1, U, Gc), s_prefix, s_len, nb, p.n_vh, p.span_x);
     if (f0 >= f1) return;
     const int n_tiles = (int)(f1 - f0);
     const uint32_t smem_base = smem_u32(smem);
@@ -663,7 +699,7 @@ verify_attention_kernel(const __grid_constant__ CUtensorMap tmap_k,
 // the weights, across the 128 dims for the sum).
 // Two ways to find a span's pieces, the launch taking the one with the
 // smaller grid:
-//  * per span: every CTA recomputes the main kernel's schedule from the
+//  * per span: every CTA recomputes the main kernel's work split from the
 //    context lengths (cheap for few requests, and done while the main
 //    kernel runs) and finds the CTAs that cut its span; a span with a single
 //    piece was written whole and is skipped;
@@ -820,16 +856,19 @@ verify_attention_merge_span_kernel(const AttnParams p, int grid_main) {
         const int T = tiles_of(L);
         const long long g_need = (W + kMinTilesPerCta - 1) / kMinTilesPerCta;
         const int Gc = (int)(g_need < (long long)grid_main ? (g_need > 0 ? g_need : 1) : grid_main);
-        const long long span0 = bf + (long long)h * T;
-        const int c_first = owner_of(span0, W, Gc);
-        const int c_last = owner_of(span0 + T - 1, W, Gc);
+        // in work units (tiles_before): the span's start units begin at vs,
+        // its tiles at vs + X; the CTA whose unit range holds its first tile
+        // holds it as its first piece unless that range starts before vs
+        // (unit vs - 1 is the previous span's last tile); every later owner
+        // holds it as its first piece
+        const int X = p.span_x;
+        const long long U = W + (long long)X * p.n_vh * nb;
+        const long long vs = bf + (long long)X * p.n_vh * bl + (long long)h * (T + X);
+        const int c_first = owner_of(vs + X, U, Gc);
+        const int c_last = owner_of(vs + X + T - 1, U, Gc);
         int n_p = 0;
-        long long start_c = (long long)c_first * W / Gc;
-        for (int cc = c_first; cc <= c_last && n_p < 2 * kMaxGrid; ++cc) {
-            const long long start_n = (long long)(cc + 1) * W / Gc;
-            if (start_n > start_c) s_slots[n_p++] = 2 * cc + ((cc == c_first && span0 > start_c) ? 1 : 0);
-            start_c = start_n;
-        }
+        for (int cc = c_first; cc <= c_last && n_p < 2 * kMaxGrid; ++cc)
+            s_slots[n_p++] = 2 * cc + ((cc == c_first && (long long)cc * U / Gc < vs) ? 1 : 0);
         s_np = n_p;
     }
     __syncthreads();
@@ -1163,6 +1202,10 @@ cs_status launch_verify_attention(const cs_attn_dims& d, const AttnPlan& pl, con
     p.n_rb = pl.n_rb;
     p.n_vh = d.n_kv_heads * pl.n_rb;
     p.n_rows_all = pl.n_rows_all;
+    // a span piece's own cost in tile units (clock stamps: ~1 tile's time at
+    // 35 rows, ~2.7 at 72 in the tcgen05 form)
+    p.span_x = pl.tc ? (pl.n_rows + 12) / 24 : 1;
+    if (p.span_x < 1) p.span_x = 1;
     const float scale = d.sm_scale > 0.f ? d.sm_scale : 1.0f / sqrtf((float)d.head_dim);
     p.scale_log2 = scale * 1.4426950408889634f;
 

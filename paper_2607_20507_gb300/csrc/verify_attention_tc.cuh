@@ -408,7 +408,9 @@ verify_attention_tc_kernel(const __grid_constant__ CUtensorMap tmap_k, const __g
     const long long g_need = (W + kMinTilesPerCta - 1) / kMinTilesPerCta;
     const int Gc = (int)(g_need < (long long)gridDim.x ? (g_need > 0 ? g_need : 1) : gridDim.x);
     const int cta = blockIdx.x;
-    long long f0 = (long long)cta * W / Gc, f1 = (long long)(cta + 1) * W / Gc;
+    const long long U = W + (long long)p.span_x * p.n_vh * nb;
+    long long f0 = tiles_before(unit_start(cta, U, Gc), s_prefix, s_len, nb, p.n_vh, p.span_x);
+    long long f1 = tiles_before(unit_start(cta + 1, U, Gc), s_prefix, s_len, nb, p.n_vh, p.span_x);
     if (cta >= Gc) f0 = f1 = 0;
     const int n_tiles = (int)(f1 - f0);
     // one dim half of a span's rows (trees: of its row block of q_nodes nodes)
