@@ -75,7 +75,7 @@ typedef struct {
     int32_t batch;              /* B >= 0 requests (0: nothing to do) */
     int32_t n_q_heads;          /* Hq > 0 query heads */
     int32_t n_kv_heads;         /* Hkv > 0 KV heads, Hq % Hkv == 0; G = Hq / Hkv */
-    int32_t head_dim;           /* D; this build implements D == 128 */
+    int32_t head_dim;           /* D; this library implements D == 128 */
     int32_t page_size;          /* ps tokens per page: 8, 16, 32, 64, 128 or 256 */
     int32_t max_pages_per_seq;  /* columns of page_table (> 0) */
     int32_t num_pages;          /* P pages in the pool (> 0) */

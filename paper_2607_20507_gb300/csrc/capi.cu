@@ -38,7 +38,7 @@ cs_status check_attn_geometry(const cs_attn_dims* d) {
     if (d->num_pages <= 0) return fail(CS_ERR_INVALID_ARG, "num_pages %d <= 0", d->num_pages);
     if (isnan(d->sm_scale) || isinf(d->sm_scale))
         return fail(CS_ERR_INVALID_ARG, "sm_scale is not finite");
-    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this build implements 128)", d->head_dim);
+    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this library implements 128)", d->head_dim);
     if (!pow2_page(d->page_size))
         return fail(CS_ERR_UNSUPPORTED, "page_size %d (supported: 8..256, powers of two)", d->page_size);
     if ((long long)d->max_pages_per_seq * d->page_size > (1LL << 30))
@@ -89,7 +89,7 @@ cs_status check_accept(const cs_accept_dims* d, int32_t n_draft, float temperatu
     if ((long long)d->batch * (n_draft + 1) * (long long)d->vocab > (1LL << 46))
         return fail(CS_ERR_INVALID_ARG, "logit tensor too large");
     if (d->vocab > CS_MAX_VOCAB)
-        return fail(CS_ERR_UNSUPPORTED, "vocab %d (this build implements up to %d)", d->vocab, CS_MAX_VOCAB);
+        return fail(CS_ERR_UNSUPPORTED, "vocab %d (this library implements up to %d)", d->vocab, CS_MAX_VOCAB);
     return CS_OK;
 }
 cs_status check_route(const cs_route_dims* d) {
@@ -112,7 +112,7 @@ cs_status check_sample(const cs_accept_dims* d, float temperature) {
     if ((long long)d->batch * (long long)d->vocab > (1LL << 46))
         return fail(CS_ERR_INVALID_ARG, "logit tensor too large");
     if (d->vocab > CS_MAX_VOCAB)
-        return fail(CS_ERR_UNSUPPORTED, "vocab %d (this build implements up to %d)", d->vocab, CS_MAX_VOCAB);
+        return fail(CS_ERR_UNSUPPORTED, "vocab %d (this library implements up to %d)", d->vocab, CS_MAX_VOCAB);
     return CS_OK;
 }
 }  // namespace
@@ -241,7 +241,7 @@ cs_status cs_kv_commit_tree(const cs_attn_dims* dims, void* k_pages, void* v_pag
     if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
     if (d->n_kv_heads <= 0 || d->page_size <= 0 || d->max_pages_per_seq <= 0 || d->num_pages <= 0)
         return fail(CS_ERR_INVALID_ARG, "n_kv_heads, page_size, max_pages_per_seq and num_pages must be positive");
-    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this build implements 128)", d->head_dim);
+    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this library implements 128)", d->head_dim);
     if (n_nodes < 1 || n_nodes > CS_MAX_TREE_NODES)
         return fail(CS_ERR_INVALID_ARG, "n_nodes %d not in [1, %d]", n_nodes, CS_MAX_TREE_NODES);
     if ((long long)d->max_pages_per_seq * d->page_size > (1LL << 30))
@@ -297,7 +297,7 @@ cs_status cs_kv_append(const cs_attn_dims* dims, const void* new_k, const void* 
     if (d->batch < 0) return fail(CS_ERR_INVALID_ARG, "batch %d < 0", d->batch);
     if (d->n_kv_heads <= 0 || d->page_size <= 0 || d->max_pages_per_seq <= 0 || d->num_pages <= 0)
         return fail(CS_ERR_INVALID_ARG, "n_kv_heads, page_size, max_pages_per_seq and num_pages must be positive");
-    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this build implements 128)", d->head_dim);
+    if (d->head_dim != 128) return fail(CS_ERR_UNSUPPORTED, "head_dim %d (this library implements 128)", d->head_dim);
     if (n_new < 1 || n_new > 4096) return fail(CS_ERR_INVALID_ARG, "n_new %d not in [1, 4096]", n_new);
     if ((long long)d->max_pages_per_seq * d->page_size > (1LL << 30))
         return fail(CS_ERR_INVALID_ARG, "max_pages_per_seq * page_size exceeds 2^30 keys");

@@ -97,7 +97,7 @@ SWEEP_SIGMAS = (0.1, 0.5, 1.0, 2.0, 4.0)
 SWEEP_KS = (1, 2, 4, 8, 16)
 SWEEP_BATCHES = (1, 8, 64, 256, 512)
 SWEEP_VOCABS = (32000, 128256, 256000)
-SWEEP_TEMPERATURE = 1.0   # the sweep states no temperature; 1.0 is this build's reading
+SWEEP_TEMPERATURE = 1.0   # the sweep states no temperature; 1.0 is the reading taken here
 
 
 def sweep_accept_cells():
