@@ -134,12 +134,12 @@ const char* cs_last_error(void);
  * (L_b-(k+1)+i < 0) outputs zeros; a page id outside [0, P) reads as zeros.
  * Pool slots past L_b may hold any bits (including NaN); they never reach
  * the output.  Arithmetic: S = q.K in bf16 with fp32 accumulation, the
- * softmax in fp32, and the P.V product in fp16 with fp32 accumulation (P
- * rounded to fp16; V converted from bf16, exact for |v| <= 65280).  From the
- * first tile whose V holds an entry fp16 cannot (|v| >= 65536, up to bf16's
- * largest value) to the end of that span piece, P.V runs in bf16 with P
- * scaled by 2^-64, so that no partial sum overflows fp32: every finite bf16
- * V gives a finite output within the stated tolerance.
+ * softmax in fp32, and the P.V product on bf16 V as stored, with P taken as
+ * the sum of two bf16 terms (hi = bf16(P), lo = bf16(P - hi): ~16
+ * significant bits) and fp32 accumulation.  P is formed scaled by 2^-64 (the
+ * row sum carries the same factor), so that no partial sum of P.V overflows
+ * fp32: every finite bf16 V, up to bf16's largest value, gives a finite
+ * output within the stated tolerance.
  *
  * Returns CS_ERR_INVALID_ARG (null pointer, misalignment, bad dimension, NaN
  * scale, n_draft out of range), CS_ERR_UNSUPPORTED (D != 128, page size,
