@@ -5,9 +5,9 @@
 // Schedule (persistent, balanced).  The work is the flattened sequence of
 // 64-key tiles of every (request b, KV head h) span, requests in order, heads
 // in order, tiles in key order; span (b, h) has T_b = ceil(L_b / 64) tiles.
-// The grid holds exactly as many CTAs as are resident at once, and CTA c
-// takes the contiguous tile range [c*W/G, (c+1)*W/G) of the W tiles, so every
-// CTA streams the same number of tiles whatever the context lengths.  A span
+// The grid holds exactly as many CTAs as are resident at once; each span also
+// costs a few work units for its start, and CTA c takes the tiles of units
+// [cU/G, (c+1)U/G) (tiles_before below), so the CTAs' work evens out.  A span
 // that lies inside one CTA's range is finished there and written in bf16;
 // a span cut by range boundaries leaves one partial per piece -- the piece's
 // own normalised output and its (m, l) -- (each CTA writes at most two: its
