@@ -8,7 +8,7 @@
 // token tree with more rows comes in row blocks of whole nodes, at most 128
 // rows each; each block is a span of its own (reading the request's keys
 // again) whose query box starts at the block's first node.
-// Same persistent schedule (equal contiguous tile ranges, spans, two partial
+// Same persistent schedule (contiguous ranges of equal work, spans, two partial
 // slots per CTA, merge kernel), one CTA per SM, twelve warps.  Each SMSP
 // (warp % 4) runs one role warp and up to two softmax warps; the live
 // softmax warps fill SMSPs 0 and 1 first, so the two producers sit on SMSPs
