@@ -907,8 +907,6 @@ template <typename T>
 __device__ __forceinline__ float cluster_mass(const DrawRow<T>& d, bool residual, int c0, int c1, int n_pass,
                                               uint32_t n_ranks, float (&s_wsum)[kDrawWarps],
                                               int (&s_wlast)[kDrawWarps], float2* s_x, int& xr) {
-    constexpr int kRun = kRunVecs * 16 / (int)sizeof(T);
-    constexpr int kPass = kDrawThreads * kRun;
     __shared__ float s_tpass[kMaxPasses];
     const float mass = slice_passes<T>(d, residual, c0, c1, n_pass, s_tpass, s_wlast).mass;
     (void)s_wsum;
