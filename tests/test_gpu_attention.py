@@ -250,3 +250,12 @@ def test_tcgen05_unaligned_query_falls_back():
                                       inp["n_draft"])
     torch.cuda.synchronize()
     assert_parity(out, ref(inp), "tc fallback")
+
+
+@pytest.mark.parametrize("k,Hq,Hkv", [(2, 8, 2), (4, 16, 2)])
+def test_batch_beyond_one_launch(k, Hq, Hkv):
+    # more requests than one launch schedules (1024): the call runs two main
+    # kernels (and merges) over the same workspace, the second on requests
+    # 1024.. -- both attention forms (12 and 40 query rows per KV head)
+    inp = W.attention_inputs(small(B=1030, k=k, Hq=Hq, Hkv=Hkv, lo=k + 1, hi=160, cell=7000 + k), DEV)
+    assert_parity(gpu(inp), ref(inp), f"B=1030 k={k} G={Hq // Hkv}")
